@@ -1,0 +1,222 @@
+/*
+ * fgq.h -- C ABI of libfgq, a GB300 (sm_103a) implementation of the data-parallel hot
+ * path of Fine-Grained Quantization (FGQ), "Ternary Neural Networks with Fine-Grained
+ * Quantization" (arXiv 1705.01462).
+ *
+ * The hot path: each output filter's weights are split into groups of G consecutive
+ * weights along the reduction axis (Section 3.1, Eq. 2; Section 3.2 groups along the
+ * input channels), each group is ternarized to codes t in {-1, 0, +1} with one fp32
+ * scale alpha (Eq. 5; Eq. 4 reaches the same optimum), activations are quantized to
+ * 8 or 4 bit dynamic fixed point (Section 4), and a convolution or fully connected layer
+ * computes  y = s_x * sum_g alpha_g * (sum_{j in g} t_j * q_j)  with the inner sums held
+ * in 32-bit integer accumulators (Section 4): one multiply per group instead of one per
+ * weight (Section 4.1).
+ *
+ * Conventions for every call
+ *   - All array pointers are DEVICE pointers owned by the caller; the library allocates
+ *     nothing.  Calls are asynchronous and ordered on the given CUDA stream.
+ *   - The return value reports errors found on the host (argument, alignment, unsupported
+ *     shape, CUDA launch failure).  Errors found by a kernel (non-finite input, a bounded
+ *     wait that ran out) are recorded in a device error word and returned by
+ *     fgq_stream_status().
+ *   - Shapes are int; products of shapes are computed in 64 bits.  Empty problems
+ *     (M, P, n or B equal to 0) are valid and launch nothing.
+ *
+ * Data layouts
+ *   Kred        reduction length.  Convolution: Kred = R*S*(C/groups), ordered (r, s, c)
+ *               with c fastest (torch OIHW weights permuted to OHWI).
+ *   Kp          ceil(Kred/G)*G, the row length padded with zero weights.
+ *   ng          Kp/G groups per filter.
+ *   codes       uint32 [M][ceil(Kp/16)].  Code of t: 0 -> 00, +1 -> 01, -1 -> 11 (10 is
+ *               never written); element j of a row sits in word j/16, bits 2(j%16) and
+ *               2(j%16)+1.  Unused bits are 0.  (This 2-bit encoding is the library's
+ *               choice; the paper only states 2-bit weights, Section 4.)
+ *   alpha       fp32 [M][ng].
+ *   activations 8-bit types: one byte per element.  4-bit types: element 2i in the low
+ *               nibble of byte i, 2i+1 in the high nibble (two's complement for S4).
+ *               Convolution inputs are NHWC [B][H][W][C] (C even for 4-bit types); GEMM
+ *               inputs are [P][Kred] (Kred even for 4-bit types).
+ *   outputs     fp32 NHWC [B][Ho][Wo][M] (convolution), [P][M] (GEMM),
+ *               Ho = (H + 2*pad - R)/stride + 1, Wo likewise.
+ */
+#ifndef FGQ_H_
+#define FGQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FGQ_OK = 0,
+  FGQ_ERR_ARG = 1,          /* invalid argument: null pointer, negative size, bad G ... */
+  FGQ_ERR_ALIGN = 2,        /* a pointer is not 16-byte aligned */
+  FGQ_ERR_UNSUPPORTED = 3,  /* valid but unsupported combination (stated per call) */
+  FGQ_ERR_NONFINITE = 4,    /* a kernel saw NaN or Inf in its fp32 input */
+  FGQ_ERR_TIMEOUT = 5,      /* a kernel's bounded wait ran out; the kernel returned early */
+  FGQ_ERR_CUDA = 6          /* a CUDA runtime call or a launch failed */
+} fgq_status;
+
+typedef enum { FGQ_U8 = 0, FGQ_S8 = 1, FGQ_U4 = 2, FGQ_S4 = 3 } fgq_act_type;
+
+/* Contraction kernel families (see fgq_set_path / fgq_last_path). */
+typedef enum {
+  FGQ_PATH_AUTO = 0,   /* choose per shape */
+  FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
+  FGQ_PATH_TC = 2      /* tensor-core path (tcgen05), K-tile aligned to the group */
+} fgq_path;
+
+/* ABI version of this header (incremented on any signature change). */
+int fgq_version(void);
+
+/* Human-readable name of a status code (static string). */
+const char* fgq_status_string(fgq_status s);
+
+/* Number of uint32 code words per filter row: ceil(ceil(Kred/G)*G / 16); 0 on bad input. */
+int64_t fgq_codes_words_per_row(int Kred, int G);
+
+/* Number of groups per filter row, ceil(Kred/G); 0 on bad input. */
+int64_t fgq_num_groups(int Kred, int G);
+
+/*
+ * FGQ ternarization (Section 3.1, Eq. 2 and Eq. 5, solved exactly per group -- the
+ * paper's "brute-force" per-group solve, Section 4).
+ *   w      fp32 [M][Kred] row-major, Kred in (r, s, c) order.
+ *   G      group size, one of 1, 2, 4, 8, 16, 32, 64, 128.
+ *   codes  out, uint32 [M][fgq_codes_words_per_row(Kred, G)], fully written.
+ *   alpha  out, fp32 [M][fgq_num_groups(Kred, G)].
+ * Per group: the kept set is {j : |w_j| >= tau} for the threshold tau maximising
+ * (sum of kept |w|)^2 / (number kept), ties to the larger tau; alpha is the fp32 nearest
+ * (ties to even) the exact mean of the kept |w|; t_j = sign(w_j) on the kept set.  An
+ * all-zero group gives alpha = 0 and zero codes.  Decisions use exact integer arithmetic,
+ * so results are bit-reproducible.  A group holding NaN/Inf gets zero codes and alpha,
+ * and FGQ_ERR_NONFINITE is recorded.
+ * Errors: FGQ_ERR_ARG (null pointer with M*Kred > 0, negative sizes, bad G),
+ * FGQ_ERR_ALIGN (w, codes or alpha not 4-byte aligned), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
+                         cudaStream_t stream);
+
+/* Bytes of device workspace fgq_quantize_act needs for n elements (0 when n == 0). */
+size_t fgq_quantize_act_workspace_bytes(size_t n);
+
+/*
+ * Dynamic-fixed-point activation quantization (Section 4: activations quantized to 8 or
+ * 4 bits before each convolution, one shared exponent per tensor).
+ *   x          fp32 [n].
+ *   type       FGQ_U8 / FGQ_S8 / FGQ_U4 / FGQ_S4; qmax = 255 / 127 / 15 / 7, qmin = 0 /
+ *              -128 / 0 / -8.
+ *   scale_in   > 0: use this scale (must be a power of two, else FGQ_ERR_ARG); <= 0: derive
+ *              it: E = smallest integer with max * 2^-E <= qmax (max = max|x|, or max(x, 0)
+ *              for unsigned types), E = 0 when max = 0, E clamped to [-149, 127].
+ *   q          out, n bytes (8-bit) or ceil(n/2) bytes (4-bit; an odd tail's high nibble
+ *              is 0).
+ *   scale_out  out, device fp32 [1]: 2^E.  May be NULL when scale_in > 0.
+ *   workspace  device scratch of fgq_quantize_act_workspace_bytes(n) bytes (ignored when
+ *              scale_in > 0); its contents on entry do not matter.
+ * q_i = clamp(round_half_even(x_i * 2^-E), qmin, qmax), exact.  Two kernels when the scale
+ * is derived (max reduction, then quantization); one when it is given.
+ * Errors: FGQ_ERR_ARG, FGQ_ERR_ALIGN (x, q not 4-byte aligned; workspace not 4-byte
+ * aligned or too small), FGQ_ERR_CUDA; NaN/Inf recorded as FGQ_ERR_NONFINITE.
+ */
+fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float scale_in, void* q,
+                            float* scale_out, void* workspace, size_t workspace_bytes,
+                            cudaStream_t stream);
+
+/*
+ * 8-bit weights for the first layer (Section 4: the first layer is kept at 8w-8a): each
+ * filter row of w fp32 [M][Kred] is quantized as a signed 8-bit DFP vector, the same rule
+ * as fgq_quantize_act with FGQ_S8 applied per row.  wq out int8 [M][Kred]; wscale out fp32
+ * [M] (2^E per row).  Errors as fgq_ternarize.
+ */
+fgq_status fgq_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
+                                   cudaStream_t stream);
+
+/*
+ * Grouped ternary GEMM (fully connected layer, Eq. 2 with 32-bit group accumulators,
+ * Section 4):  y[p][m] = act_scale[0] * sum_g alpha[m][g] * s[m][g][p],
+ *              s[m][g][p] = sum_{j in g} t[m][j] * q[p][j]   (exact int32).
+ *   q          activations [P][Kred] of the given type.
+ *   act_scale  device fp32 [1] (e.g. the scale_out of fgq_quantize_act).
+ *   codes, alpha as produced by fgq_ternarize for (M, Kred, G).
+ *   y          out, fp32 [P][M].
+ * The fp32 result is within 1e-5 * act_scale * sum_g |alpha_g * s_g| of the exact value.
+ * Errors: FGQ_ERR_ARG (null pointers, bad sizes, Kred odd for 4-bit types),
+ * FGQ_ERR_ALIGN (any pointer not 16-byte aligned), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_gemm(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                    const uint32_t* codes, const float* alpha, int M, int G, float* y,
+                    cudaStream_t stream);
+
+/*
+ * Grouped ternary convolution as an implicit GEMM (Section 3.2 grouping along the input
+ * channels, Eq. 2, Section 4):  out[b][ho][wo][m] = act_scale[0] * sum_g alpha[m][g] *
+ * s[m][g][b,ho,wo], where the group sums run over the im2col column of (b, ho, wo):
+ * element (r, s, c) is act[b][ho*stride-pad+r][wo*stride-pad+s][gi*C/groups + c], zero
+ * outside the image, gi = the conv group of filter m (m / (M/groups)).
+ *   act        NHWC [B][H][W][C] of the given type.
+ *   codes, alpha  from fgq_ternarize with Kred = R*S*(C/groups).
+ *   groups     convolution channel groups (C and M divisible by it); unrelated to G.
+ *   out        fp32 NHWC [B][Ho][Wo][M].
+ * Tolerance and errors as fgq_gemm (C odd for 4-bit types is FGQ_ERR_ARG).
+ */
+fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale, int B, int H,
+                      int W, int C, int R, int S, int stride, int pad, int groups,
+                      const uint32_t* codes, const float* alpha, int M, int G, float* out,
+                      cudaStream_t stream);
+
+/*
+ * Dense 8-bit-weight convolution for the first layer (8w-8a, Section 4):
+ *   out = act_scale[0] * wscale[m] * sum_j wq[m][j] * col[j]   (exact int32 dot product).
+ *   wq int8 [M][Kred], wscale fp32 [M] (as from fgq_quantize_weights_w8).  Other arguments
+ *   as fgq_conv2d.  Errors as fgq_conv2d.
+ */
+fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_scale, int B,
+                         int H, int W, int C, int R, int S, int stride, int pad, int groups,
+                         const int8_t* wq, const float* wscale, int M, float* out,
+                         cudaStream_t stream);
+
+/*
+ * The 32-bit group accumulators themselves (Section 4), for verification:
+ *   s[m][g][p] = sum_{j in g, j < Kred} t[m][j] * q[p][j],  int32 [M][ng][P].
+ * q as in fgq_gemm.  Errors as fgq_gemm.
+ */
+fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred,
+                          const uint32_t* codes, int M, int G, int32_t* s, cudaStream_t stream);
+
+/*
+ * Synchronizes the stream, then returns (and clears) the first error a kernel recorded
+ * since the last call (FGQ_OK if none), or FGQ_ERR_CUDA if the synchronization failed.
+ */
+fgq_status fgq_stream_status(cudaStream_t stream);
+
+/*
+ * Restricts contraction calls to one kernel family (FGQ_PATH_AUTO restores the default
+ * per-shape choice).  A forced path that cannot run a shape makes the call return
+ * FGQ_ERR_UNSUPPORTED.  Process-wide; returns the previous setting.
+ */
+int fgq_set_path(int path);
+
+/* The kernel family (fgq_path) the most recent contraction call on this host thread used. */
+int fgq_last_path(void);
+
+/* Number of kernels this library has launched in this process (all calls, all threads). */
+uint64_t fgq_launch_count(void);
+
+/*
+ * Failure-detection self test: launches one block that waits, with an iteration limit,
+ * on an mbarrier that nothing arrives on, and records FGQ_ERR_TIMEOUT when the limit
+ * runs out.  Read the result with fgq_stream_status().  Paper counterpart: none (library
+ * health check).
+ */
+fgq_status fgq_selftest_wait_timeout(uint32_t max_iterations, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FGQ_H_ */

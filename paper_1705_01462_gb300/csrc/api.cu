@@ -1,0 +1,258 @@
+// libfgq C ABI: argument validation, kernel-family dispatch, the device error word and
+// status reporting.  Every computation happens in the kernels of the other files.
+#include <atomic>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "fgq_internal.h"
+
+namespace fgq {
+namespace {
+
+__device__ unsigned int g_error_word;
+
+constexpr int kMaxDevices = 64;
+unsigned int* g_err_ptr[kMaxDevices];
+std::mutex g_err_mu;
+std::atomic<uint64_t> g_launches{0};
+std::atomic<int> g_path{FGQ_PATH_AUTO};
+thread_local int t_last_path = FGQ_PATH_AUTO;
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool valid_type(int t) { return t == FGQ_U8 || t == FGQ_S8 || t == FGQ_U4 || t == FGQ_S4; }
+
+bool valid_G(int G) {
+  return G == 1 || G == 2 || G == 4 || G == 8 || G == 16 || G == 32 || G == 64 || G == 128;
+}
+
+bool is4(int t) { return t == FGQ_U4 || t == FGQ_S4; }
+
+// Fill a Geom for a convolution; returns FGQ_OK or FGQ_ERR_ARG.
+fgq_status make_geom(int type, int B, int H, int W, int C, int R, int S, int stride, int pad, int groups,
+                     int M, int G, int is_conv, Geom& g) {
+  if (!valid_type(type) || B < 0 || H <= 0 || W <= 0 || C <= 0 || R <= 0 || S <= 0 || stride <= 0 ||
+      pad < 0 || groups <= 0 || M < 0 || C % groups != 0 || M % groups != 0 || G <= 0)
+    return FGQ_ERR_ARG;
+  if (is4(type) && (C % 2 != 0)) return FGQ_ERR_ARG;
+  g.B = B; g.H = H; g.W = W; g.C = C; g.R = R; g.S = S; g.stride = stride; g.pad = pad; g.groups = groups;
+  g.Ho = (H + 2 * pad - R) / stride + 1;
+  g.Wo = (W + 2 * pad - S) / stride + 1;
+  if (H + 2 * pad < R || W + 2 * pad < S || g.Ho <= 0 || g.Wo <= 0) return FGQ_ERR_ARG;
+  g.Cg = C / groups;
+  g.Kred = R * S * g.Cg;
+  g.G = G;
+  g.ng = (g.Kred + G - 1) / G;
+  g.Kp = g.ng * G;
+  g.wrow = (g.Kp + 15) / 16;
+  g.M = M;
+  g.Mg = groups ? M / groups : 0;
+  g.act_type = type;
+  g.is_conv = is_conv;
+  g.P = (int64_t)B * g.Ho * g.Wo;
+  return FGQ_OK;
+}
+
+int choose_path(const Geom& g) {
+  const int forced = g_path.load();
+  if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
+  if (forced == FGQ_PATH_TC) return tc_supports(g) ? FGQ_PATH_TC : -1;
+  return tc_supports(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
+}
+
+fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
+                    const float* act_scale, float* out, int32_t* sums, cudaStream_t s) {
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  const int path = choose_path(g);
+  if (path < 0) return FGQ_ERR_UNSUPPORTED;
+  t_last_path = path;
+  unsigned int* err = device_error_word();
+  if (path == FGQ_PATH_TC) return launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
+  return launch_simt_contract(act, g, codes, alpha, 0, act_scale, out, sums, s);
+}
+
+}  // namespace
+
+unsigned int* device_error_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(g_err_mu);
+  if (!g_err_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+    g_err_ptr[dev] = static_cast<unsigned int*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+fgq_status after_launch() {
+  g_launches.fetch_add(1);
+  return cudaGetLastError() == cudaSuccess ? FGQ_OK : FGQ_ERR_CUDA;
+}
+
+}  // namespace fgq
+
+using namespace fgq;
+
+extern "C" {
+
+int fgq_version(void) { return 1; }
+
+const char* fgq_status_string(fgq_status s) {
+  switch (s) {
+    case FGQ_OK: return "FGQ_OK";
+    case FGQ_ERR_ARG: return "FGQ_ERR_ARG: invalid argument";
+    case FGQ_ERR_ALIGN: return "FGQ_ERR_ALIGN: misaligned pointer";
+    case FGQ_ERR_UNSUPPORTED: return "FGQ_ERR_UNSUPPORTED: unsupported shape or path";
+    case FGQ_ERR_NONFINITE: return "FGQ_ERR_NONFINITE: NaN or Inf in input";
+    case FGQ_ERR_TIMEOUT: return "FGQ_ERR_TIMEOUT: a bounded wait ran out";
+    case FGQ_ERR_CUDA: return "FGQ_ERR_CUDA: CUDA error";
+  }
+  return "unknown fgq_status";
+}
+
+int64_t fgq_codes_words_per_row(int Kred, int G) {
+  if (Kred < 0 || !valid_G(G)) return 0;
+  const int64_t ng = ((int64_t)Kred + G - 1) / G;
+  return (ng * G + 15) / 16;
+}
+
+int64_t fgq_num_groups(int Kred, int G) {
+  if (Kred < 0 || !valid_G(G)) return 0;
+  return ((int64_t)Kred + G - 1) / G;
+}
+
+fgq_status fgq_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
+                         cudaStream_t stream) {
+  if (M < 0 || Kred < 0 || !valid_G(G)) return FGQ_ERR_ARG;
+  if ((int64_t)M * Kred == 0) return FGQ_OK;
+  if (!w || !codes || !alpha) return FGQ_ERR_ARG;
+  if (!aligned(w, 4) || !aligned(codes, 4) || !aligned(alpha, 4)) return FGQ_ERR_ALIGN;
+  if ((int64_t)Kred + G > INT32_MAX) return FGQ_ERR_ARG;
+  return launch_ternarize(w, M, Kred, G, codes, alpha, device_error_word(), stream);
+}
+
+size_t fgq_quantize_act_workspace_bytes(size_t n) { return quantize_workspace_bytes(n); }
+
+fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float scale_in, void* q,
+                            float* scale_out, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  if (!valid_type(type)) return FGQ_ERR_ARG;
+  int E = 0;
+  const bool derive = !(scale_in > 0.0f);
+  if (!derive) {  // the given scale must be a power of two 2^E (subnormal ones included)
+    uint32_t b;
+    memcpy(&b, &scale_in, sizeof b);
+    const uint32_t ex = b >> 23, man = b & 0x7fffffu;
+    if (ex == 255) return FGQ_ERR_ARG;
+    if (ex > 0) {
+      if (man != 0) return FGQ_ERR_ARG;
+      E = (int)ex - 127;
+    } else {
+      if (man & (man - 1)) return FGQ_ERR_ARG;
+      E = -149 + (31 - __builtin_clz(man));
+    }
+  }
+  if (n == 0) return FGQ_OK;  // nothing is written
+  if (!x || !q || (derive && (!scale_out || !workspace))) return FGQ_ERR_ARG;
+  if (!aligned(x, 16) || !aligned(q, 16) || (scale_out && !aligned(scale_out, 4))) return FGQ_ERR_ALIGN;
+  if (derive) {
+    if (!aligned(workspace, 4)) return FGQ_ERR_ALIGN;
+    if (workspace_bytes < quantize_workspace_bytes(n)) return FGQ_ERR_ARG;
+  }
+  return launch_quantize(x, n, type, E, derive, q, scale_out, static_cast<uint32_t*>(workspace),
+                         device_error_word(), stream);
+}
+
+fgq_status fgq_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
+                                   cudaStream_t stream) {
+  if (M < 0 || Kred < 0) return FGQ_ERR_ARG;
+  if ((int64_t)M * Kred == 0) return FGQ_OK;
+  if (!w || !wq || !wscale) return FGQ_ERR_ARG;
+  if (!aligned(w, 4) || !aligned(wscale, 4)) return FGQ_ERR_ALIGN;
+  return launch_quantize_weights_w8(w, M, Kred, wq, wscale, device_error_word(), stream);
+}
+
+fgq_status fgq_gemm(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                    const uint32_t* codes, const float* alpha, int M, int G, float* y, cudaStream_t stream) {
+  if (!valid_G(G) || P < 0 || Kred <= 0 || M < 0) return FGQ_ERR_ARG;
+  if (is4(type) && Kred % 2) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, P, 1, 1, Kred, 1, 1, 1, 0, 1, M, G, 0, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!q || !act_scale || !codes || !alpha || !y) return FGQ_ERR_ARG;
+  if (!aligned(q, 16) || !aligned(codes, 16) || !aligned(alpha, 16) || !aligned(y, 16) || !aligned(act_scale, 4))
+    return FGQ_ERR_ALIGN;
+  return contract(q, g, codes, alpha, act_scale, y, nullptr, stream);
+}
+
+fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
+                      int R, int S, int stride, int pad, int groups, const uint32_t* codes, const float* alpha,
+                      int M, int G, float* out, cudaStream_t stream) {
+  if (!valid_G(G)) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !act_scale || !codes || !alpha || !out) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(codes, 16) || !aligned(alpha, 16) || !aligned(out, 16) ||
+      !aligned(act_scale, 4))
+    return FGQ_ERR_ALIGN;
+  return contract(act, g, codes, alpha, act_scale, out, nullptr, stream);
+}
+
+fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
+                         int R, int S, int stride, int pad, int groups, const int8_t* wq, const float* wscale,
+                         int M, float* out, cudaStream_t stream) {
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, 4, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !act_scale || !wq || !wscale || !out) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(wscale, 4) || !aligned(out, 16) || !aligned(act_scale, 4))
+    return FGQ_ERR_ALIGN;
+  t_last_path = FGQ_PATH_SIMT;
+  return launch_simt_contract(act, g, wq, wscale, 1, act_scale, out, nullptr, stream);
+}
+
+fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred, const uint32_t* codes, int M, int G,
+                          int32_t* s, cudaStream_t stream) {
+  if (!valid_G(G) || P < 0 || Kred <= 0 || M < 0) return FGQ_ERR_ARG;
+  if (is4(type) && Kred % 2) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, P, 1, 1, Kred, 1, 1, 1, 0, 1, M, G, 0, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!q || !codes || !s) return FGQ_ERR_ARG;
+  if (!aligned(q, 16) || !aligned(codes, 16) || !aligned(s, 4)) return FGQ_ERR_ALIGN;
+  return contract(q, g, codes, nullptr, nullptr, nullptr, s, stream);
+}
+
+fgq_status fgq_stream_status(cudaStream_t stream) {
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return FGQ_ERR_CUDA;
+  unsigned int* e = device_error_word();
+  if (!e) return FGQ_ERR_CUDA;
+  unsigned int v = 0;
+  if (cudaMemcpy(&v, e, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return FGQ_ERR_CUDA;
+  if (v != 0) {
+    const unsigned int zero = 0;
+    if (cudaMemcpy(e, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return FGQ_ERR_CUDA;
+  }
+  return (fgq_status)v;
+}
+
+int fgq_set_path(int path) {
+  if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC) return -1;
+  return g_path.exchange(path);
+}
+
+int fgq_last_path(void) { return t_last_path; }
+
+uint64_t fgq_launch_count(void) { return g_launches.load(); }
+
+fgq_status fgq_selftest_wait_timeout(uint32_t max_iterations, cudaStream_t stream) {
+  return launch_wait_timeout_selftest(max_iterations, device_error_word(), stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,54 @@
+// Internal declarations shared by the libfgq translation units (not part of the ABI).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime_api.h>
+
+#include "../../include/fgq.h"
+
+namespace fgq {
+
+// Geometry of one contraction call.  A GEMM is the convolution with B = P, H = W = 1,
+// R = S = 1, C = Kred, stride 1, pad 0, groups 1.
+struct Geom {
+  int B, H, W, C, R, S, stride, pad, groups;
+  int Ho, Wo, Cg, Kred, Kp, ng, M, Mg, G, wrow;
+  int act_type;  // fgq_act_type
+  int is_conv;
+  int64_t P;     // B * Ho * Wo
+};
+
+// Device error word of the current device (first error wins; cleared by
+// fgq_stream_status).  Returns nullptr if the symbol address cannot be obtained.
+unsigned int* device_error_word();
+
+// Counts one kernel launch (for fgq_launch_count) and converts a launch error.
+fgq_status after_launch();
+
+// Kernel launchers (each returns FGQ_OK or FGQ_ERR_CUDA / FGQ_ERR_UNSUPPORTED).
+fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
+                            unsigned int* err, cudaStream_t s);
+fgq_status launch_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
+                                      unsigned int* err, cudaStream_t s);
+size_t quantize_workspace_bytes(size_t n);
+fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool derive, void* q,
+                           float* scale_out, uint32_t* partials, unsigned int* err, cudaStream_t s);
+
+// CUDA-core contraction (dp4a).  codes/alpha for ternary weights, or wq/wscale for dense
+// 8-bit weights (dense != 0).  sums != nullptr writes the int32 group sums [M][ng][P]
+// instead of the fp32 output.
+fgq_status launch_simt_contract(const void* act, const Geom& g, const void* weights,
+                                const float* scales, int dense, const float* act_scale, float* out,
+                                int32_t* sums, cudaStream_t s);
+// Tensor-core contraction (tcgen05), G in {64, 128}; returns FGQ_ERR_UNSUPPORTED for shapes
+// it does not cover.
+bool tc_supports(const Geom& g);
+fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* codes,
+                              const float* alpha, const float* act_scale, float* out,
+                              int32_t* sums, unsigned int* err, cudaStream_t s);
+
+fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
+
+}  // namespace fgq

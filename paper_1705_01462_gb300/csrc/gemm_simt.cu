@@ -1,0 +1,354 @@
+// CUDA-core grouped ternary contraction (Eq. 2 on a convolution or fully connected layer,
+// 32-bit group accumulators of Section 4, one multiply per group as counted in Section 4.1).
+//
+// For each group of G weights (G a multiple of 4) the int32 group sum is a chain of G/4
+// dp4a instructions over int8x4 activation words and int8x4 code words expanded from the
+// 2-bit codes; the sum is then scaled by alpha into an fp32 accumulator.  The dp4a chain
+// starts at the bit pattern of 1.5*2^23, so its int32 result reads directly as the fp32
+// number 1.5*2^23 + s and one packed fp32x2 add recovers s exactly (no int->fp32
+// conversion instruction).  The group-scaled partials are accumulated with packed fp32x2
+// FMAs: per (filter, position, group) one dp4a per 4 weights plus one add and one FMA.
+//
+// Tiling: a 256-thread block computes 64 filters x 128 output positions; each thread owns
+// 4 filters x 8 positions.  The reduction axis is staged through shared memory in chunks
+// of max(16, G/4) words: activation words gathered from the implicit im2col (zero outside
+// the image), code words expanded through a 256-entry byte table, and the chunk's alphas.
+//
+// The same kernel runs the dense 8-bit-weight first layer (int32 dot product over the
+// whole row, scaled once at the end) and can write the raw int32 group sums.
+#include <cstdint>
+
+#include "fgq_device.cuh"
+
+namespace fgq {
+namespace {
+
+constexpr int BM = 64;    // filters per block
+constexpr int BP = 128;   // positions per block
+constexpr int NT = 256;   // threads per block
+
+// Per-thread view of one output position for the im2col gather.
+struct PosInfo {
+  int valid;
+  int b, hb, wb;  // image, and the input row/col of tap (0, 0): ho*stride - pad, wo*stride - pad
+};
+
+__device__ __forceinline__ PosInfo pos_info(const Geom& g, int64_t p) {
+  PosInfo pi;
+  pi.valid = p < g.P;
+  if (!pi.valid) p = 0;
+  const int wo = (int)(p % g.Wo);
+  const int64_t t = p / g.Wo;
+  const int ho = (int)(t % g.Ho);
+  pi.b = (int)(t / g.Ho);
+  pi.hb = ho * g.stride - g.pad;
+  pi.wb = wo * g.stride - g.pad;
+  return pi;
+}
+
+// Element offset of reduction index k (k < Kred) for position pi in conv group gi, or -1
+// if it falls in the zero padding.
+__device__ __forceinline__ int64_t act_elem(const Geom& g, const PosInfo& pi, int gi, int k) {
+  const int tap = k / g.Cg;
+  const int c = k - tap * g.Cg;
+  const int r = tap / g.S;
+  const int s = tap - r * g.S;
+  const int hi = pi.hb + r, wi = pi.wb + s;
+  if (hi < 0 || hi >= g.H || wi < 0 || wi >= g.W) return -1;
+  return (((int64_t)pi.b * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + c;
+}
+
+// One activation element as a byte lane (8-bit types: the byte; 4-bit types: the nibble,
+// sign-extended for S4).
+__device__ __forceinline__ uint32_t act_byte(const uint8_t* act, int type, int64_t e) {
+  if (e < 0) return 0;
+  if (type == FGQ_U8 || type == FGQ_S8) return act[e];
+  uint32_t nib = (act[e >> 1] >> (4 * (e & 1))) & 0xfu;
+  if (type == FGQ_S4) nib = (uint32_t)(((int)nib ^ 8) - 8) & 0xffu;
+  return nib;
+}
+
+// Four consecutive reduction elements k..k+3 as an int8x4 word.
+// mode 0: 8-bit, 4-byte aligned word within one tap; 1: 4-bit, 2-byte word within one tap;
+// 2: byte-by-byte gather.
+__device__ __forceinline__ uint32_t act_word(const uint8_t* act, const Geom& g, const PosInfo& pi,
+                                             int gi, int k, int mode) {
+  if (!pi.valid || k >= g.Kred) return 0;
+  if (mode == 0) {
+    const int64_t e = act_elem(g, pi, gi, k);
+    return e < 0 ? 0u : __ldg(reinterpret_cast<const uint32_t*>(act + e));
+  }
+  if (mode == 1) {
+    const int64_t e = act_elem(g, pi, gi, k);
+    if (e < 0) return 0u;
+    const uint32_t h = __ldg(reinterpret_cast<const uint16_t*>(act + (e >> 1)));
+    uint32_t v = (h & 0xfu) | ((h & 0xf0u) << 4) | ((h & 0xf00u) << 8) | ((h & 0xf000u) << 12);
+    if (g.act_type == FGQ_S4) v = __vsub4(v ^ 0x08080808u, 0x08080808u);
+    return v;
+  }
+  uint32_t v = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (k + i < g.Kred) v |= act_byte(act, g.act_type, act_elem(g, pi, gi, k + i)) << (8 * i);
+  }
+  return v;
+}
+
+template <int G, bool SA, bool DW, bool SUMS>
+__global__ void __launch_bounds__(NT) simt_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
+                                                           const void* __restrict__ weights,
+                                                           const float* __restrict__ scales,
+                                                           const float* __restrict__ act_scale,
+                                                           float* __restrict__ out, int32_t* __restrict__ sums,
+                                                           int mode, int mtiles) {
+  constexpr int KW = (G / 4 > 16) ? G / 4 : 16;  // words (4 elements) per chunk
+  constexpr int GPC = DW ? 1 : (KW * 4) / G;     // groups per chunk
+  constexpr int WPG = G / 4;                      // words per group
+
+  __shared__ uint32_t As[BP][KW + 1];
+  __shared__ __align__(16) uint32_t Ws[KW][BM];
+  __shared__ __align__(16) float Al[GPC][BM];
+  __shared__ uint32_t lut[256];
+
+  const int tid = threadIdx.x;
+  const int tx = tid % 16, ty = tid / 16;
+  const int gi = blockIdx.y / mtiles;
+  const int mt = blockIdx.y - gi * mtiles;
+  const int mlo = gi * g.Mg + mt * BM;        // first filter of the block
+  const int mhi = min(gi * g.Mg + g.Mg, g.M);  // end of this conv group
+  const int64_t p0 = (int64_t)blockIdx.x * BP;
+
+  if (!DW) {
+    for (int i = tid; i < 256; i += NT) lut[i] = expand_code_byte((uint32_t)i);
+  }
+
+  // staging assignment: one position, half of the chunk's words
+  const int spl = tid % BP;
+  const int swr = tid / BP;
+  const PosInfo spi = pos_info(g, p0 + spl);
+
+  float acc[4][8];
+  int iacc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      acc[i][j] = 0.0f;
+      iacc[i][j] = 0;
+    }
+
+  const int nchunks = (g.Kp + 4 * KW - 1) / (4 * KW);
+  const uint32_t* codes = static_cast<const uint32_t*>(weights);
+  const int8_t* wq = static_cast<const int8_t*>(weights);
+
+  for (int c = 0; c < nchunks; ++c) {
+    const int k0 = c * 4 * KW;
+    __syncthreads();
+    // activations
+#pragma unroll 4
+    for (int i = 0; i < KW / 2; ++i) {
+      const int kw = swr * (KW / 2) + i;
+      As[spl][kw] = act_word(act, g, spi, gi, k0 + 4 * kw, mode);
+    }
+    // weights
+    if (!DW) {
+      for (int idx = tid; idx < BM * (KW / 4); idx += NT) {
+        const int ml = idx % BM, cw = idx / BM;
+        const int m = mlo + ml;
+        const int wi = k0 / 16 + cw;
+        uint32_t word = 0;
+        if (m < mhi && wi < g.wrow) word = __ldg(codes + (int64_t)m * g.wrow + wi);
+#pragma unroll
+        for (int b = 0; b < 4; ++b) Ws[cw * 4 + b][ml] = lut[(word >> (8 * b)) & 0xffu];
+      }
+      for (int idx = tid; !SUMS && idx < BM * GPC; idx += NT) {
+        const int ml = idx % BM, gl = idx / BM;
+        const int m = mlo + ml;
+        const int gg = c * GPC + gl;
+        Al[gl][ml] = (m < mhi && gg < g.ng) ? __ldg(scales + (int64_t)m * g.ng + gg) : 0.0f;
+      }
+    } else {
+      for (int idx = tid; idx < BM * KW; idx += NT) {
+        const int ml = idx % BM, kw = idx / BM;
+        const int m = mlo + ml;
+        uint32_t v = 0;
+        if (m < mhi) {
+#pragma unroll
+          for (int b = 0; b < 4; ++b) {
+            const int k = k0 + 4 * kw + b;
+            if (k < g.Kred) v |= ((uint32_t)(uint8_t)wq[(int64_t)m * g.Kred + k]) << (8 * b);
+          }
+        }
+        Ws[kw][ml] = v;
+      }
+    }
+    __syncthreads();
+
+    if (DW) {
+#pragma unroll 4
+      for (int kw = 0; kw < KW; ++kw) {
+        const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[kw][ty * 4]);
+        const uint32_t bv[4] = {bw.x, bw.y, bw.z, bw.w};
+        uint32_t a[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) a[j] = As[tx + 16 * j][kw];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) iacc[i][j] = SA ? dp4a_ss(a[j], bv[i], iacc[i][j]) : dp4a_us(a[j], bv[i], iacc[i][j]);
+      }
+    } else {
+#pragma unroll 1
+      for (int gl = 0; gl < GPC; ++gl) {
+        const float4 al4 = *reinterpret_cast<const float4*>(&Al[gl][ty * 4]);
+        const float al[4] = {al4.x, al4.y, al4.z, al4.w};
+        int sm[4][8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) sm[i][j] = kMagicI;
+#pragma unroll
+        for (int wv = 0; wv < WPG; ++wv) {
+          const int kw = gl * WPG + wv;
+          const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[kw][ty * 4]);
+          const uint32_t bv[4] = {bw.x, bw.y, bw.z, bw.w};
+          uint32_t a[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) a[j] = As[tx + 16 * j][kw];
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sm[i][j] = SA ? dp4a_ss(a[j], bv[i], sm[i][j]) : dp4a_us(a[j], bv[i], sm[i][j]);
+        }
+        if (SUMS) {
+          const int gg = c * GPC + gl;
+          if (gg < g.ng) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int m = mlo + ty * 4 + i;
+              if (m >= mhi) continue;
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const int64_t p = p0 + tx + 16 * j;
+                if (p < g.P) sums[((int64_t)m * g.ng + gg) * g.P + p] = sm[i][j] - kMagicI;
+              }
+            }
+          }
+        } else {
+          const unsigned long long negc = pack_f2(-kMagicF, -kMagicF);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const unsigned long long a2 = pack_f2(al[i], al[i]);
+#pragma unroll
+            for (int j = 0; j < 8; j += 2) {
+              const unsigned long long s2 = add_f2(pack_f2(__int_as_float(sm[i][j]), __int_as_float(sm[i][j + 1])), negc);
+              unsigned long long c2 = pack_f2(acc[i][j], acc[i][j + 1]);
+              c2 = fma_f2(a2, s2, c2);
+              unpack_f2(c2, acc[i][j], acc[i][j + 1]);
+            }
+          }
+        }
+      }
+    }
+  }
+
+  if (SUMS) return;
+  const float sx = __ldg(act_scale);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int64_t p = p0 + tx + 16 * j;
+    if (p >= g.P) continue;
+    float* orow = out + p * g.M;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int m = mlo + ty * 4 + i;
+      if (m >= mhi) continue;
+      float v;
+      if (DW) v = sx * __ldg(scales + m) * (float)iacc[i][j];
+      else v = sx * acc[i][j];
+      orow[m] = v;
+    }
+  }
+}
+
+// Plain reference-style kernel for any G (used for G = 1 and 2): one thread per output.
+__global__ void simple_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
+                                       const uint32_t* __restrict__ codes, const float* __restrict__ alpha,
+                                       const float* __restrict__ act_scale, float* __restrict__ out,
+                                       int32_t* __restrict__ sums) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= g.P * g.M) return;
+  const int m = (int)(idx % g.M);
+  const int64_t p = idx / g.M;
+  const int gi = m / g.Mg;
+  const PosInfo pi = pos_info(g, p);
+  float acc = 0.0f;
+  for (int gg = 0; gg < g.ng; ++gg) {
+    int s = 0;
+    for (int j = gg * g.G; j < (gg + 1) * g.G && j < g.Kred; ++j) {
+      const uint32_t code = (codes[(int64_t)m * g.wrow + j / 16] >> (2 * (j % 16))) & 3u;
+      if (code == 0) continue;
+      int a = (int)act_byte(act, g.act_type, act_elem(g, pi, gi, j));
+      if (g.act_type == FGQ_S8 || g.act_type == FGQ_S4) a = (int)(int8_t)(uint8_t)a;
+      s += code == 1u ? a : -a;
+    }
+    if (sums) sums[((int64_t)m * g.ng + gg) * g.P + p] = s;
+    else acc = fmaf(alpha[(int64_t)m * g.ng + gg], (float)s, acc);
+  }
+  if (!sums) out[p * g.M + m] = acc * act_scale[0];
+}
+
+template <int G, bool SA, bool DW, bool SUMS>
+void launch_one(const void* act, const Geom& g, const void* w, const float* sc, const float* as, float* out,
+                int32_t* sums, int mode, cudaStream_t s) {
+  const int mtiles = (g.Mg + BM - 1) / BM;
+  dim3 grid((unsigned)((g.P + BP - 1) / BP), (unsigned)(mtiles * g.groups));
+  simt_contract_kernel<G, SA, DW, SUMS><<<grid, NT, 0, s>>>(static_cast<const uint8_t*>(act), g, w, sc, as, out,
+                                                            sums, mode, mtiles);
+}
+
+template <bool SA, bool SUMS>
+bool launch_g(const void* act, const Geom& g, const void* w, const float* sc, const float* as, float* out,
+              int32_t* sums, int mode, cudaStream_t s) {
+  switch (g.G) {
+    case 4: launch_one<4, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+    case 8: launch_one<8, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+    case 16: launch_one<16, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+    case 32: launch_one<32, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+    case 64: launch_one<64, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+    case 128: launch_one<128, SA, false, SUMS>(act, g, w, sc, as, out, sums, mode, s); return true;
+  }
+  return false;
+}
+
+}  // namespace
+
+fgq_status launch_simt_contract(const void* act, const Geom& g, const void* weights, const float* scales,
+                                int dense, const float* act_scale, float* out, int32_t* sums, cudaStream_t s) {
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  const bool is4 = g.act_type == FGQ_U4 || g.act_type == FGQ_S4;
+  const bool sa = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
+  // gather mode: whole words inside one tap need Cg % 4 == 0 (and alignment of the words)
+  int mode = 2;
+  if (g.Cg % 4 == 0 && g.C % 4 == 0) mode = is4 ? 1 : 0;
+  if (!dense && (g.G == 1 || g.G == 2)) {
+    const int64_t n = g.P * g.M;
+    simple_contract_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(
+        static_cast<const uint8_t*>(act), g, static_cast<const uint32_t*>(weights), scales, act_scale, out, sums);
+    return after_launch();
+  }
+  if (dense) {
+    if (sa) launch_one<4, true, true, false>(act, g, weights, scales, act_scale, out, nullptr, mode, s);
+    else launch_one<4, false, true, false>(act, g, weights, scales, act_scale, out, nullptr, mode, s);
+    return after_launch();
+  }
+  bool ok;
+  if (sums) ok = sa ? launch_g<true, true>(act, g, weights, scales, act_scale, out, sums, mode, s)
+                    : launch_g<false, true>(act, g, weights, scales, act_scale, out, sums, mode, s);
+  else ok = sa ? launch_g<true, false>(act, g, weights, scales, act_scale, out, sums, mode, s)
+               : launch_g<false, false>(act, g, weights, scales, act_scale, out, sums, mode, s);
+  if (!ok) return FGQ_ERR_UNSUPPORTED;
+  return after_launch();
+}
+
+}  // namespace fgq

@@ -1,0 +1,198 @@
+// Dynamic-fixed-point activation quantization (Section 4: activations are quantized to 8
+// or 4 bits before each convolution, with one shared exponent per tensor).
+//
+//   E   = smallest integer with max * 2^-E <= qmax (max = max|x|, or max(x, 0) for the
+//         unsigned types), 0 when max = 0, clamped to [-149, 127];
+//   q_i = clamp(round_half_even(x_i * 2^-E), qmin, qmax),   scale = 2^E.
+//
+// x * 2^-E is exact in fp32 whenever the result is at least 2^-126 (a power-of-two
+// scaling), and a product below that rounds to the integer 0 whichever way it is rounded,
+// so the codes are exact.  When 2^-E exceeds the fp32 range the scaling is applied as two
+// exact factors.
+//
+// Pass 1 (derived scale only): per-block maxima of the magnitude bit patterns (non-negative
+// floats order like their bits) into the caller's workspace.  Pass 2: every block reduces
+// the block maxima, derives E, and quantizes a grid-stride share of 16-element chunks.
+#include <climits>
+#include <cstdint>
+
+#include "fgq_device.cuh"
+
+namespace fgq {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ uint32_t mag_bits(float x, bool is_unsigned) {
+  const uint32_t b = __float_as_uint(x);
+  if (is_unsigned) return (b >> 31) ? 0u : b;  // negative (and -0) count as 0
+  return b & 0x7fffffffu;
+}
+
+__global__ void __launch_bounds__(kThreads) qa_max_kernel(const float* __restrict__ x, size_t n, int is_unsigned,
+                                                          uint32_t* __restrict__ partials, unsigned int* err) {
+  uint32_t mx = 0;
+  bool bad = false;
+  const size_t n4 = n / 4;
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const size_t nth = (size_t)gridDim.x * blockDim.x;
+  for (size_t i = tid; i < n4; i += nth) {
+    const float4 f = __ldg(x4 + i);
+    const float e[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      bad |= (__float_as_uint(e[j]) & 0x7fffffffu) >= 0x7f800000u;
+      mx = max(mx, mag_bits(e[j], is_unsigned));
+    }
+  }
+  for (size_t i = n4 * 4 + tid; i < n; i += nth) {
+    const float e = __ldg(x + i);
+    bad |= (__float_as_uint(e) & 0x7fffffffu) >= 0x7f800000u;
+    mx = max(mx, mag_bits(e, is_unsigned));
+  }
+  __shared__ uint32_t red[kThreads / 32];
+  mx = __reduce_max_sync(FULL_MASK, mx);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  if (__syncthreads_or(bad) && threadIdx.x == 0) record_error(err, FGQ_ERR_NONFINITE);
+  if (threadIdx.x == 0) {
+    uint32_t m = 0;
+    for (int i = 0; i < kThreads / 32; ++i) m = max(m, red[i]);
+    partials[blockIdx.x] = m;
+  }
+}
+
+__device__ __forceinline__ int dfp_exponent(uint32_t mbits, int qmax) {
+  if (mbits == 0 || mbits >= 0x7f800000u) return 0;
+  const double md = (double)__uint_as_float(mbits);
+  int E = (int)((__double_as_longlong(md) >> 52) & 0x7ff) - 1023 - 10;  // condition fails here
+  while (md * pow2d(-E) > (double)qmax) ++E;
+  return max(-149, min(127, E));
+}
+
+template <int TYPE>
+struct QTraits;
+template <> struct QTraits<FGQ_U8> { static constexpr int qmin = 0, qmax = 255, bits = 8; };
+template <> struct QTraits<FGQ_S8> { static constexpr int qmin = -128, qmax = 127, bits = 8; };
+template <> struct QTraits<FGQ_U4> { static constexpr int qmin = 0, qmax = 15, bits = 4; };
+template <> struct QTraits<FGQ_S4> { static constexpr int qmin = -8, qmax = 7, bits = 4; };
+
+template <int TYPE>
+__device__ __forceinline__ uint32_t qcode(float x, float mul1, float mul2) {
+  using T = QTraits<TYPE>;
+  int r = __float2int_rn(x * mul1 * mul2);
+  r = max(T::qmin, min(T::qmax, r));
+  return (uint32_t)r & ((1u << T::bits) - 1u);
+}
+
+template <int TYPE>
+__global__ void __launch_bounds__(kThreads) qa_quant_kernel(const float* __restrict__ x, size_t n,
+                                                            const uint32_t* __restrict__ partials, int nparts,
+                                                            int E_given, uint8_t* __restrict__ q,
+                                                            float* __restrict__ scale_out) {
+  using T = QTraits<TYPE>;
+  __shared__ int sE;
+  __shared__ uint32_t red[kThreads / 32];
+  int E = E_given;
+  if (partials != nullptr) {
+    uint32_t mx = 0;
+    for (int i = threadIdx.x; i < nparts; i += blockDim.x) mx = max(mx, partials[i]);
+    mx = __reduce_max_sync(FULL_MASK, mx);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      uint32_t m = 0;
+      for (int i = 0; i < kThreads / 32; ++i) m = max(m, red[i]);
+      sE = dfp_exponent(m, T::qmax);
+    }
+    __syncthreads();
+    E = sE;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0 && scale_out != nullptr) *scale_out = pow2f(E);
+  const float mul1 = (-E <= 127) ? pow2f(-E) : pow2f(64);
+  const float mul2 = (-E <= 127) ? 1.0f : pow2f(-E - 64);
+
+  const size_t n16 = n / 16;
+  const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const size_t nth = (size_t)gridDim.x * blockDim.x;
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  for (size_t c = tid; c < n16; c += nth) {
+    float e[16];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 f = __ldg(x4 + 4 * c + j);
+      e[4 * j] = f.x; e[4 * j + 1] = f.y; e[4 * j + 2] = f.z; e[4 * j + 3] = f.w;
+    }
+    if (T::bits == 8) {
+      uint4 o;
+      uint32_t wv[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        wv[j] = qcode<TYPE>(e[4 * j], mul1, mul2) | (qcode<TYPE>(e[4 * j + 1], mul1, mul2) << 8) |
+                (qcode<TYPE>(e[4 * j + 2], mul1, mul2) << 16) | (qcode<TYPE>(e[4 * j + 3], mul1, mul2) << 24);
+      }
+      o.x = wv[0]; o.y = wv[1]; o.z = wv[2]; o.w = wv[3];
+      reinterpret_cast<uint4*>(q)[c] = o;
+    } else {
+      uint32_t wv[2] = {0u, 0u};
+#pragma unroll
+      for (int j = 0; j < 16; ++j) wv[j / 8] |= qcode<TYPE>(e[j], mul1, mul2) << (4 * (j % 8));
+      reinterpret_cast<uint2*>(q)[c] = make_uint2(wv[0], wv[1]);
+    }
+  }
+  if (tid == 0) {  // ragged tail of fewer than 16 elements
+    for (size_t i = n16 * 16; i < n; ++i) {
+      const uint32_t code = qcode<TYPE>(x[i], mul1, mul2);
+      if (T::bits == 8) {
+        q[i] = (uint8_t)code;
+      } else if ((i & 1) == 0) {
+        q[i / 2] = (uint8_t)code;  // the high nibble of an odd tail stays 0
+      } else {
+        q[i / 2] = (uint8_t)(q[i / 2] | (code << 4));
+      }
+    }
+  }
+}
+
+int num_sms() {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms;
+}
+
+int max_blocks(size_t n) {
+  const size_t need = (n / 16 + kThreads - 1) / kThreads;
+  const size_t cap = (size_t)num_sms() * 8;
+  return (int)(need < 1 ? 1 : (need < cap ? need : cap));
+}
+
+}  // namespace
+
+size_t quantize_workspace_bytes(size_t n) {
+  if (n == 0) return 0;
+  return sizeof(uint32_t) * (size_t)max_blocks(n);
+}
+
+fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool derive, void* q,
+                           float* scale_out, uint32_t* partials, unsigned int* err, cudaStream_t s) {
+  const int blocks = max_blocks(n);
+  if (derive) {
+    qa_max_kernel<<<blocks, kThreads, 0, s>>>(x, n, (type == FGQ_U8 || type == FGQ_U4) ? 1 : 0, partials, err);
+    fgq_status st = after_launch();
+    if (st != FGQ_OK) return st;
+  } else {
+    partials = nullptr;
+  }
+  uint8_t* qb = static_cast<uint8_t*>(q);
+  switch (type) {
+    case FGQ_U8: qa_quant_kernel<FGQ_U8><<<blocks, kThreads, 0, s>>>(x, n, partials, blocks, E_given, qb, scale_out); break;
+    case FGQ_S8: qa_quant_kernel<FGQ_S8><<<blocks, kThreads, 0, s>>>(x, n, partials, blocks, E_given, qb, scale_out); break;
+    case FGQ_U4: qa_quant_kernel<FGQ_U4><<<blocks, kThreads, 0, s>>>(x, n, partials, blocks, E_given, qb, scale_out); break;
+    case FGQ_S4: qa_quant_kernel<FGQ_S4><<<blocks, kThreads, 0, s>>>(x, n, partials, blocks, E_given, qb, scale_out); break;
+    default: return FGQ_ERR_ARG;
+  }
+  return after_launch();
+}
+
+}  // namespace fgq

@@ -1,0 +1,245 @@
+"""Python binding of libfgq (the FGQ CUDA library): argument marshalling only.
+
+Every function here checks tensor dtypes/devices, passes raw device pointers, sizes and
+the current CUDA stream to the C ABI of ``include/fgq.h`` and raises on a non-OK status.
+All computation happens in the library's CUDA kernels; there is no CPU fallback, and
+loading fails loudly if the library is missing or CUDA is unavailable.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfgq.so")
+
+FGQ_OK, FGQ_ERR_ARG, FGQ_ERR_ALIGN, FGQ_ERR_UNSUPPORTED, FGQ_ERR_NONFINITE, FGQ_ERR_TIMEOUT, FGQ_ERR_CUDA = range(7)
+U8, S8, U4, S4 = 0, 1, 2, 3
+PATH_AUTO, PATH_SIMT, PATH_TC = 0, 1, 2
+ACT_TYPES = {"u8": U8, "s8": S8, "u4": U4, "s4": S4}
+
+_lib: Optional[ctypes.CDLL] = None
+
+# (name, restype, argtypes) of every exported symbol of include/fgq.h
+_vp, _i, _i64, _u32, _u64, _f, _sz = (ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_uint32,
+                                      ctypes.c_uint64, ctypes.c_float, ctypes.c_size_t)
+SIGNATURES = [
+    ("fgq_version", _i, []),
+    ("fgq_status_string", ctypes.c_char_p, [_i]),
+    ("fgq_codes_words_per_row", _i64, [_i, _i]),
+    ("fgq_num_groups", _i64, [_i, _i]),
+    ("fgq_ternarize", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_quantize_act_workspace_bytes", _sz, [_sz]),
+    ("fgq_quantize_act", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp, _sz, _vp]),
+    ("fgq_quantize_weights_w8", _i, [_vp, _i, _i, _vp, _vp, _vp]),
+    ("fgq_gemm", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _vp, _vp]),
+    ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
+    ("fgq_conv2d_w8", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _vp]),
+    ("fgq_group_sums", _i, [_vp, _i, _i, _i, _vp, _i, _i, _vp, _vp]),
+    ("fgq_stream_status", _i, [_vp]),
+    ("fgq_set_path", _i, [_i]),
+    ("fgq_last_path", _i, []),
+    ("fgq_launch_count", _u64, []),
+    ("fgq_selftest_wait_timeout", _i, [_u32, _vp]),
+]
+
+
+class FGQError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        name = lib().fgq_status_string(code).decode() if _lib is not None else str(code)
+        super().__init__(f"{what}: {name}")
+        self.code = code
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libfgq.so (built by paper_1705_01462_gb300.build) and declare its signatures."""
+    if not os.path.exists(path):
+        raise RuntimeError(f"libfgq.so not found at {path}: build it with "
+                           "`python -c 'import __graft_entry__ as g; g.build()'` (no CPU fallback exists)")
+    L = ctypes.CDLL(path)
+    for name, res, args in SIGNATURES:
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    return L
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        _lib = load()
+    return _lib
+
+
+def _require_cuda():
+    if not torch.cuda.is_available():
+        raise RuntimeError("libfgq needs a CUDA GPU; there is no CPU fallback")
+
+
+def _check(code: int, what: str):
+    if code != FGQ_OK:
+        raise FGQError(code, what)
+
+
+def _stream(stream=None) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _dev(t: torch.Tensor, dtype, name: str) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _act_type(t) -> int:
+    return ACT_TYPES[t] if isinstance(t, str) else int(t)
+
+
+# --------------------------------------------------------------------------- sizes
+
+def codes_words_per_row(Kred: int, G: int) -> int:
+    return int(lib().fgq_codes_words_per_row(Kred, G))
+
+
+def num_groups(Kred: int, G: int) -> int:
+    return int(lib().fgq_num_groups(Kred, G))
+
+
+def quantize_act_workspace_bytes(n: int) -> int:
+    return int(lib().fgq_quantize_act_workspace_bytes(n))
+
+
+def act_bytes(n: int, act_type) -> int:
+    return n if _act_type(act_type) in (U8, S8) else (n + 1) // 2
+
+
+# --------------------------------------------------------------------------- calls
+
+def fgq_ternarize(w: torch.Tensor, G: int, codes: Optional[torch.Tensor] = None,
+                  alpha: Optional[torch.Tensor] = None, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """w fp32 [M][Kred] -> (codes int32-view of uint32 [M][words], alpha fp32 [M][ng])."""
+    _require_cuda()
+    M, Kred = w.shape
+    if codes is None:
+        codes = torch.empty((M, codes_words_per_row(Kred, G)), dtype=torch.int32, device=w.device)
+    if alpha is None:
+        alpha = torch.empty((M, num_groups(Kred, G)), dtype=torch.float32, device=w.device)
+    _check(lib().fgq_ternarize(_dev(w, torch.float32, "w"), M, Kred, G, _dev(codes, torch.int32, "codes"),
+                               _dev(alpha, torch.float32, "alpha"), _stream(stream)), "fgq_ternarize")
+    return codes, alpha
+
+
+def fgq_quantize_act(x: torch.Tensor, act_type="u8", scale_in: float = 0.0, q: Optional[torch.Tensor] = None,
+                     scale_out: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                     stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """fp32 tensor -> (codes uint8 [n or ceil(n/2)], scale fp32 [1] = 2^E)."""
+    _require_cuda()
+    ty = _act_type(act_type)
+    n = x.numel()
+    if q is None:
+        q = torch.empty(act_bytes(n, ty), dtype=torch.uint8, device=x.device)
+    if scale_out is None:
+        scale_out = torch.empty(1, dtype=torch.float32, device=x.device)
+        if scale_in > 0:
+            scale_out.fill_(scale_in)
+    wsb = quantize_act_workspace_bytes(n)
+    if workspace is None and scale_in <= 0:
+        workspace = torch.empty(max(wsb, 4), dtype=torch.uint8, device=x.device)
+    ws_ptr = workspace.data_ptr() if workspace is not None else None
+    ws_len = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().fgq_quantize_act(_dev(x, torch.float32, "x"), n, ty, float(scale_in), _dev(q, torch.uint8, "q"),
+                                  _dev(scale_out, torch.float32, "scale_out") if scale_in <= 0 else None,
+                                  ws_ptr, ws_len, _stream(stream)), "fgq_quantize_act")
+    return q, scale_out
+
+
+def fgq_quantize_weights_w8(w: torch.Tensor, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    _require_cuda()
+    M, Kred = w.shape
+    wq = torch.empty((M, Kred), dtype=torch.int8, device=w.device)
+    ws = torch.empty(M, dtype=torch.float32, device=w.device)
+    _check(lib().fgq_quantize_weights_w8(_dev(w, torch.float32, "w"), M, Kred, wq.data_ptr(), ws.data_ptr(),
+                                         _stream(stream)), "fgq_quantize_weights_w8")
+    return wq, ws
+
+
+def fgq_gemm(q: torch.Tensor, act_type, act_scale: torch.Tensor, P: int, Kred: int, codes: torch.Tensor,
+             alpha: torch.Tensor, M: int, G: int, y: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    _require_cuda()
+    if y is None:
+        y = torch.empty((P, M), dtype=torch.float32, device=q.device)
+    _check(lib().fgq_gemm(_dev(q, torch.uint8, "q"), _act_type(act_type), _dev(act_scale, torch.float32, "act_scale"),
+                          P, Kred, _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
+                          _dev(y, torch.float32, "y"), _stream(stream)), "fgq_gemm")
+    return y
+
+
+def conv_out_hw(H, W, R, S, stride, pad):
+    return (H + 2 * pad - R) // stride + 1, (W + 2 * pad - S) // stride + 1
+
+
+def fgq_conv2d(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, H: int, W: int, C: int, R: int, S: int,
+               stride: int, pad: int, groups: int, codes: torch.Tensor, alpha: torch.Tensor, M: int, G: int,
+               out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if out is None:
+        out = torch.empty((B, Ho, Wo, M), dtype=torch.float32, device=act.device)
+    _check(lib().fgq_conv2d(_dev(act, torch.uint8, "act"), _act_type(act_type),
+                            _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
+                            _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
+                            _dev(out, torch.float32, "out"), _stream(stream)), "fgq_conv2d")
+    return out
+
+
+def fgq_conv2d_w8(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, H: int, W: int, C: int, R: int,
+                  S: int, stride: int, pad: int, groups: int, wq: torch.Tensor, wscale: torch.Tensor, M: int,
+                  out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if out is None:
+        out = torch.empty((B, Ho, Wo, M), dtype=torch.float32, device=act.device)
+    _check(lib().fgq_conv2d_w8(_dev(act, torch.uint8, "act"), _act_type(act_type),
+                               _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
+                               _dev(wq, torch.int8, "wq"), _dev(wscale, torch.float32, "wscale"), M,
+                               _dev(out, torch.float32, "out"), _stream(stream)), "fgq_conv2d_w8")
+    return out
+
+
+def fgq_group_sums(q: torch.Tensor, act_type, P: int, Kred: int, codes: torch.Tensor, M: int, G: int,
+                   stream=None) -> torch.Tensor:
+    _require_cuda()
+    s = torch.empty((M, num_groups(Kred, G), P), dtype=torch.int32, device=q.device)
+    _check(lib().fgq_group_sums(_dev(q, torch.uint8, "q"), _act_type(act_type), P, Kred,
+                                _dev(codes, torch.int32, "codes"), M, G, s.data_ptr(), _stream(stream)),
+           "fgq_group_sums")
+    return s
+
+
+def fgq_stream_status(stream=None) -> int:
+    return int(lib().fgq_stream_status(_stream(stream)))
+
+
+def fgq_set_path(path: int) -> int:
+    return int(lib().fgq_set_path(path))
+
+
+def fgq_last_path() -> int:
+    return int(lib().fgq_last_path())
+
+
+def fgq_launch_count() -> int:
+    return int(lib().fgq_launch_count())
+
+
+def fgq_selftest_wait_timeout(max_iterations: int, stream=None) -> int:
+    _check(lib().fgq_selftest_wait_timeout(max_iterations, _stream(stream)), "fgq_selftest_wait_timeout")
+    return fgq_stream_status(stream)

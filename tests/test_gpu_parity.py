@@ -1,0 +1,236 @@
+"""GPU parity: the CUDA kernels (called through the C ABI) against the CPU oracle.
+
+Integer outputs (codes, packed activations, group sums) must match bit for bit; fp32
+alphas bit for bit (both sides round the exact mean to nearest); fp32 contraction outputs
+within 1e-5 * act_scale * sum_g |alpha_g * s_g| per element.
+"""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_1705_01462_gb300 import fgq, synth
+from _gpu import (dev, to_dev, codes_u32, check_within, make_codes, quantize_oracle, random_acts,
+                  ORACLE_TYPE)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _clean_status():
+    fgq.fgq_set_path(fgq.PATH_AUTO)
+    yield
+    fgq.fgq_set_path(fgq.PATH_AUTO)
+    assert fgq.fgq_stream_status() == fgq.FGQ_OK
+
+
+# ----------------------------------------------------------------------------- ternarize
+
+def _adversarial_weights(M, K, seed):
+    rng = np.random.default_rng(seed)
+    w = rng.standard_normal((M, K)).astype(np.float32)
+    w[0::7] = rng.choice([-0.5, 0.25, 0.5, 0.125], (len(w[0::7]), K))               # ties
+    w[1::7] *= (rng.random((len(w[1::7]), K)) < 0.3)                                 # zeros
+    w[2::7] *= np.float32(2.0 ** -140)                                               # subnormal
+    w[3::7] *= (2.0 ** rng.integers(-30, 4, (len(w[3::7]), K))).astype(np.float32)    # wide range
+    w[4::7] = 0.0                                                                    # all zero
+    w[5::7] = (rng.exponential(1.0, (len(w[5::7]), K)) * rng.choice([-1, 1], (len(w[5::7]), K)))
+    return w.astype(np.float32)
+
+
+@pytest.mark.parametrize("G", [1, 2, 4, 8, 16, 32, 64, 128])
+@pytest.mark.parametrize("K", [7, 64, 147, 576, 1000])
+def test_ternarize_bit_exact(G, K):
+    w = _adversarial_weights(37, K, seed=G * 1000 + K)
+    t, al, codes = make_codes(w, G)
+    gc, ga = fgq.fgq_ternarize(to_dev(w), G)
+    assert np.array_equal(codes_u32(gc), codes)
+    assert np.array_equal(ga.cpu().numpy().view(np.uint32), al.view(np.uint32))
+
+
+@pytest.mark.parametrize("G", [4, 16, 64])
+def test_ternarize_resnet50_weight_set(G):
+    """Full ResNet-50 weight set (53 convs + fc, 25,502,912 weights), every group bit-exact."""
+    layers = synth.resnet50_convs() + [synth.resnet50_fc()]
+    for i, layer in enumerate(layers):
+        w = synth.weights(layer, synth.layer_seed(i))
+        t, al, codes = make_codes(w, G)
+        gc, ga = fgq.fgq_ternarize(to_dev(w), G)
+        assert np.array_equal(codes_u32(gc), codes), layer.name
+        assert np.array_equal(ga.cpu().numpy(), al), layer.name
+
+
+def test_ternarize_nonfinite_status():
+    w = np.ones((4, 64), np.float32)
+    w[1, 5] = np.nan
+    gc, ga = fgq.fgq_ternarize(to_dev(w), 4)
+    assert fgq.fgq_stream_status() == fgq.FGQ_ERR_NONFINITE
+    a = ga.cpu().numpy()
+    assert a[1, 1] == 0 and a[1, 0] == 1.0 and codes_u32(gc)[1, 0] & 0xff00 == 0
+
+
+def test_quantize_weights_w8():
+    rng = np.random.default_rng(5)
+    w = (rng.standard_normal((64, 147)) * 0.1).astype(np.float32)
+    wq, ws = fgq.fgq_quantize_weights_w8(to_dev(w))
+    owq, ows = O.quantize_weights_w8(w)
+    assert np.array_equal(wq.cpu().numpy(), owq) and np.array_equal(ws.cpu().numpy(), ows)
+
+
+# ----------------------------------------------------------------------------- quantize
+
+@pytest.mark.parametrize("act_type", ["u8", "s8", "u4", "s4"])
+@pytest.mark.parametrize("n", [1, 15, 16, 17, 4096 + 7, 1 << 20])
+def test_quantize_bit_exact(act_type, n):
+    rng = np.random.default_rng(n)
+    x = (rng.standard_normal(n) * 3).astype(np.float32)
+    q, sc, packed = quantize_oracle(x, act_type)
+    gq, gs = fgq.fgq_quantize_act(to_dev(x), act_type)
+    assert np.array_equal(gq.cpu().numpy(), packed)
+    assert gs.item() == sc
+
+
+@pytest.mark.parametrize("scale_exp", [-149, -140, -60, 0, 20, 120])
+def test_quantize_extreme_scales(scale_exp):
+    rng = np.random.default_rng(scale_exp + 200)
+    x = (rng.standard_normal(1000) * 2.0 ** scale_exp).astype(np.float32)
+    for act_type in ("u8", "s4"):
+        q, sc, packed = quantize_oracle(x, act_type)
+        gq, gs = fgq.fgq_quantize_act(to_dev(x), act_type)
+        assert np.array_equal(gq.cpu().numpy(), packed) and gs.item() == sc
+        # given power-of-two scale, including ones that saturate
+        for e in (scale_exp - 9, scale_exp + 3):
+            if -149 <= e <= 127:
+                s_in = float(np.float32(2.0 ** e))
+                oq, _, _, _ = O.quantize(x, ORACLE_TYPE[act_type], s_in)
+                gq, _ = fgq.fgq_quantize_act(to_dev(x), act_type, scale_in=s_in)
+                assert np.array_equal(gq.cpu().numpy(), O.pack_act(oq, ORACLE_TYPE[act_type]))
+
+
+def test_quantize_zero_and_nonfinite():
+    gq, gs = fgq.fgq_quantize_act(to_dev(np.zeros(100, np.float32)), "u8")
+    assert gs.item() == 1.0 and not gq.cpu().numpy().any()
+    x = np.ones(64, np.float32)
+    x[3] = np.inf
+    fgq.fgq_quantize_act(to_dev(x), "u8")
+    assert fgq.fgq_stream_status() == fgq.FGQ_ERR_NONFINITE
+
+
+# ----------------------------------------------------------------------------- contraction
+
+CONV_CASES = [
+    # B, H, W, C, M, R, S, stride, pad, groups, G, act
+    (1, 56, 56, 64, 64, 3, 3, 1, 1, 1, 4, "u8"),     # ResNet-50 conv2_x 3x3 at batch 1
+    (2, 9, 11, 64, 70, 3, 3, 1, 1, 1, 4, "u8"),      # ragged M and P tiles
+    (1, 13, 13, 64, 96, 3, 3, 2, 1, 1, 8, "s8"),
+    (2, 8, 8, 32, 40, 1, 1, 1, 0, 1, 16, "u8"),
+    (1, 7, 7, 64, 33, 3, 3, 1, 1, 1, 32, "u8"),
+    (2, 7, 7, 128, 130, 3, 3, 1, 1, 1, 64, "u8"),
+    (1, 6, 6, 256, 64, 1, 1, 1, 0, 1, 128, "s8"),
+    (1, 14, 14, 64, 64, 1, 1, 2, 0, 1, 64, "u8"),    # strided 1x1
+    (1, 27, 27, 48, 64, 5, 5, 1, 2, 2, 4, "u8"),     # conv groups = 2 (AlexNet towers)
+    (1, 23, 23, 3, 16, 11, 11, 4, 0, 1, 4, "u8"),    # C = 3: groups straddle taps
+    (1, 9, 9, 16, 8, 3, 3, 1, 1, 1, 1, "u8"),        # G = 1
+    (1, 9, 9, 16, 8, 3, 3, 1, 1, 1, 2, "s8"),        # G = 2
+    (2, 10, 10, 64, 64, 3, 3, 1, 1, 1, 4, "u4"),     # packed 4-bit activations
+    (1, 10, 10, 128, 64, 3, 3, 1, 1, 1, 64, "u4"),
+    (1, 8, 8, 64, 32, 3, 3, 1, 1, 1, 4, "s4"),
+    (1, 9, 9, 6, 8, 3, 3, 1, 1, 1, 4, "u4"),         # 4-bit with C % 4 != 0
+]
+
+
+@pytest.mark.parametrize("case", CONV_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_conv2d_parity(case):
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()))
+    Cg = C // groups
+    w = (rng.standard_normal((M, R * S * Cg)) * np.sqrt(2.0 / (R * S * Cg))).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    gout = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride,
+                          pad, groups, to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    check_within(gout.cpu().numpy(), y, ym, f"conv2d {case}")
+
+
+GEMM_CASES = [(1, 9216, 64, 4, "u8"), (37, 576, 70, 4, "s8"), (129, 200, 65, 8, "u8"), (64, 4096, 128, 64, "u8"),
+              (5, 130, 17, 64, "s8"), (300, 256, 64, 128, "u8"), (16, 96, 24, 32, "u4"), (3, 22, 5, 2, "u8")]
+
+
+@pytest.mark.parametrize("case", GEMM_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_gemm_and_group_sums(case):
+    P, K, M, G, act = case
+    rng = np.random.default_rng(P * 31 + K)
+    w = rng.standard_normal((M, K)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((P, K), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.gemm(q, sc, t, al, G)
+    gy = fgq.fgq_gemm(to_dev(packed), act, to_dev(np.array([sc], np.float32)), P, K, to_dev(codes.view(np.int32)),
+                      to_dev(al), M, G)
+    check_within(gy.cpu().numpy(), y, ym, f"gemm {case}")
+    s = O.group_sums(q, t, G)
+    gs = fgq.fgq_group_sums(to_dev(packed), act, P, K, to_dev(codes.view(np.int32)), M, G)
+    assert np.array_equal(gs.cpu().numpy().astype(np.int64), s)
+
+
+def test_conv2d_w8_first_layer():
+    """ResNet stem shape (7x7/2, C = 3) with 8-bit weights, at a reduced image size."""
+    rng = np.random.default_rng(9)
+    B, H, W, C, M, R, stride, pad = 2, 40, 36, 3, 64, 7, 2, 3
+    w = (rng.standard_normal((M, R * R * C)) * np.sqrt(2.0 / 147)).astype(np.float32)
+    x = np.abs(rng.standard_normal((B, H, W, C))).astype(np.float32)
+    q, sc, packed = quantize_oracle(x, "u8")
+    wq, ws = fgq.fgq_quantize_weights_w8(to_dev(w))
+    owq, ows = O.quantize_weights_w8(w)
+    y, ym = O.conv2d_w8(q, sc, R, R, stride, pad, 1, owq, ows)
+    g = fgq.fgq_conv2d_w8(to_dev(packed), "u8", to_dev(np.array([sc], np.float32)), B, H, W, C, R, R, stride, pad, 1,
+                          wq, ws, M)
+    check_within(g.cpu().numpy(), y, ym, "conv2d_w8")
+
+
+def test_chain_quantize_ternarize_conv_on_device():
+    """The whole hot path on device buffers: fp32 weights and activations in, fp32 out."""
+    layer = synth.conv2x_3x3()
+    B, G = 1, 4
+    w = synth.weights(layer, 11)
+    x = synth.activations((B, layer.H, layer.W, layer.C), 12)
+    t, al, _ = make_codes(w, G)
+    q, sc, _ = quantize_oracle(x, "u8")
+    y, ym = O.conv2d(q, sc, 3, 3, 1, 1, 1, t, al, G)
+    codes, alpha = fgq.fgq_ternarize(to_dev(w), G)
+    gq, gs = fgq.fgq_quantize_act(to_dev(x), "u8")
+    out = fgq.fgq_conv2d(gq, "u8", gs, B, layer.H, layer.W, layer.C, 3, 3, 1, 1, 1, codes, alpha, layer.M, G)
+    check_within(out.cpu().numpy(), y, ym, "chain")
+
+
+@pytest.mark.parametrize("G", [4, 64])
+def test_config2_batch32_sampled(G):
+    """ResNet-50 conv2_x 3x3 at batch 32 (100,352 positions): sampled positions, all filters."""
+    layer = synth.conv2x_3x3()
+    B = 32
+    w = synth.weights(layer, 21)
+    x = synth.activations((B, layer.H, layer.W, layer.C), 22)
+    t, al, codes = make_codes(w, G)
+    q, sc, packed = quantize_oracle(x, "u8")
+    out = fgq.fgq_conv2d(to_dev(packed), "u8", to_dev(np.array([sc], np.float32)), B, layer.H, layer.W, layer.C,
+                         3, 3, 1, 1, 1, to_dev(codes.view(np.int32)), to_dev(al), layer.M, G)
+    rng = np.random.default_rng(G)
+    P = layer.P(B)
+    pos = np.unique(np.r_[rng.choice(P, 600, replace=False), [0, P - 1, 55, 56, 3135, 3136]])
+    y, ym = O.conv2d(q, sc, 3, 3, 1, 1, 1, t, al, G, positions=pos)
+    check_within(out.reshape(P, layer.M).cpu().numpy()[pos], y, ym, "config2")
+
+
+def test_wait_timeout_selftest():
+    assert fgq.fgq_selftest_wait_timeout(4) == fgq.FGQ_ERR_TIMEOUT
+    assert fgq.fgq_stream_status() == fgq.FGQ_OK  # cleared by the read
+
+
+def test_launch_counter_counts():
+    n0 = fgq.fgq_launch_count()
+    fgq.fgq_quantize_act(to_dev(np.ones(100, np.float32)), "u8")
+    assert fgq.fgq_launch_count() == n0 + 2
