@@ -183,7 +183,8 @@ fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_sc
 /*
  * The 32-bit group accumulators themselves (Section 4), for verification:
  *   s[m][g][p] = sum_{j in g, j < Kred} t[m][j] * q[p][j],  int32 [M][ng][P].
- * q as in fgq_gemm.  Errors as fgq_gemm.
+ * q as in fgq_gemm.  Always computed by the CUDA-core (dp4a) kernel family, whatever
+ * fgq_set_path selects.  Errors as fgq_gemm.
  */
 fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred,
                           const uint32_t* codes, int M, int G, int32_t* s, cudaStream_t stream);

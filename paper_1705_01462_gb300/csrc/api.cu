@@ -54,8 +54,9 @@ fgq_status make_geom(int type, int B, int H, int W, int C, int R, int S, int str
   return FGQ_OK;
 }
 
-int choose_path(const Geom& g) {
+int choose_path(const Geom& g, bool sums) {
   const int forced = g_path.load();
+  if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
   if (forced == FGQ_PATH_TC) return tc_supports(g) ? FGQ_PATH_TC : -1;
   return tc_supports(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
@@ -64,7 +65,7 @@ int choose_path(const Geom& g) {
 fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                     const float* act_scale, float* out, int32_t* sums, cudaStream_t s) {
   if (g.P == 0 || g.M == 0) return FGQ_OK;
-  const int path = choose_path(g);
+  const int path = choose_path(g, sums != nullptr);
   if (path < 0) return FGQ_ERR_UNSUPPORTED;
   t_last_path = path;
   unsigned int* err = device_error_word();

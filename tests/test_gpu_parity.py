@@ -234,3 +234,65 @@ def test_launch_counter_counts():
     n0 = fgq.fgq_launch_count()
     fgq.fgq_quantize_act(to_dev(np.ones(100, np.float32)), "u8")
     assert fgq.fgq_launch_count() == n0 + 2
+
+
+# ----------------------------------------------------------------------------- tensor-core path
+
+TC_CASES = [
+    # B, H, W, C, M, R, S, stride, pad, groups, G, act
+    (1, 7, 9, 64, 128, 1, 1, 1, 0, 1, 64, "u8"),     # single tile, 1x1
+    (2, 9, 11, 64, 64, 3, 3, 1, 1, 1, 64, "u8"),     # M = 64 (half tile), ragged P
+    (1, 12, 12, 128, 200, 3, 3, 1, 1, 1, 64, "s8"),  # ragged M tile
+    (2, 14, 14, 128, 256, 1, 1, 2, 0, 1, 64, "u8"),  # strided 1x1, two M tiles
+    (1, 8, 8, 256, 96, 3, 3, 1, 1, 1, 128, "u8"),    # G = 128: two K-tiles per group
+    (1, 13, 13, 384, 384, 3, 3, 1, 1, 2, 64, "u8"),  # conv groups = 2, Mg = 192
+    (2, 10, 10, 128, 64, 3, 3, 1, 1, 1, 64, "u4"),
+    (1, 9, 9, 64, 70, 3, 3, 1, 1, 1, 64, "s4"),
+    (3, 28, 28, 64, 64, 3, 3, 1, 1, 1, 64, "u8"),    # many tiles per CTA (persistent loop)
+]
+
+
+@pytest.mark.parametrize("case", TC_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_tc_conv2d_parity(case):
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()) + 1)
+    Cg = C // groups
+    w = (rng.standard_normal((M, R * S * Cg)) * np.sqrt(2.0 / (R * S * Cg))).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    fgq.fgq_set_path(fgq.PATH_TC)
+    gout = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride,
+                          pad, groups, to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    assert fgq.fgq_last_path() == fgq.PATH_TC
+    check_within(gout.cpu().numpy(), y, ym, f"tc conv2d {case}")
+
+
+@pytest.mark.parametrize("case", [(128, 64, 128, 64, "u8"), (1, 9216, 4096, 64, "u8"), (300, 256, 64, 128, "s8"),
+                                  (257, 1024, 1000, 64, "u8"), (64, 512, 130, 64, "u4")],
+                         ids=lambda c: "x".join(map(str, c)))
+def test_tc_gemm_parity(case):
+    P, K, M, G, act = case
+    rng = np.random.default_rng(P * 7 + K)
+    w = rng.standard_normal((M, K)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((P, K), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.gemm(q, sc, t, al, G)
+    fgq.fgq_set_path(fgq.PATH_TC)
+    gy = fgq.fgq_gemm(to_dev(packed), act, to_dev(np.array([sc], np.float32)), P, K, to_dev(codes.view(np.int32)),
+                      to_dev(al), M, G)
+    assert fgq.fgq_last_path() == fgq.PATH_TC
+    check_within(gy.cpu().numpy(), y, ym, f"tc gemm {case}")
+
+
+def test_tc_forced_on_unsupported_shape():
+    """A forced tensor-core path on a shape it cannot run returns FGQ_ERR_UNSUPPORTED."""
+    fgq.fgq_set_path(fgq.PATH_TC)
+    q = torch.zeros(64 * 48, dtype=torch.uint8, device=dev())
+    codes = torch.zeros((8, 4), dtype=torch.int32, device=dev())
+    al = torch.zeros((8, 1), dtype=torch.float32, device=dev())
+    with pytest.raises(fgq.FGQError) as e:
+        fgq.fgq_gemm(q, "u8", torch.ones(1, device=dev()), 64, 48, codes, al, 8, 64)
+    assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
