@@ -243,11 +243,12 @@ class Workload:
 
 
 def alu_peak_tops(G, sm_count, clk_hz):
-    """Issue-bound peak of the CUDA-core contraction: per (filter, position, group) it issues
-    G/4 dp4a plus one packed fp32x2 add and one packed fp32x2 FMA, each covering two
-    outputs (one issue per output), for 2G effective ops; an SM issues 4 x 32 lane
-    instructions per clock."""
-    return sm_count * 128 * clk_hz * (2.0 * G) / (G / 4 + 1) / 1e12
+    """ALU peak of the CUDA-core contraction in effective TOPS.  Per (filter, position,
+    group) it runs G/4 dp4a, which only the FMA-heavy pipe executes (64 lanes/clk/SM), plus
+    one fp32 add and one fp32 FMA, which the heavy and lite pipes share (128 lanes/clk/SM),
+    for 2G effective ops; the unit costs max((G/4)/64, (G/4 + 2)/128) clocks per SM."""
+    clk_per_unit = max((G / 4) / 64.0, (G / 4 + 2) / 128.0)
+    return sm_count * clk_hz * (2.0 * G) / clk_per_unit / 1e12
 
 
 def family_roofline(fam, layers, B, peaks, sm_count, sec_per_step, paths):

@@ -120,7 +120,7 @@ size_t fgq_quantize_act_workspace_bytes(size_t n);
  *              scale_in > 0); its contents on entry do not matter.
  * q_i = clamp(round_half_even(x_i * 2^-E), qmin, qmax), exact.  Two kernels when the scale
  * is derived (max reduction, then quantization); one when it is given.
- * Errors: FGQ_ERR_ARG, FGQ_ERR_ALIGN (x, q not 4-byte aligned; workspace not 4-byte
+ * Errors: FGQ_ERR_ARG, FGQ_ERR_ALIGN (x, q not 16-byte aligned; workspace not 4-byte
  * aligned or too small), FGQ_ERR_CUDA; NaN/Inf recorded as FGQ_ERR_NONFINITE.
  */
 fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float scale_in, void* q,
