@@ -128,6 +128,24 @@ fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float s
                             cudaStream_t stream);
 
 /*
+ * Allocation-free variant of fgq_quantize_act (no counterpart in the paper).  For callers
+ * that cannot allocate device memory themselves -- hosts whose device memory is owned by a
+ * framework pool with a fixed budget, plugins that only receive pre-allocated buffers, or
+ * latency-critical loops that cannot afford cudaMalloc/cudaFree (cudaFree synchronizes the
+ * device) -- it keeps the derived-scale pass's per-block maxima in a static 16 KB device
+ * array inside the library (4096 words), so no workspace argument is needed.  Arguments,
+ * results and errors are those of fgq_quantize_act; the caller still passes x, q and
+ * scale_out.  The call itself allocates nothing.  Its first call on each device looks up the
+ * array's device address (cudaGetSymbolAddress) with that device current, so make that
+ * first call before any stream capture.  Every GPU that loads the library holds the array
+ * until exit; all calls share it, so calls that overlap on the GPU (other streams or host
+ * threads) race and must be serialized.  Returns FGQ_ERR_UNSUPPORTED if the scale pass
+ * would need more than 4096 blocks (devices with more than 512 SMs).
+ */
+fgq_status fgq_quantize_act_noalloc(const float* x, size_t n, fgq_act_type type, float scale_in,
+                                    void* q, float* scale_out, cudaStream_t stream);
+
+/*
  * 8-bit weights for the first layer (Section 4: the first layer is kept at 8w-8a): each
  * filter row of w fp32 [M][Kred] is quantized as a signed 8-bit DFP vector, the same rule
  * as fgq_quantize_act with FGQ_S8 applied per row.  wq out int8 [M][Kred]; wscale out fp32

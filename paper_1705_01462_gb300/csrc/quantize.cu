@@ -15,6 +15,8 @@
 // the block maxima, derives E, and quantizes a grid-stride share of 16-element chunks.
 #include <climits>
 #include <cstdint>
+#include <cstring>
+#include <mutex>
 
 #include "fgq_device.cuh"
 
@@ -196,3 +198,77 @@ fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool
 }
 
 }  // namespace fgq
+
+// ----------------------------------------------------------------------------------------
+// fgq_quantize_act_noalloc: the derived-scale quantizer for callers that cannot allocate
+// device memory.  Some hosts own every device allocation themselves (a framework's memory
+// pool with a fixed budget, a plugin that only receives pre-allocated tensors) or cannot
+// afford cudaMalloc/cudaFree on the inference path (cudaFree synchronizes the device, and a
+// fresh allocation can stall or fail under memory pressure).  For them the per-block maxima
+// of pass 1 live in this file-scope device array instead of a caller-provided workspace.
+//
+// The array is a host-side stand-in in host code, not a device address, so its address is
+// obtained once per device with cudaGetSymbolAddress (with that device current) and passed
+// to the kernels.  That set-up happens in the first call on each device, which should
+// therefore come before any stream capture.  Every GPU that loads the library keeps the
+// array (16 KB) until exit.  All calls share it: each call fully rewrites the slots it uses
+// before reading them, so nothing needs clearing, but calls that overlap on the GPU (in
+// different streams, or from different threads) race on it and must be serialized.
+namespace fgq {
+namespace {
+
+constexpr int kNoallocScratchWords = 4096;  // maximum number of pass-1 blocks
+static __device__ __align__(256) uint32_t g_noalloc_scratch[kNoallocScratchWords];
+
+constexpr int kNoallocMaxDevices = 64;
+uint32_t* g_noalloc_ptr[kNoallocMaxDevices];
+std::mutex g_noalloc_mu;
+
+// Device address of the scratch array on the current device (nullptr on failure).
+uint32_t* noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoallocMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    g_noalloc_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  return g_noalloc_ptr[dev];
+}
+
+}  // namespace
+}  // namespace fgq
+
+extern "C" fgq_status fgq_quantize_act_noalloc(const float* x, size_t n, fgq_act_type type, float scale_in,
+                                               void* q, float* scale_out, cudaStream_t stream) {
+  using namespace fgq;
+  if (type != FGQ_U8 && type != FGQ_S8 && type != FGQ_U4 && type != FGQ_S4) return FGQ_ERR_ARG;
+  int E = 0;
+  const bool derive = !(scale_in > 0.0f);
+  if (!derive) {  // a given scale must be a power of two 2^E (subnormal ones included)
+    uint32_t b;
+    memcpy(&b, &scale_in, sizeof b);
+    const uint32_t ex = b >> 23, man = b & 0x7fffffu;
+    if (ex == 255) return FGQ_ERR_ARG;
+    if (ex > 0) {
+      if (man != 0) return FGQ_ERR_ARG;
+      E = (int)ex - 127;
+    } else {
+      if (man & (man - 1)) return FGQ_ERR_ARG;
+      E = -149 + (31 - __builtin_clz(man));
+    }
+  }
+  if (n == 0) return FGQ_OK;
+  if (!x || !q || (derive && !scale_out)) return FGQ_ERR_ARG;
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(q) & 15) ||
+      (scale_out && (reinterpret_cast<uintptr_t>(scale_out) & 3)))
+    return FGQ_ERR_ALIGN;
+  uint32_t* scratch = nullptr;
+  if (derive) {
+    if (quantize_workspace_bytes(n) > sizeof(uint32_t) * (size_t)kNoallocScratchWords) return FGQ_ERR_UNSUPPORTED;
+    scratch = noalloc_scratch();
+    if (!scratch) return FGQ_ERR_CUDA;
+  }
+  return launch_quantize(x, n, type, E, derive, q, scale_out, scratch, device_error_word(), stream);
+}

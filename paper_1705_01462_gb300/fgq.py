@@ -34,6 +34,7 @@ SIGNATURES = [
     ("fgq_ternarize", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
     ("fgq_quantize_act_workspace_bytes", _sz, [_sz]),
     ("fgq_quantize_act", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp, _sz, _vp]),
+    ("fgq_quantize_act_noalloc", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp]),
     ("fgq_quantize_weights_w8", _i, [_vp, _i, _i, _vp, _vp, _vp]),
     ("fgq_gemm", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
