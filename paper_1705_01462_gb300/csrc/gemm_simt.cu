@@ -5,14 +5,16 @@
 // dp4a instructions over int8x4 activation words and int8x4 code words expanded from the
 // 2-bit codes; the sum is then scaled by alpha into an fp32 accumulator.  The dp4a chain
 // starts at the bit pattern of 1.5*2^23, so its int32 result reads directly as the fp32
-// number 1.5*2^23 + s and one packed fp32x2 add recovers s exactly (no int->fp32
-// conversion instruction).  The group-scaled partials are accumulated with packed fp32x2
-// FMAs: per (filter, position, group) one dp4a per 4 weights plus one add and one FMA.
+// number 1.5*2^23 + s and one fp32 add recovers s exactly (no int->fp32 conversion
+// instruction).  Per (filter, position, group): one dp4a per 4 weights (FMA-heavy pipe)
+// plus one fp32 add and one fp32 FMA, which the heavy and lite FMA pipes share.
 //
 // Tiling: a 256-thread block computes 64 filters x 128 output positions; each thread owns
 // 4 filters x 8 positions.  The reduction axis is staged through shared memory in chunks
 // of max(16, G/4) words: activation words gathered from the implicit im2col (zero outside
 // the image), code words expanded through a 256-entry byte table, and the chunk's alphas.
+// The next chunk's global loads are issued into registers before the current chunk's
+// math (double-buffered shared tiles, one barrier per chunk).
 //
 // The same kernel runs the dense 8-bit-weight first layer (int32 dot product over the
 // whole row, scaled once at the end) and can write the raw int32 group sums.
@@ -70,7 +72,8 @@ __device__ __forceinline__ uint32_t act_byte(const uint8_t* act, int type, int64
 
 // Four consecutive reduction elements k..k+3 as an int8x4 word.
 // mode 0: 8-bit, 4-byte aligned word within one tap; 1: 4-bit, 2-byte word within one tap;
-// 2: byte-by-byte gather.
+// 2: byte-by-byte gather.  (Mode 3, whole 16-byte runs inside one tap, is handled by the
+// tiled kernel's staging directly.)
 __device__ __forceinline__ uint32_t act_word(const uint8_t* act, const Geom& g, const PosInfo& pi,
                                              int gi, int k, int mode) {
   if (!pi.valid || k >= g.Kred) return 0;
@@ -94,38 +97,138 @@ __device__ __forceinline__ uint32_t act_word(const uint8_t* act, const Geom& g, 
   return v;
 }
 
+#ifndef FGQ_SIMT_PACKED_FP
+#define FGQ_SIMT_PACKED_FP 0  // 1: packed fp32x2 add/FMA for the per-group scaling (measured 2-3% slower)
+#endif
+
+// Thread layout: tid -> filters 4*(tid % 16) .. +3 and positions {64j + 4*(tid / 16) + e :
+// j = 0, 1; e = 0..3}.  Lanes run along the filters, so each 16-byte output store of a warp
+// covers two whole 256-byte rows of y; the transposed activation tile As[word][position]
+// gives a thread 4 positions per 16-byte shared load.
 template <int G, bool SA, bool DW, bool SUMS>
-__global__ void __launch_bounds__(NT) simt_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
-                                                           const void* __restrict__ weights,
-                                                           const float* __restrict__ scales,
-                                                           const float* __restrict__ act_scale,
-                                                           float* __restrict__ out, int32_t* __restrict__ sums,
-                                                           int mode, int mtiles) {
+__global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
+                                                              const void* __restrict__ weights,
+                                                              const float* __restrict__ scales,
+                                                              const float* __restrict__ act_scale,
+                                                              float* __restrict__ out, int32_t* __restrict__ sums,
+                                                              int mode, int mtiles) {
   constexpr int KW = (G / 4 > 16) ? G / 4 : 16;  // words (4 elements) per chunk
   constexpr int GPC = DW ? 1 : (KW * 4) / G;     // groups per chunk
   constexpr int WPG = G / 4;                      // words per group
+  constexpr int SW = (BP * KW) / NT;              // activation words staged per thread
+  constexpr int CW = (BM * (KW / 4) + NT - 1) / NT;  // code words staged per thread
+  constexpr int AW = (BM * GPC + NT - 1) / NT;    // alphas staged per thread
 
-  __shared__ uint32_t As[BP][KW + 1];
-  __shared__ __align__(16) uint32_t Ws[KW][BM];
-  __shared__ __align__(16) float Al[GPC][BM];
-  __shared__ uint32_t lut[256];
+  extern __shared__ __align__(16) uint8_t smem_simt[];
+  uint32_t (*As)[KW][BP] = reinterpret_cast<uint32_t (*)[KW][BP]>(smem_simt);
+  uint32_t (*Ws)[KW][BM] = reinterpret_cast<uint32_t (*)[KW][BM]>(smem_simt + 2 * KW * BP * 4);
+  float (*Al)[GPC][BM] = reinterpret_cast<float (*)[GPC][BM]>(smem_simt + 2 * KW * BP * 4 + 2 * KW * BM * 4);
+  uint32_t* lut = reinterpret_cast<uint32_t*>(smem_simt + 2 * KW * BP * 4 + 2 * KW * BM * 4 + 2 * GPC * BM * 4);
 
   const int tid = threadIdx.x;
-  const int tx = tid % 16, ty = tid / 16;
+  const int ty = tid % 16, tx = tid / 16;
   const int gi = blockIdx.y / mtiles;
   const int mt = blockIdx.y - gi * mtiles;
-  const int mlo = gi * g.Mg + mt * BM;        // first filter of the block
-  const int mhi = min(gi * g.Mg + g.Mg, g.M);  // end of this conv group
+  const int mlo = gi * g.Mg + mt * BM;
+  const int mhi = min(gi * g.Mg + g.Mg, g.M);
   const int64_t p0 = (int64_t)blockIdx.x * BP;
 
   if (!DW) {
     for (int i = tid; i < 256; i += NT) lut[i] = expand_code_byte((uint32_t)i);
   }
 
-  // staging assignment: one position, half of the chunk's words
+  // staging assignment: activations -- one position, SW consecutive words of the chunk
   const int spl = tid % BP;
-  const int swr = tid / BP;
+  const int sw0 = (tid / BP) * SW;
   const PosInfo spi = pos_info(g, p0 + spl);
+  const uint32_t* codes = static_cast<const uint32_t*>(weights);
+  const int8_t* wq = static_cast<const int8_t*>(weights);
+
+  uint32_t ra[SW];  // prefetched activation words
+  uint32_t rc[DW ? (BM * KW + NT - 1) / NT : CW];  // prefetched code words / dense weight words
+  float ral[AW];
+
+  auto fetch = [&](int c) {
+    const int k0 = c * 4 * KW;
+    if (mode == 3) {
+      // fast path: this thread's 4*SW elements lie inside one filter tap (C/groups is a
+      // multiple of 4*SW) and start 16-byte aligned: one decomposition, 16-byte loads
+      const int k = k0 + 4 * sw0;
+      int64_t e = -1;
+      if (spi.valid && k < g.Kred) e = act_elem(g, spi, gi, k);
+#pragma unroll
+      for (int i = 0; i < SW; i += 4) {
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (e >= 0) v = __ldg(reinterpret_cast<const uint4*>(act + e) + i / 4);
+        ra[i] = v.x; ra[i + 1] = v.y; ra[i + 2] = v.z; ra[i + 3] = v.w;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < SW; ++i) ra[i] = act_word(act, g, spi, gi, k0 + 4 * (sw0 + i), mode);
+    }
+    if (!DW) {
+#pragma unroll
+      for (int r = 0; r < CW; ++r) {
+        const int idx = tid + r * NT;
+        const int ml = idx % BM, cw = idx / BM;
+        const int m = mlo + ml, wi = k0 / 16 + cw;
+        rc[r] = (idx < BM * (KW / 4) && m < mhi && wi < g.wrow) ? __ldg(codes + (int64_t)m * g.wrow + wi) : 0u;
+      }
+      if (!SUMS) {
+#pragma unroll
+        for (int r = 0; r < AW; ++r) {
+          const int idx = tid + r * NT;
+          const int ml = idx % BM, gl = idx / BM;
+          const int m = mlo + ml, gg = c * GPC + gl;
+          ral[r] = (idx < BM * GPC && m < mhi && gg < g.ng) ? __ldg(scales + (int64_t)m * g.ng + gg) : 0.0f;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int r = 0; r < (BM * KW + NT - 1) / NT; ++r) {
+        const int idx = tid + r * NT;
+        const int ml = idx % BM, kw = idx / BM;
+        const int m = mlo + ml;
+        uint32_t v = 0;
+        if (idx < BM * KW && m < mhi) {
+#pragma unroll
+          for (int b = 0; b < 4; ++b) {
+            const int k = k0 + 4 * kw + b;
+            if (k < g.Kred) v |= ((uint32_t)(uint8_t)wq[(int64_t)m * g.Kred + k]) << (8 * b);
+          }
+        }
+        rc[r] = v;
+      }
+    }
+  };
+  auto stash = [&](int buf) {
+#pragma unroll
+    for (int i = 0; i < SW; ++i) As[buf][sw0 + i][spl] = ra[i];
+    if (!DW) {
+#pragma unroll
+      for (int r = 0; r < CW; ++r) {
+        const int idx = tid + r * NT;
+        if (idx < BM * (KW / 4)) {
+          const int ml = idx % BM, cw = idx / BM;
+#pragma unroll
+          for (int b = 0; b < 4; ++b) Ws[buf][cw * 4 + b][ml] = lut[(rc[r] >> (8 * b)) & 0xffu];
+        }
+      }
+      if (!SUMS) {
+#pragma unroll
+        for (int r = 0; r < AW; ++r) {
+          const int idx = tid + r * NT;
+          if (idx < BM * GPC) Al[buf][idx / BM][idx % BM] = ral[r];
+        }
+      }
+    } else {
+#pragma unroll
+      for (int r = 0; r < (BM * KW + NT - 1) / NT; ++r) {
+        const int idx = tid + r * NT;
+        if (idx < BM * KW) Ws[buf][idx / BM][idx % BM] = rc[r];
+      }
+    }
+  };
 
   float acc[4][8];
   int iacc[4][8];
@@ -138,70 +241,31 @@ __global__ void __launch_bounds__(NT) simt_contract_kernel(const uint8_t* __rest
     }
 
   const int nchunks = (g.Kp + 4 * KW - 1) / (4 * KW);
-  const uint32_t* codes = static_cast<const uint32_t*>(weights);
-  const int8_t* wq = static_cast<const int8_t*>(weights);
+  fetch(0);
+  __syncthreads();  // lut ready
+  stash(0);
+  __syncthreads();
 
   for (int c = 0; c < nchunks; ++c) {
-    const int k0 = c * 4 * KW;
-    __syncthreads();
-    // activations
-#pragma unroll 4
-    for (int i = 0; i < KW / 2; ++i) {
-      const int kw = swr * (KW / 2) + i;
-      As[spl][kw] = act_word(act, g, spi, gi, k0 + 4 * kw, mode);
-    }
-    // weights
-    if (!DW) {
-      for (int idx = tid; idx < BM * (KW / 4); idx += NT) {
-        const int ml = idx % BM, cw = idx / BM;
-        const int m = mlo + ml;
-        const int wi = k0 / 16 + cw;
-        uint32_t word = 0;
-        if (m < mhi && wi < g.wrow) word = __ldg(codes + (int64_t)m * g.wrow + wi);
-#pragma unroll
-        for (int b = 0; b < 4; ++b) Ws[cw * 4 + b][ml] = lut[(word >> (8 * b)) & 0xffu];
-      }
-      for (int idx = tid; !SUMS && idx < BM * GPC; idx += NT) {
-        const int ml = idx % BM, gl = idx / BM;
-        const int m = mlo + ml;
-        const int gg = c * GPC + gl;
-        Al[gl][ml] = (m < mhi && gg < g.ng) ? __ldg(scales + (int64_t)m * g.ng + gg) : 0.0f;
-      }
-    } else {
-      for (int idx = tid; idx < BM * KW; idx += NT) {
-        const int ml = idx % BM, kw = idx / BM;
-        const int m = mlo + ml;
-        uint32_t v = 0;
-        if (m < mhi) {
-#pragma unroll
-          for (int b = 0; b < 4; ++b) {
-            const int k = k0 + 4 * kw + b;
-            if (k < g.Kred) v |= ((uint32_t)(uint8_t)wq[(int64_t)m * g.Kred + k]) << (8 * b);
-          }
-        }
-        Ws[kw][ml] = v;
-      }
-    }
-    __syncthreads();
+    const int buf = c & 1;
+    if (c + 1 < nchunks) fetch(c + 1);  // global loads in flight during this chunk's math
 
     if (DW) {
 #pragma unroll 4
       for (int kw = 0; kw < KW; ++kw) {
-        const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[kw][ty * 4]);
+        const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[buf][kw][ty * 4]);
         const uint32_t bv[4] = {bw.x, bw.y, bw.z, bw.w};
-        uint32_t a[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) a[j] = As[tx + 16 * j][kw];
+        const uint4 a0 = *reinterpret_cast<const uint4*>(&As[buf][kw][4 * tx]);
+        const uint4 a1 = *reinterpret_cast<const uint4*>(&As[buf][kw][64 + 4 * tx]);
+        const uint32_t a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
           for (int j = 0; j < 8; ++j) iacc[i][j] = SA ? dp4a_ss(a[j], bv[i], iacc[i][j]) : dp4a_us(a[j], bv[i], iacc[i][j]);
       }
     } else {
-#pragma unroll 1
+#pragma unroll 2
       for (int gl = 0; gl < GPC; ++gl) {
-        const float4 al4 = *reinterpret_cast<const float4*>(&Al[gl][ty * 4]);
-        const float al[4] = {al4.x, al4.y, al4.z, al4.w};
         int sm[4][8];
 #pragma unroll
         for (int i = 0; i < 4; ++i)
@@ -210,11 +274,11 @@ __global__ void __launch_bounds__(NT) simt_contract_kernel(const uint8_t* __rest
 #pragma unroll
         for (int wv = 0; wv < WPG; ++wv) {
           const int kw = gl * WPG + wv;
-          const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[kw][ty * 4]);
+          const uint4 bw = *reinterpret_cast<const uint4*>(&Ws[buf][kw][ty * 4]);
           const uint32_t bv[4] = {bw.x, bw.y, bw.z, bw.w};
-          uint32_t a[8];
-#pragma unroll
-          for (int j = 0; j < 8; ++j) a[j] = As[tx + 16 * j][kw];
+          const uint4 a0 = *reinterpret_cast<const uint4*>(&As[buf][kw][4 * tx]);
+          const uint4 a1 = *reinterpret_cast<const uint4*>(&As[buf][kw][64 + 4 * tx]);
+          const uint32_t a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
 #pragma unroll
           for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -229,46 +293,67 @@ __global__ void __launch_bounds__(NT) simt_contract_kernel(const uint8_t* __rest
               if (m >= mhi) continue;
 #pragma unroll
               for (int j = 0; j < 8; ++j) {
-                const int64_t p = p0 + tx + 16 * j;
+                const int64_t p = p0 + 64 * (j / 4) + 4 * tx + (j % 4);
                 if (p < g.P) sums[((int64_t)m * g.ng + gg) * g.P + p] = sm[i][j] - kMagicI;
               }
             }
           }
         } else {
-          const unsigned long long negc = pack_f2(-kMagicF, -kMagicF);
+          const float4 al4 = *reinterpret_cast<const float4*>(&Al[buf][gl][ty * 4]);
+          const float al[4] = {al4.x, al4.y, al4.z, al4.w};
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            const unsigned long long a2 = pack_f2(al[i], al[i]);
+            if (FGQ_SIMT_PACKED_FP) {
+              const unsigned long long negc = pack_f2(-kMagicF, -kMagicF);
+              const unsigned long long a2 = pack_f2(al[i], al[i]);
 #pragma unroll
-            for (int j = 0; j < 8; j += 2) {
-              const unsigned long long s2 = add_f2(pack_f2(__int_as_float(sm[i][j]), __int_as_float(sm[i][j + 1])), negc);
-              unsigned long long c2 = pack_f2(acc[i][j], acc[i][j + 1]);
-              c2 = fma_f2(a2, s2, c2);
-              unpack_f2(c2, acc[i][j], acc[i][j + 1]);
+              for (int j = 0; j < 8; j += 2) {
+                const unsigned long long s2 =
+                    add_f2(pack_f2(__int_as_float(sm[i][j]), __int_as_float(sm[i][j + 1])), negc);
+                unsigned long long c2 = pack_f2(acc[i][j], acc[i][j + 1]);
+                c2 = fma_f2(a2, s2, c2);
+                unpack_f2(c2, acc[i][j], acc[i][j + 1]);
+              }
+            } else {
+#pragma unroll
+              for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(al[i], __int_as_float(sm[i][j]) - kMagicF, acc[i][j]);
             }
           }
         }
       }
     }
+
+    if (c + 1 < nchunks) stash(buf ^ 1);
+    __syncthreads();
   }
 
   if (SUMS) return;
   const float sx = __ldg(act_scale);
+  const int m = mlo + ty * 4;
+  const bool vec = (g.M % 4 == 0) && (m + 3 < mhi);
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
-    const int64_t p = p0 + tx + 16 * j;
+    const int64_t p = p0 + 64 * (j / 4) + 4 * tx + (j % 4);
     if (p >= g.P) continue;
-    float* orow = out + p * g.M;
+    float v[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int m = mlo + ty * 4 + i;
-      if (m >= mhi) continue;
-      float v;
-      if (DW) v = sx * __ldg(scales + m) * (float)iacc[i][j];
-      else v = sx * acc[i][j];
-      orow[m] = v;
+    for (int i = 0; i < 4; ++i) v[i] = DW ? sx * __ldg(scales + min(m + i, g.M - 1)) * (float)iacc[i][j] : sx * acc[i][j];
+    float* orow = out + p * g.M;
+    if (vec) {
+      *reinterpret_cast<float4*>(orow + m) = make_float4(v[0], v[1], v[2], v[3]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (m + i < mhi) orow[m + i] = v[i];
     }
   }
+}
+
+template <int G, bool DW>
+constexpr size_t simt_smem_bytes() {
+  constexpr int KW = (G / 4 > 16) ? G / 4 : 16;
+  constexpr int GPC = DW ? 1 : (KW * 4) / G;
+  return (size_t)2 * KW * BP * 4 + 2 * KW * BM * 4 + 2 * GPC * BM * 4 + 256 * 4;
 }
 
 // Plain reference-style kernel for any G (used for G = 1 and 2): one thread per output.
@@ -301,10 +386,17 @@ __global__ void simple_contract_kernel(const uint8_t* __restrict__ act, const Ge
 template <int G, bool SA, bool DW, bool SUMS>
 void launch_one(const void* act, const Geom& g, const void* w, const float* sc, const float* as, float* out,
                 int32_t* sums, int mode, cudaStream_t s) {
+  constexpr size_t smem = simt_smem_bytes<G, DW>();
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaFuncSetAttribute(simt_contract_kernel<G, SA, DW, SUMS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    attr_set = true;
+  }
   const int mtiles = (g.Mg + BM - 1) / BM;
   dim3 grid((unsigned)((g.P + BP - 1) / BP), (unsigned)(mtiles * g.groups));
-  simt_contract_kernel<G, SA, DW, SUMS><<<grid, NT, 0, s>>>(static_cast<const uint8_t*>(act), g, w, sc, as, out,
-                                                            sums, mode, mtiles);
+  simt_contract_kernel<G, SA, DW, SUMS><<<grid, NT, smem, s>>>(static_cast<const uint8_t*>(act), g, w, sc, as, out,
+                                                               sums, mode, mtiles);
 }
 
 template <bool SA, bool SUMS>
@@ -331,6 +423,10 @@ fgq_status launch_simt_contract(const void* act, const Geom& g, const void* weig
   // gather mode: whole words inside one tap need Cg % 4 == 0 (and alignment of the words)
   int mode = 2;
   if (g.Cg % 4 == 0 && g.C % 4 == 0) mode = is4 ? 1 : 0;
+  // 8-bit activations whose per-thread staging run (32 elements; 64 when G = 128) stays in
+  // one tap and starts 16-byte aligned
+  const int run = (g.G == 128) ? 64 : 32;
+  if (!is4 && !dense && g.G >= 4 && g.Cg % run == 0 && g.C % 16 == 0) mode = 3;
   if (!dense && (g.G == 1 || g.G == 2)) {
     const int64_t n = g.P * g.M;
     simple_contract_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(

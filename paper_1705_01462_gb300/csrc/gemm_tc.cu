@@ -12,14 +12,17 @@
 // it by alpha[m][g] and adds it into an fp32 register accumulator (one multiply per group,
 // Section 4.1).  Two TMEM buffers let group g+1's MMAs run while group g is drained.
 //
-// Warp roles (288 threads, one CTA per SM, persistent over tiles):
-//   warps 0-3  epilogue: thread t owns filter row t of the tile (TMEM lane t); per group
-//              tcgen05.ld of the 128 columns, FMA with alpha, at tile end fp32 stores.
-//   warps 4-7  loaders/converters: thread t owns activation row t (one output position,
+// Warp roles (416 threads, one CTA per SM, persistent over tiles):
+//   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
+//              64*(w/4).. (positions) of the drained buffer: one 64-column tcgen05.ld and
+//              one wait per group, release of the buffer, then 64 FMAs with alpha into
+//              fp32 registers; fp32 stores at tile end.
+//   warps 8-11 loaders/converters: thread t owns activation row t (one output position,
 //              implicit im2col) and code row t (one filter) of every K-tile; cp.async
 //              copies raw bytes into a 6-deep staging ring, then the thread converts its
 //              own rows to fp16 in the 128-byte-swizzled K-major layout the MMA reads.
-//   warp 8     MMA issuer (one thread): 4 tcgen05.mma (K = 16) per K-tile.
+//   warp 12    TMEM allocation and the MMA issuer (one thread): 4 tcgen05.mma (K = 16)
+//              per K-tile into one of four 128-column TMEM accumulators.
 // Every mbarrier wait is bounded; on expiry the kernel records FGQ_ERR_TIMEOUT, every
 // role leaves its loop, in-flight copies and MMAs are waited for, and TMEM is freed.
 #include <cstdint>
@@ -33,10 +36,14 @@ namespace {
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 128;        // positions per tile (MMA N)
 constexpr int TC_KT = 64;         // reduction elements per K-tile
-constexpr int TC_NO = 3;          // operand ring depth
+constexpr int TC_NO = 4;          // operand ring depth
 constexpr int TC_NS = 6;          // staging ring depth
-constexpr int TC_THREADS = 288;
-constexpr int TC_TMEM_COLS = 256; // two 128-column fp32 accumulators
+constexpr int TC_NACC = 4;        // TMEM accumulator buffers
+constexpr int TC_EPI_WARPS = 8;
+constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // loaders: warps 8-11
+constexpr int TC_MMA_WARP = TC_EPI_WARPS + 4;    // warp 12
+constexpr int TC_THREADS = 32 * (TC_MMA_WARP + 1);
+constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
 constexpr uint32_t TC_WAIT_LIMIT = 1u << 22;
 
 constexpr int OP_TILE = TC_BM * TC_KT * 2;            // 16 KB: one fp16 operand tile
@@ -46,8 +53,9 @@ constexpr int ST_CODE = TC_BM * 16;                    // 2 KB raw code words
 constexpr int ST_STAGE = ST_ACT + ST_CODE;
 constexpr int SMEM_OP = TC_NO * OP_STAGE;
 constexpr int SMEM_ST = TC_NS * ST_STAGE;
-constexpr int SMEM_BAR = 8 * (2 * TC_NO + 4 + 1) + 16;
-constexpr int TC_SMEM = 1024 + SMEM_OP + SMEM_ST + SMEM_BAR;
+constexpr int SMEM_LUT = 256 * 8;                      // code byte -> 4 fp16
+constexpr int SMEM_BAR = 8 * (2 * TC_NO + 2 * TC_NACC + 1) + 16;
+constexpr int TC_SMEM = 1024 + SMEM_OP + SMEM_ST + SMEM_LUT + SMEM_BAR;
 
 struct TcArgs {
   const uint8_t* act;
@@ -94,13 +102,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* op = smem;                       // TC_NO x {A tile, B tile}
   uint8_t* st = smem + SMEM_OP;             // TC_NS x {act bytes, code bytes}
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP + SMEM_ST);
+  uint2* lut = reinterpret_cast<uint2*>(smem + SMEM_OP + SMEM_ST);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP + SMEM_ST + SMEM_LUT);
   uint64_t* op_full = bars;
   uint64_t* op_empty = bars + TC_NO;
   uint64_t* acc_full = bars + 2 * TC_NO;
-  uint64_t* acc_empty = bars + 2 * TC_NO + 2;
-  uint64_t* drain_bar = bars + 2 * TC_NO + 4;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * TC_NO + 5);
+  uint64_t* acc_empty = bars + 2 * TC_NO + TC_NACC;
+  uint64_t* drain_bar = bars + 2 * TC_NO + 2 * TC_NACC;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile uint32_t* abort_flag = tmem_slot + 1;
 
   const int warp = threadIdx.x >> 5;
@@ -112,15 +121,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
       mbar_init(&op_full[i], 128);
       mbar_init(&op_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < TC_NACC; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], 128);
+      mbar_init(&acc_empty[i], 32 * TC_EPI_WARPS);
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 8) {
+  // code byte (four 2-bit codes) -> four fp16 {0, +1, -1}
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+    uint32_t h[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t c = (i >> (2 * e)) & 3u;
+      h[e] = c == 1u ? 0x3C00u : (c == 3u ? 0xBC00u : 0u);
+    }
+    lut[i] = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+  }
+  if (warp == TC_MMA_WARP) {
     tmem_alloc(tmem_slot, TC_TMEM_COLS);
     tmem_relinquish();
   }
@@ -128,6 +147,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
 
   auto fail = [&]() {
     *abort_flag = 1;
@@ -135,51 +155,52 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   };
 
   // ------------------------------------------------------------------ loaders/converters
-  if (warp >= 4 && warp < 8) {
-    const int t = threadIdx.x - 128;  // row owned in every tile
-    const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+  if (warp >= TC_LOAD_WARP0 && warp < TC_MMA_WARP) {
+    const int t = threadIdx.x - 32 * TC_LOAD_WARP0;  // row owned in every tile
     const int total = my_tiles * a.ktiles;
     constexpr int ACT_BYTES = TC_KT * ABITS / 8;  // 64 (8-bit) or 32 (4-bit) bytes per row
     constexpr int ACT_CHUNKS = ACT_BYTES / 16;
 
-    // issue the copies of this CTA's j-th K-tile into staging slot j % TC_NS
+    // per-tile state of this thread's rows (refreshed when the issued K-tile enters a new tile)
+    int cur_tile = -1, gi = 0, m0 = 0, pb = 0, phb = 0, pwb = 0;
+    bool pvalid = false;
     auto issue = [&](int j) {
       const int tl = j / a.ktiles;
       const int kk = j - tl * a.ktiles;
-      int gi, m0;
-      int64_t p0;
-      tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+      if (tl != cur_tile) {
+        cur_tile = tl;
+        int64_t p0;
+        tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+        const int64_t p = p0 + t;
+        pvalid = p < g.P;
+        const int pp = pvalid ? (int)p : 0;
+        const int wo = pp % g.Wo;
+        const int q = pp / g.Wo;
+        const int ho = q % g.Ho;
+        pb = q / g.Ho;
+        phb = ho * g.stride - g.pad;
+        pwb = wo * g.stride - g.pad;
+      }
       uint8_t* sa = st + (j % TC_NS) * ST_STAGE;
       const uint32_t sact = smem_u32(sa + t * ACT_BYTES);
       const uint32_t scode = smem_u32(sa + ST_ACT + t * 16);
       const int k0 = kk * TC_KT;
-      // activation row: output position p0 + t, reduction elements k0 .. k0+63
-      const int64_t p = p0 + t;
       const uint8_t* src = a.act;
-      int valid_bytes = 0;
-      if (p < g.P) {
-        const int wo = (int)(p % g.Wo);
-        const int64_t q = p / g.Wo;
-        const int ho = (int)(q % g.Ho);
-        const int b = (int)(q / g.Ho);
+      bool inside = false;
+      if (pvalid) {
         const int tap = k0 / g.Cg;
         const int c0 = k0 - tap * g.Cg;
-        const int r = tap / g.S, s = tap - (tap / g.S) * g.S;
-        const int hi = ho * g.stride - g.pad + r, wi = wo * g.stride - g.pad + s;
+        const int r = tap / g.S, s = tap - r * g.S;
+        const int hi = phb + r, wi = pwb + s;
         if (hi >= 0 && hi < g.H && wi >= 0 && wi < g.W) {
-          const int64_t e = (((int64_t)b * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + c0;
+          const int64_t e = (((int64_t)pb * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + c0;
           src = a.act + e * ABITS / 8;
-          const int remain = (g.Cg - c0) * ABITS / 8;  // bytes of this pixel's group channels left
-          valid_bytes = remain < ACT_BYTES ? remain : ACT_BYTES;
+          inside = true;
         }
       }
 #pragma unroll
-      for (int c = 0; c < ACT_CHUNKS; ++c) {
-        int nb = valid_bytes - 16 * c;
-        nb = nb < 0 ? 0 : (nb > 16 ? 16 : nb);
-        cp_async16(sact + 16 * c, nb ? (const void*)(src + 16 * c) : (const void*)a.act, (uint32_t)nb);
-      }
-      // code row: filter m0 + t, code words k0/16 .. k0/16 + 3
+      for (int c = 0; c < ACT_CHUNKS; ++c)
+        cp_async16(sact + 16 * c, inside ? (const void*)(src + 16 * c) : (const void*)a.act, inside ? 16u : 0u);
       const int m = m0 + t;
       const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
       const uint32_t* csrc = mok ? a.codes + (int64_t)m * g.wrow + k0 / 16 : a.codes;
@@ -196,7 +217,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
       cp_async_commit();
       cp_async_wait<TC_NS - 1>();  // this thread's copies of K-tile j have landed
       const int os = j % TC_NO;
-      if (!mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag) || *abort_flag) {
+      if (!mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)) {
         if (!*abort_flag) fail();
         ok = false;
         break;
@@ -232,12 +253,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             // 8 nibbles -> 8 bytes (element order preserved), then 8 fp16
-            uint32_t x = w4[q];
-            uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);          // elements 0,1 / 4,5
-            uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // 2,3 / 6,7
-            uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                // bytes e0 e1 e2 e3
-            uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                        // bytes e4 e5 e6 e7
-            if (SIGNED) { b0 ^= 0x08080808u; b1 ^= 0x08080808u; }
+            const uint32_t x = w4[q];
+            const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
+            const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
+            uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                            // e0 e1 e2 e3
+            uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                                    // e4 e5 e6 e7
+            if (SIGNED) {
+              b0 ^= 0x08080808u;
+              b1 ^= 0x08080808u;
+            }
             uint4 o;
             o.x = u8pair_to_h2(b0, 0x4140, bias2); o.y = u8pair_to_h2(b0, 0x4342, bias2);
             o.z = u8pair_to_h2(b1, 0x4140, bias2); o.w = u8pair_to_h2(b1, 0x4342, bias2);
@@ -245,22 +269,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
           }
         }
       }
-      // codes -> fp16 row t of A: 64 codes, 8 per 16-byte chunk
+      // codes -> fp16 row t of A: 64 codes, 8 per 16-byte chunk, 4 per table lookup
       {
         const uint4 cv = *reinterpret_cast<const uint4*>(sa + ST_ACT + t * 16);
         const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           const uint32_t bits = (cw[c / 2] >> (16 * (c & 1))) & 0xffffu;  // 8 codes
-          uint32_t h[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const uint32_t c0 = (bits >> (4 * e)) & 3u, c1 = (bits >> (4 * e + 2)) & 3u;
-            const uint32_t lo = ((c0 & 1u) * 0x3C00u) | ((c0 & 2u) << 14);
-            const uint32_t hi2 = ((c1 & 1u) * 0x3C00u) | ((c1 & 2u) << 14);
-            h[e] = lo | (hi2 << 16);
-          }
-          *reinterpret_cast<uint4*>(A + sw128(t, c)) = make_uint4(h[0], h[1], h[2], h[3]);
+          const uint2 lo = lut[bits & 0xffu], hi = lut[bits >> 8];
+          *reinterpret_cast<uint4*>(A + sw128(t, c)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
         }
       }
       fence_proxy_async_smem();
@@ -270,16 +287,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   }
 
   // ------------------------------------------------------------------ MMA issuer
-  if (warp == 8 && lane == 0) {
+  if (warp == TC_MMA_WARP && lane == 0) {
     const uint32_t idesc = idesc_f16_f32(TC_BM, TC_BN);
-    const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
     const uint32_t op_base = smem_u32(op);
     int kt = 0, gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
       for (int grp = 0; grp < g.ng && ok; ++grp, ++gc) {
-        const int b = gc & 1;
-        if (!mbar_wait_or_abort(&acc_empty[b], ((gc >> 1) & 1) ^ 1, a.wait_limit, abort_flag) || *abort_flag) {
+        const int b = gc % TC_NACC;
+        if (!mbar_wait_or_abort(&acc_empty[b], ((gc / TC_NACC) & 1) ^ 1, a.wait_limit, abort_flag)) {
           if (!*abort_flag) fail();
           ok = false;
           break;
@@ -288,7 +304,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
         const uint32_t d = tmem + (uint32_t)(b * TC_BN);
         for (int sub = 0; sub < a.kt_per_group; ++sub, ++kt) {
           const int os = kt % TC_NO;
-          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag) || *abort_flag) {
+          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag)) {
             if (!*abort_flag) fail();
             ok = false;
             break;
@@ -313,11 +329,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   }
 
   // ------------------------------------------------------------------ epilogue
-  if (warp < 4) {
-    const int t = threadIdx.x;  // TMEM lane = filter row of the tile
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  if (warp < TC_EPI_WARPS) {
+    const int quarter = warp & 3, half = warp >> 2;
+    const int t = 32 * quarter + lane;  // TMEM lane = filter row of the tile
+    const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(64 * half);
     const float sx = __ldg(a.act_scale);
-    const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
     int gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
@@ -327,34 +343,36 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
       const int m = m0 + t;
       const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
       const float* arow = a.alpha + (int64_t)(mok ? m : 0) * g.ng;
-      float acc[TC_BN];
+      float acc[64];
 #pragma unroll
-      for (int j = 0; j < TC_BN; ++j) acc[j] = 0.0f;
+      for (int j = 0; j < 64; ++j) acc[j] = 0.0f;
       for (int grp = 0; grp < g.ng; ++grp, ++gc) {
-        const int b = gc & 1;
+        const int b = gc % TC_NACC;
         const float al = mok ? __ldg(arow + grp) : 0.0f;
-        if (!mbar_wait_or_abort(&acc_full[b], (gc >> 1) & 1, a.wait_limit, abort_flag) || *abort_flag) {
+        if (!mbar_wait_or_abort(&acc_full[b], (gc / TC_NACC) & 1, a.wait_limit, abort_flag)) {
           if (!*abort_flag) fail();
           ok = false;
           break;
         }
         tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < TC_BN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_base + (uint32_t)(b * TC_BN + 32 * c), r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) acc[32 * c + j] = fmaf(al, __uint_as_float(r[j]), acc[32 * c + j]);
-        }
+        uint32_t r0[32], r1[32];
+        tmem_ld32(tbase + (uint32_t)(b * TC_BN), r0);
+        tmem_ld32(tbase + (uint32_t)(b * TC_BN + 32), r1);
+        tmem_ld_wait();
         tc_fence_before();
-        mbar_arrive(&acc_empty[b]);
+        mbar_arrive(&acc_empty[b]);  // the buffer is free once the values are in registers
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          acc[j] = fmaf(al, __uint_as_float(r0[j]), acc[j]);
+          acc[32 + j] = fmaf(al, __uint_as_float(r1[j]), acc[32 + j]);
+        }
       }
       if (!ok) break;
       if (mok) {
+        const int64_t pbase = p0 + 64 * half;
 #pragma unroll
-        for (int j = 0; j < TC_BN; ++j) {
-          const int64_t p = p0 + j;
+        for (int j = 0; j < 64; ++j) {
+          const int64_t p = pbase + j;
           if (p < g.P) a.out[p * g.M + m] = sx * acc[j];
         }
       }
@@ -363,7 +381,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == TC_MMA_WARP) {
     tc_fence_after();
     tmem_dealloc(tmem, TC_TMEM_COLS);
   }
@@ -401,6 +419,7 @@ bool tc_supports(const Geom& g) {
   if (g.G != 64 && g.G != 128) return false;
   if (g.Cg % TC_KT != 0) return false;     // every K-tile inside one filter tap (conv) or row (GEMM)
   if (g.C % 16 != 0) return false;         // 16-byte aligned activation rows
+  if (g.P >= (int64_t)1 << 31) return false;  // positions decoded in 32 bits
   return true;
 }
 
