@@ -97,6 +97,9 @@ __device__ __forceinline__ uint32_t act_word(const uint8_t* act, const Geom& g, 
   return v;
 }
 
+#ifndef FGQ_SIMT_MIN_BLOCKS
+#define FGQ_SIMT_MIN_BLOCKS 2  // resident blocks per SM the register allocation targets
+#endif
 #ifndef FGQ_SIMT_PACKED_FP
 #define FGQ_SIMT_PACKED_FP 0  // 1: packed fp32x2 add/FMA for the per-group scaling (measured 2-3% slower)
 #endif
@@ -105,8 +108,26 @@ __device__ __forceinline__ uint32_t act_word(const uint8_t* act, const Geom& g, 
 // j = 0, 1; e = 0..3}.  Lanes run along the filters, so each 16-byte output store of a warp
 // covers two whole 256-byte rows of y; the transposed activation tile As[word][position]
 // gives a thread 4 positions per 16-byte shared load.
+// Mode 4: the byte gather of mode 2 driven by a per-block table tbl[k] = r | s << 8 | c << 16
+// of the reduction index's filter tap and channel (all ones past Kred), built once per block.
+__device__ __forceinline__ uint32_t act_word_tbl(const uint8_t* act, const Geom& g, const PosInfo& pi, int gi,
+                                                 int k, const uint32_t* tbl) {
+  if (!pi.valid) return 0;
+  uint32_t v = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t e = tbl[k + i];
+    if (e == 0xffffffffu) continue;
+    const int hi = pi.hb + (int)(e & 0xffu), wi = pi.wb + (int)((e >> 8) & 0xffu);
+    if (hi < 0 || hi >= g.H || wi < 0 || wi >= g.W) continue;
+    const int64_t el = (((int64_t)pi.b * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + (int)(e >> 16);
+    v |= act_byte(act, g.act_type, el) << (8 * i);
+  }
+  return v;
+}
+
 template <int G, bool SA, bool DW, bool SUMS>
-__global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
+__global__ void __launch_bounds__(NT, FGQ_SIMT_MIN_BLOCKS) simt_contract_kernel(const uint8_t* __restrict__ act, const Geom g,
                                                               const void* __restrict__ weights,
                                                               const float* __restrict__ scales,
                                                               const float* __restrict__ act_scale,
@@ -124,6 +145,7 @@ __global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __r
   uint32_t (*Ws)[KW][BM] = reinterpret_cast<uint32_t (*)[KW][BM]>(smem_simt + 2 * KW * BP * 4);
   float (*Al)[GPC][BM] = reinterpret_cast<float (*)[GPC][BM]>(smem_simt + 2 * KW * BP * 4 + 2 * KW * BM * 4);
   uint32_t* lut = reinterpret_cast<uint32_t*>(smem_simt + 2 * KW * BP * 4 + 2 * KW * BM * 4 + 2 * GPC * BM * 4);
+  uint32_t* ktab = lut + 256;  // mode 4 only: one entry per reduction index of all chunks
 
   const int tid = threadIdx.x;
   const int ty = tid % 16, tx = tid / 16;
@@ -135,6 +157,19 @@ __global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __r
 
   if (!DW) {
     for (int i = tid; i < 256; i += NT) lut[i] = expand_code_byte((uint32_t)i);
+  }
+  const int nchunks = (g.Kp + 4 * KW - 1) / (4 * KW);
+  if (mode == 4) {
+    for (int k = tid; k < nchunks * 4 * KW; k += NT) {
+      uint32_t e = 0xffffffffu;
+      if (k < g.Kred) {
+        const int tap = k / g.Cg, c = k - (k / g.Cg) * g.Cg;
+        const int r = tap / g.S, s2 = tap - (tap / g.S) * g.S;
+        e = (uint32_t)r | ((uint32_t)s2 << 8) | ((uint32_t)c << 16);
+      }
+      ktab[k] = e;
+    }
+    __syncthreads();
   }
 
   // staging assignment: activations -- one position, SW consecutive words of the chunk
@@ -162,6 +197,9 @@ __global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __r
         if (e >= 0) v = __ldg(reinterpret_cast<const uint4*>(act + e) + i / 4);
         ra[i] = v.x; ra[i + 1] = v.y; ra[i + 2] = v.z; ra[i + 3] = v.w;
       }
+    } else if (mode == 4) {
+#pragma unroll
+      for (int i = 0; i < SW; ++i) ra[i] = act_word_tbl(act, g, spi, gi, k0 + 4 * (sw0 + i), ktab);
     } else {
 #pragma unroll
       for (int i = 0; i < SW; ++i) ra[i] = act_word(act, g, spi, gi, k0 + 4 * (sw0 + i), mode);
@@ -240,7 +278,6 @@ __global__ void __launch_bounds__(NT, 2) simt_contract_kernel(const uint8_t* __r
       iacc[i][j] = 0;
     }
 
-  const int nchunks = (g.Kp + 4 * KW - 1) / (4 * KW);
   fetch(0);
   __syncthreads();  // lut ready
   stash(0);
@@ -386,12 +423,14 @@ __global__ void simple_contract_kernel(const uint8_t* __restrict__ act, const Ge
 template <int G, bool SA, bool DW, bool SUMS>
 void launch_one(const void* act, const Geom& g, const void* w, const float* sc, const float* as, float* out,
                 int32_t* sums, int mode, cudaStream_t s) {
-  constexpr size_t smem = simt_smem_bytes<G, DW>();
-  static bool attr_set = false;
-  if (!attr_set) {
+  constexpr int KW = (G / 4 > 16) ? G / 4 : 16;
+  const size_t nk = (size_t)((g.Kp + 4 * KW - 1) / (4 * KW)) * 4 * KW;
+  const size_t smem = simt_smem_bytes<G, DW>() + (mode == 4 ? 4 * nk : 0);
+  static int attr_set = 0;
+  if (attr_set < (int)smem) {
     cudaFuncSetAttribute(simt_contract_kernel<G, SA, DW, SUMS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
-    attr_set = true;
+                         (int)(smem > 48 * 1024 ? smem : 48 * 1024));
+    attr_set = (int)(smem > 48 * 1024 ? smem : 48 * 1024);
   }
   const int mtiles = (g.Mg + BM - 1) / BM;
   dim3 grid((unsigned)((g.P + BP - 1) / BP), (unsigned)(mtiles * g.groups));
@@ -427,6 +466,8 @@ fgq_status launch_simt_contract(const void* act, const Geom& g, const void* weig
   // one tap and starts 16-byte aligned
   const int run = (g.G == 128) ? 64 : 32;
   if (!is4 && !dense && g.G >= 4 && g.Cg % run == 0 && g.C % 16 == 0) mode = 3;
+  // byte gathers driven by a per-block (tap, channel) table while it fits in shared memory
+  if (mode == 2 && g.Kp <= 8192) mode = 4;
   if (!dense && (g.G == 1 || g.G == 2)) {
     const int64_t n = g.P * g.M;
     simple_contract_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(

@@ -10,22 +10,34 @@
 // MMA chain is 64 and aligned to the group, so after a group's MMAs the TMEM accumulator
 // holds exactly s[m][g][p] for a 128-filter x 128-position tile; the epilogue multiplies
 // it by alpha[m][g] and adds it into an fp32 register accumulator (one multiply per group,
-// Section 4.1).  Two TMEM buffers let group g+1's MMAs run while group g is drained.
+// Section 4.1).  Four TMEM buffers let the MMAs of later groups run while a group drains.
 //
 // Warp roles (416 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
 //              64*(w/4).. (positions) of the drained buffer: one 64-column tcgen05.ld and
-//              one wait per group, release of the buffer, then 64 FMAs with alpha into
-//              fp32 registers; fp32 stores at tile end.
-//   warps 8-11 loaders/converters: thread t owns activation row t (one output position,
-//              implicit im2col) and code row t (one filter) of every K-tile; cp.async
-//              copies raw bytes into a 6-deep staging ring, then the thread converts its
-//              own rows to fp16 in the 128-byte-swizzled K-major layout the MMA reads.
+//              two 32-column tcgen05.ld per group, release of the buffer, FMAs with alpha into
+//              fp32 registers.  At tile end the fp32 tile goes to shared memory and one
+//              thread writes it to HBM with a TMA box store (direct stores when the
+//              output has several conv groups or M % 4 != 0).
+//   warps 8-11 loaders/converters: per K-tile one thread issues a TMA box load of the
+//              tile's 128 code rows (16 bytes each) and, for layers whose im2col rows are
+//              contiguous input rows (1x1 stride-1 convolutions, GEMMs), one TMA box load
+//              of the 128 activation rows; for other layers each thread copies its own
+//              activation row and code row with 16-byte cp.async.  Thread t converts row t of both
+//              tiles to fp16 in the 128-byte-swizzled K-major layout the MMA reads; a
+//              staging slot is refilled by TMA only after every loader has released it
+//              (st_empty), so the loader warps never wait for each other otherwise.
 //   warp 12    TMEM allocation and the MMA issuer (one thread): 4 tcgen05.mma (K = 16)
 //              per K-tile into one of four 128-column TMEM accumulators.
-// Every mbarrier wait is bounded; on expiry the kernel records FGQ_ERR_TIMEOUT, every
-// role leaves its loop, in-flight copies and MMAs are waited for, and TMEM is freed.
+// Every mbarrier wait is bounded; on expiry the kernel records FGQ_ERR_TIMEOUT, each role
+// leaves its loop (uniformly within a role that uses named barriers), in-flight copies
+// and MMAs are waited for, and TMEM is freed.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <cstdint>
+#include <cstring>
+#include <mutex>
 
 #include "fgq_device.cuh"
 #include "ptx_sm100.cuh"
@@ -36,28 +48,41 @@ namespace {
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 128;        // positions per tile (MMA N)
 constexpr int TC_KT = 64;         // reduction elements per K-tile
-constexpr int TC_NO = 4;          // operand ring depth
-constexpr int TC_NS = 6;          // staging ring depth
+constexpr int TC_NO = 3;          // operand ring depth
+constexpr int TC_NS_TMA = 6;      // staging ring depth of the TMA path (room for the output tile)
+constexpr int TC_NS_GATHER = 12;  // staging ring depth of the gather path (about 1.5 us of copies)
 constexpr int TC_NACC = 4;        // TMEM accumulator buffers
 constexpr int TC_EPI_WARPS = 8;
-constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // loaders: warps 8-11
-constexpr int TC_MMA_WARP = TC_EPI_WARPS + 4;    // warp 12
+constexpr int TC_LOAD_WARPS = 4;
+constexpr int TC_LOADERS = 32 * TC_LOAD_WARPS;  // loader threads
+constexpr int TC_LPR = TC_LOADERS / 128;         // loader threads per tile row
+static_assert(TC_LPR == 1, "the cp.async gather path reads only copies made by the same thread");
+constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // loaders: warps 8 .. 8 + TC_LOAD_WARPS - 1
+constexpr int TC_MMA_WARP = TC_EPI_WARPS + TC_LOAD_WARPS;  // warp 16
 constexpr int TC_THREADS = 32 * (TC_MMA_WARP + 1);
 constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
-constexpr uint32_t TC_WAIT_LIMIT = 1u << 22;
+constexpr uint32_t TC_WAIT_LIMIT = 50000;        // polls of up to 20 us: about 1 s per wait
+constexpr uint32_t BAR_EPI = 2;                  // named barrier of the 256 epilogue threads
 
 constexpr int OP_TILE = TC_BM * TC_KT * 2;            // 16 KB: one fp16 operand tile
 constexpr int OP_STAGE = 2 * OP_TILE;                  // A (codes) + B (activations)
 constexpr int ST_ACT = TC_BN * TC_KT;                  // 8 KB raw activation bytes (8-bit)
 constexpr int ST_CODE = TC_BM * 16;                    // 2 KB raw code words
 constexpr int ST_STAGE = ST_ACT + ST_CODE;
+constexpr int OUT_TILE = TC_BN * TC_BM * 4;            // 64 KB fp32 output tile
 constexpr int SMEM_OP = TC_NO * OP_STAGE;
-constexpr int SMEM_ST = TC_NS * ST_STAGE;
-constexpr int SMEM_LUT = 256 * 8;                      // code byte -> 4 fp16
-constexpr int SMEM_BAR = 8 * (2 * TC_NO + 2 * TC_NACC + 1) + 16;
-constexpr int TC_SMEM = 1024 + SMEM_OP + SMEM_ST + SMEM_LUT + SMEM_BAR;
+constexpr int SMEM_LUT = 16 * 32 * 4;                  // 2 codes -> 2 fp16, one copy per bank
+constexpr int SMEM_BAR = 8 * (2 * TC_NO + 2 * TC_NS_GATHER + 2 * TC_NACC + 1) + 16;
+// TMA path: staging ring + fp32 output tile; gather path: a deeper staging ring, no tile.
+constexpr int SMEM_MID_TMA = TC_NS_TMA * ST_STAGE + OUT_TILE;
+constexpr int SMEM_MID_GATHER = TC_NS_GATHER * ST_STAGE;
+constexpr int SMEM_MID = SMEM_MID_TMA > SMEM_MID_GATHER ? SMEM_MID_TMA : SMEM_MID_GATHER;
+constexpr int TC_SMEM = 1024 + SMEM_OP + SMEM_MID + SMEM_LUT + SMEM_BAR;
 
 struct TcArgs {
+  CUtensorMap codes_map;  // uint32 [M][wrow], box {4 words, 128 rows}
+  CUtensorMap act_map;    // uint8 [pixels][row bytes], box {64 (or 32) bytes, 128 rows}; if act_tma
+  CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 128 positions}; if out_tma
   const uint8_t* act;
   const uint32_t* codes;
   const float* alpha;
@@ -70,12 +95,24 @@ struct TcArgs {
   int ntiles;       // groups * mtiles * ptiles
   int ktiles;       // K-tiles per tile (= ng * G / 64)
   int kt_per_group; // G / 64
+  int act_tma;      // activation rows by TMA (im2col rows are consecutive input rows)
+  int out_tma;      // output tile by TMA store (one conv group, M % 4 == 0)
   uint32_t wait_limit;
 };
 
 // Byte offset of 16-byte chunk c (0..7) of row r in a 128B-swizzled K-major tile.
 __device__ __forceinline__ uint32_t sw128(int r, int c) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// Byte offset of 16-byte chunk c of staging row t.  Rows are 64 bytes (8-bit activations,
+// 4 chunks) or 32 bytes (4-bit, 2 chunks); the chunk index is XOR-ed with row bits so that
+// eight consecutive rows read the same chunk from eight different bank groups.  This is
+// the layout a TMA box load with the 64-byte (32-byte) swizzle produces.
+template <int ABITS>
+__device__ __forceinline__ uint32_t st_off(int t, int c) {
+  if (ABITS == 8) return (uint32_t)(t * 64 + ((c ^ ((t >> 1) & 3)) << 4));
+  return (uint32_t)(t * 32 + ((c ^ ((t >> 2) & 1)) << 4));
 }
 
 __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, int& m0, int64_t& p0) {
@@ -96,19 +133,25 @@ __device__ __forceinline__ uint32_t u8pair_to_h2(uint32_t x, uint32_t sel, uint3
   return r;
 }
 
-template <int ABITS, bool SIGNED>
-__global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs a) {
+// TMAP: the layer's im2col rows are contiguous input rows (TMA loads, TMA-store epilogue);
+// otherwise rows are gathered with cp.async.
+template <int ABITS, bool SIGNED, bool TMAP>
+__global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid_constant__ TcArgs a) {
+  constexpr int TC_NS = TMAP ? TC_NS_TMA : TC_NS_GATHER;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* op = smem;                       // TC_NO x {A tile, B tile}
-  uint8_t* st = smem + SMEM_OP;             // TC_NS x {act bytes, code bytes}
-  uint2* lut = reinterpret_cast<uint2*>(smem + SMEM_OP + SMEM_ST);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP + SMEM_ST + SMEM_LUT);
+  uint8_t* op = smem;                               // TC_NO x {A tile, B tile}
+  uint8_t* st = smem + SMEM_OP;                     // TC_NS x {act bytes, code bytes}
+  float* otile = reinterpret_cast<float*>(smem + SMEM_OP + TC_NS_TMA * ST_STAGE);  // TMA path: [128 pos][128 filters]
+  uint32_t* lut = reinterpret_cast<uint32_t*>(smem + SMEM_OP + SMEM_MID);  // [16][32]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP + SMEM_MID + SMEM_LUT);
   uint64_t* op_full = bars;
   uint64_t* op_empty = bars + TC_NO;
-  uint64_t* acc_full = bars + 2 * TC_NO;
-  uint64_t* acc_empty = bars + 2 * TC_NO + TC_NACC;
-  uint64_t* drain_bar = bars + 2 * TC_NO + 2 * TC_NACC;
+  uint64_t* st_full = bars + 2 * TC_NO;
+  uint64_t* st_empty = st_full + TC_NS;
+  uint64_t* acc_full = st_empty + TC_NS;
+  uint64_t* acc_empty = acc_full + TC_NACC;
+  uint64_t* drain_bar = acc_empty + TC_NACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile uint32_t* abort_flag = tmem_slot + 1;
 
@@ -118,8 +161,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < TC_NO; ++i) {
-      mbar_init(&op_full[i], 128);
+      mbar_init(&op_full[i], TC_LOADERS);
       mbar_init(&op_empty[i], 1);
+    }
+    for (int i = 0; i < TC_NS; ++i) {
+      mbar_init(&st_full[i], 1);
+      mbar_init(&st_empty[i], TC_LOADERS);
     }
     for (int i = 0; i < TC_NACC; ++i) {
       mbar_init(&acc_full[i], 1);
@@ -129,15 +176,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
     *abort_flag = 0;
     fence_mbar_init();
   }
-  // code byte (four 2-bit codes) -> four fp16 {0, +1, -1}
-  for (int i = threadIdx.x; i < 256; i += blockDim.x) {
-    uint32_t h[4];
+  // two 2-bit codes (a nibble) -> two fp16 {0, +1, -1}; 32 copies so every lane reads its own bank
+  for (int i = threadIdx.x; i < 16 * 32; i += blockDim.x) {
+    const uint32_t x = (uint32_t)i >> 5;
+    uint32_t h[2];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const uint32_t c = (i >> (2 * e)) & 3u;
+    for (int e = 0; e < 2; ++e) {
+      const uint32_t c = (x >> (2 * e)) & 3u;
       h[e] = c == 1u ? 0x3C00u : (c == 3u ? 0xBC00u : 0u);
     }
-    lut[i] = make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+    lut[i] = h[0] | (h[1] << 16);
   }
   if (warp == TC_MMA_WARP) {
     tmem_alloc(tmem_slot, TC_TMEM_COLS);
@@ -156,21 +204,29 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
 
   // ------------------------------------------------------------------ loaders/converters
   if (warp >= TC_LOAD_WARP0 && warp < TC_MMA_WARP) {
-    const int t = threadIdx.x - 32 * TC_LOAD_WARP0;  // row owned in every tile
+    const int tid = threadIdx.x - 32 * TC_LOAD_WARP0;
+    const int t = tid & (TC_BN - 1);  // tile row converted (and gathered) by this thread
+    const int h = tid >> 7;           // which part of the row (when TC_LPR > 1)
     const int total = my_tiles * a.ktiles;
-    constexpr int ACT_BYTES = TC_KT * ABITS / 8;  // 64 (8-bit) or 32 (4-bit) bytes per row
-    constexpr int ACT_CHUNKS = ACT_BYTES / 16;
+    constexpr int ROW_BYTES = TC_KT * ABITS / 8;     // 64 (8-bit) or 32 (4-bit)
+    constexpr int CPR = ROW_BYTES / 16;              // 16-byte chunks per activation row
+    constexpr int HC = CPR / TC_LPR;                 // activation chunks this thread handles
+    constexpr uint32_t TX_CODES = TC_BM * 16;
+    constexpr uint32_t TX_ACT = TC_BN * ROW_BYTES;
 
-    // per-tile state of this thread's rows (refreshed when the issued K-tile enters a new tile)
-    int cur_tile = -1, gi = 0, m0 = 0, pb = 0, phb = 0, pwb = 0;
+    // per-tile state: conv group, first filter, this thread's row position; the filter
+    // tap (tr, ts) and channel offset tc0 of the next issued K-tile advance incrementally
+    int cur_tile = -1, gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0;
+    int64_t p0 = 0;
+    int pb = 0, phb = 0, pwb = 0;
     bool pvalid = false;
+    int issued = 0;  // K-tiles whose copies have been started
     auto issue = [&](int j) {
       const int tl = j / a.ktiles;
-      const int kk = j - tl * a.ktiles;
       if (tl != cur_tile) {
         cur_tile = tl;
-        int64_t p0;
         tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+        tr = ts = tc0 = 0;
         const int64_t p = p0 + t;
         pvalid = p < g.P;
         const int pp = pvalid ? (int)p : 0;
@@ -181,57 +237,87 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
         phb = ho * g.stride - g.pad;
         pwb = wo * g.stride - g.pad;
       }
-      uint8_t* sa = st + (j % TC_NS) * ST_STAGE;
-      const uint32_t sact = smem_u32(sa + t * ACT_BYTES);
-      const uint32_t scode = smem_u32(sa + ST_ACT + t * 16);
-      const int k0 = kk * TC_KT;
-      const uint8_t* src = a.act;
-      bool inside = false;
-      if (pvalid) {
-        const int tap = k0 / g.Cg;
-        const int c0 = k0 - tap * g.Cg;
-        const int r = tap / g.S, s = tap - r * g.S;
-        const int hi = phb + r, wi = pwb + s;
-        if (hi >= 0 && hi < g.H && wi >= 0 && wi < g.W) {
-          const int64_t e = (((int64_t)pb * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + c0;
-          src = a.act + e * ABITS / 8;
-          inside = true;
+      const int slot = j % TC_NS;
+      uint8_t* sa = st + slot * ST_STAGE;
+      const int kk = j - tl * a.ktiles;
+      if (TMAP && tid == 0) {
+        // the slot's previous contents (K-tile j - TC_NS) have been released by every thread
+        bool free_ok = true;
+        if (j >= TC_NS)
+          free_ok = mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag);
+        if (free_ok) {
+          mbar_arrive_expect_tx(&st_full[slot], TX_CODES + (TMAP ? TX_ACT : 0u));
+          tma_load_2d(smem_u32(sa + ST_ACT), &a.codes_map, kk * (TC_KT / 16), m0, &st_full[slot]);
+          if (TMAP)
+            tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
+          issued = j + 1;
+        } else {
+          if (!*abort_flag) fail();
         }
       }
+      if (!TMAP) {
+        const uint8_t* src = a.act;
+        bool inside = false;
+        if (pvalid) {
+          const int hi = phb + tr, wi = pwb + ts;
+          if (hi >= 0 && hi < g.H && wi >= 0 && wi < g.W) {
+            const int64_t e = (((int64_t)pb * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + tc0;
+            src = a.act + e * ABITS / 8;
+            inside = true;
+          }
+        }
 #pragma unroll
-      for (int c = 0; c < ACT_CHUNKS; ++c)
-        cp_async16(sact + 16 * c, inside ? (const void*)(src + 16 * c) : (const void*)a.act, inside ? 16u : 0u);
-      const int m = m0 + t;
-      const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
-      const uint32_t* csrc = mok ? a.codes + (int64_t)m * g.wrow + k0 / 16 : a.codes;
-      cp_async16(scode, csrc, mok ? 16u : 0u);
+        for (int c = 0; c < HC; ++c) {
+          const int ch = h * HC + c;
+          cp_async16(smem_u32(sa + st_off<ABITS>(t, ch)), inside ? (const void*)(src + 16 * ch) : (const void*)a.act,
+                     inside ? 16u : 0u);
+        }
+        // this thread's part of code row t (filter m0 + t): 16 / TC_LPR bytes of 4 code words
+        const int m = m0 + t;
+        const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
+        if (TC_LPR == 1 || h == 0) {
+          const uint32_t* csrc = mok ? a.codes + (int64_t)m * g.wrow + kk * (TC_KT / 16) : a.codes;
+          cp_async16(smem_u32(sa + ST_ACT + t * 16), csrc, mok ? 16u : 0u);
+        }
+      }
+      tc0 += TC_KT;  // next K-tile of this tile
+      if (tc0 == g.Cg) {
+        tc0 = 0;
+        if (++ts == g.S) {
+          ts = 0;
+          ++tr;
+        }
+      }
     };
 
-    bool ok = true;
     for (int j = 0; j < TC_NS - 1; ++j) {
       if (j < total) issue(j);
       cp_async_commit();
     }
-    for (int j = 0; j < total && ok; ++j) {
+    int consumed = 0;
+    for (int j = 0; j < total; ++j) {
+      if (*abort_flag) break;
       if (j + TC_NS - 1 < total) issue(j + TC_NS - 1);
       cp_async_commit();
-      cp_async_wait<TC_NS - 1>();  // this thread's copies of K-tile j have landed
+      if (!TMAP) cp_async_wait<TC_NS - 1>();  // this thread's copies for K-tile j have landed
+      const int slot = j % TC_NS;
       const int os = j % TC_NO;
-      if (!mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)) {
+      if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag)) ||
+          !mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)) {
         if (!*abort_flag) fail();
-        ok = false;
         break;
       }
-      const uint8_t* sa = st + (j % TC_NS) * ST_STAGE;
+      consumed = j + 1;
+      const uint8_t* sa = st + slot * ST_STAGE;
       uint8_t* A = op + os * OP_STAGE;
       uint8_t* Bt = A + OP_TILE;
-      // activations -> fp16 row t of B
+      // activations -> fp16 (this thread's part of row t of B)
       if (ABITS == 8) {
-        const uint4* src = reinterpret_cast<const uint4*>(sa + t * 64);
         const uint32_t bias2 = SIGNED ? 0x64806480u : 0x64006400u;  // 1152 or 1024 in both halves
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint4 v = src[c];
+        for (int cc = 0; cc < HC; ++cc) {
+          const int c = HC * h + cc;
+          uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<8>(t, c));
           if (SIGNED) {
             v.x ^= 0x80808080u; v.y ^= 0x80808080u; v.z ^= 0x80808080u; v.w ^= 0x80808080u;
           }
@@ -244,46 +330,57 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
           *reinterpret_cast<uint4*>(Bt + sw128(t, 2 * c + 1)) = o1;
         }
       } else {
-        const uint4* src = reinterpret_cast<const uint4*>(sa + t * 32);
         const uint32_t bias2 = SIGNED ? 0x64086408u : 0x64006400u;  // 1032 or 1024
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          const uint4 v = src[c];
-          const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+        for (int cc = 0; cc < HC; ++cc) {
+        const int c = HC * h + cc;
+        const uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<4>(t, c));
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            // 8 nibbles -> 8 bytes (element order preserved), then 8 fp16
-            const uint32_t x = w4[q];
-            const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
-            const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
-            uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                            // e0 e1 e2 e3
-            uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                                    // e4 e5 e6 e7
-            if (SIGNED) {
-              b0 ^= 0x08080808u;
-              b1 ^= 0x08080808u;
-            }
-            uint4 o;
-            o.x = u8pair_to_h2(b0, 0x4140, bias2); o.y = u8pair_to_h2(b0, 0x4342, bias2);
-            o.z = u8pair_to_h2(b1, 0x4140, bias2); o.w = u8pair_to_h2(b1, 0x4342, bias2);
-            *reinterpret_cast<uint4*>(Bt + sw128(t, 4 * c + q)) = o;
+        for (int q = 0; q < 4; ++q) {
+          // 8 nibbles -> 8 bytes (element order preserved), then 8 fp16
+          const uint32_t x = w4[q];
+          const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
+          const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
+          uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                            // e0 e1 e2 e3
+          uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                                    // e4 e5 e6 e7
+          if (SIGNED) {
+            b0 ^= 0x08080808u;
+            b1 ^= 0x08080808u;
           }
+          uint4 o;
+          o.x = u8pair_to_h2(b0, 0x4140, bias2); o.y = u8pair_to_h2(b0, 0x4342, bias2);
+          o.z = u8pair_to_h2(b1, 0x4140, bias2); o.w = u8pair_to_h2(b1, 0x4342, bias2);
+          *reinterpret_cast<uint4*>(Bt + sw128(t, 4 * c + q)) = o;
+        }
         }
       }
-      // codes -> fp16 row t of A: 64 codes, 8 per 16-byte chunk, 4 per table lookup
+      // codes -> fp16 (this thread's part of row t of A): 8 codes per 16-byte chunk, 2 per
+      // table lookup
       {
-        const uint4 cv = *reinterpret_cast<const uint4*>(sa + ST_ACT + t * 16);
-        const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+        constexpr int CC = 8 / TC_LPR;  // 16-byte fp16 chunks of A converted by this thread
+        uint32_t cw[CC / 2];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const uint32_t bits = (cw[c / 2] >> (16 * (c & 1))) & 0xffffu;  // 8 codes
-          const uint2 lo = lut[bits & 0xffu], hi = lut[bits >> 8];
-          *reinterpret_cast<uint4*>(A + sw128(t, c)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+        for (int i = 0; i < CC / 2; ++i) cw[i] = *reinterpret_cast<const uint32_t*>(sa + ST_ACT + t * 16 + 4 * (i + (CC / 2) * h));
+        const uint32_t* lt = lut + lane;
+#pragma unroll
+        for (int cc = 0; cc < CC; ++cc) {
+          const uint32_t bits = (cw[cc / 2] >> (16 * (cc & 1))) & 0xffffu;  // 8 codes
+          *reinterpret_cast<uint4*>(A + sw128(t, CC * h + cc)) =
+              make_uint4(lt[32 * (bits & 15u)], lt[32 * ((bits >> 4) & 15u)], lt[32 * ((bits >> 8) & 15u)],
+                         lt[32 * (bits >> 12)]);
         }
       }
       fence_proxy_async_smem();
       mbar_arrive(&op_full[os]);
+      if (TMAP) mbar_arrive(&st_empty[slot]);  // done reading this TMA-filled staging slot
     }
     cp_async_wait_all();
+    // TMA loads issued but not consumed (only after a failure): wait, bounded, for their
+    // bytes to land so that no copy into this CTA's shared memory outlives it
+    if (tid == 0) {
+      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % TC_NS], (j / TC_NS) & 1, 1u << 16);
+    }
   }
 
   // ------------------------------------------------------------------ MMA issuer
@@ -334,9 +431,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
     const int t = 32 * quarter + lane;  // TMEM lane = filter row of the tile
     const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(64 * half);
     const float sx = __ldg(a.act_scale);
+    const bool leader = threadIdx.x == 0;
     int gc = 0;
     bool ok = true;
-    for (int tl = 0; tl < my_tiles && ok; ++tl) {
+    for (int tl = 0; tl < my_tiles; ++tl) {
       int gi, m0;
       int64_t p0;
       tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
@@ -346,29 +444,45 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
       float acc[64];
 #pragma unroll
       for (int j = 0; j < 64; ++j) acc[j] = 0.0f;
+      float al_next = mok ? __ldg(arow) : 0.0f;
       for (int grp = 0; grp < g.ng; ++grp, ++gc) {
+        if (!ok) continue;  // after a failed wait: run out the tile, then leave with the others
         const int b = gc % TC_NACC;
-        const float al = mok ? __ldg(arow + grp) : 0.0f;
+        const float al = al_next;  // alpha of this group, loaded one group ahead
+        if (mok && grp + 1 < g.ng) al_next = __ldg(arow + grp + 1);
         if (!mbar_wait_or_abort(&acc_full[b], (gc / TC_NACC) & 1, a.wait_limit, abort_flag)) {
           if (!*abort_flag) fail();
           ok = false;
-          break;
+          continue;
         }
         tc_fence_after();
-        uint32_t r0[32], r1[32];
-        tmem_ld32(tbase + (uint32_t)(b * TC_BN), r0);
-        tmem_ld32(tbase + (uint32_t)(b * TC_BN + 32), r1);
+        uint32_t r[32];
+        tmem_ld32(tbase + (uint32_t)(b * TC_BN), r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) acc[j] = fmaf(al, __uint_as_float(r[j]), acc[j]);
+        tmem_ld32(tbase + (uint32_t)(b * TC_BN + 32), r);
         tmem_ld_wait();
         tc_fence_before();
         mbar_arrive(&acc_empty[b]);  // the buffer is free once the values are in registers
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          acc[j] = fmaf(al, __uint_as_float(r0[j]), acc[j]);
-          acc[32 + j] = fmaf(al, __uint_as_float(r1[j]), acc[32 + j]);
-        }
+        for (int j = 0; j < 32; ++j) acc[32 + j] = fmaf(al, __uint_as_float(r[j]), acc[32 + j]);
       }
-      if (!ok) break;
-      if (mok) {
+      if (named_bar_or(BAR_EPI, 32 * TC_EPI_WARPS, !ok)) break;  // leave together
+      if (TMAP && a.out_tma) {
+        // the previous tile's store has finished reading the staging tile
+        if (leader) bulk_wait_read_all();
+        named_bar_sync(BAR_EPI, 32 * TC_EPI_WARPS);
+        float* orow = otile + (64 * half) * TC_BM + t;
+#pragma unroll
+        for (int j = 0; j < 64; ++j) orow[j * TC_BM] = sx * acc[j];
+        fence_proxy_async_smem();
+        named_bar_sync(BAR_EPI, 32 * TC_EPI_WARPS);
+        if (leader) {
+          tma_store_2d(&a.out_map, m0, (int)p0, smem_u32(otile));
+          bulk_commit();
+        }
+      } else if (mok) {
         const int64_t pbase = p0 + 64 * half;
 #pragma unroll
         for (int j = 0; j < 64; ++j) {
@@ -377,6 +491,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
         }
       }
     }
+    if (leader) bulk_wait_all();  // this thread's TMA stores are complete
   }
 
   tc_fence_before();
@@ -387,17 +502,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const TcArgs
   }
 }
 
-template <int ABITS, bool SIGNED>
+template <int ABITS, bool SIGNED, bool TMAP>
 fgq_status launch_tc(const TcArgs& args, int grid, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(tc_contract_kernel<ABITS, SIGNED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(tc_contract_kernel<ABITS, SIGNED, TMAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              TC_SMEM) != cudaSuccess)
       return FGQ_ERR_CUDA;
     attr_set = true;
   }
-  tc_contract_kernel<ABITS, SIGNED><<<grid, TC_THREADS, TC_SMEM, s>>>(args);
+  tc_contract_kernel<ABITS, SIGNED, TMAP><<<grid, TC_THREADS, TC_SMEM, s>>>(args);
   return after_launch();
+}
+
+template <int ABITS, bool SIGNED>
+fgq_status launch_tc_path(const TcArgs& args, int grid, cudaStream_t s) {
+  return args.act_tma ? launch_tc<ABITS, SIGNED, true>(args, grid, s) : launch_tc<ABITS, SIGNED, false>(args, grid, s);
 }
 
 // One block waits on an mbarrier that nothing arrives on; every wait is bounded, so the
@@ -413,13 +533,41 @@ __global__ void wait_timeout_selftest_kernel(uint32_t max_iter, unsigned int* er
   if (!ok && threadIdx.x == 0) record_error(err, FGQ_ERR_TIMEOUT);
 }
 
+// cuTensorMapEncodeTiled from the driver, looked up once through the runtime.
+PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2D tiled map: dims {d0 (innermost), d1}, row pitch in bytes, box {b0, b1}.
+bool make_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t d0, uint64_t d1,
+                 uint64_t pitch, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {
+  auto enc = encode_tiled();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {d0, d1};
+  const cuuint64_t strides[1] = {pitch};
+  const cuuint32_t box[2] = {b0, b1};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 bool tc_supports(const Geom& g) {
   if (g.G != 64 && g.G != 128) return false;
-  if (g.Cg % TC_KT != 0) return false;     // every K-tile inside one filter tap (conv) or row (GEMM)
-  if (g.C % 16 != 0) return false;         // 16-byte aligned activation rows
+  if (g.Cg % TC_KT != 0) return false;        // every K-tile inside one filter tap (conv) or row (GEMM)
+  if (g.C % 16 != 0) return false;            // 16-byte aligned activation rows
   if (g.P >= (int64_t)1 << 31) return false;  // positions decoded in 32 bits
+  if (encode_tiled() == nullptr) return false;
   return true;
 }
 
@@ -428,6 +576,7 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                               cudaStream_t s) {
   if (sums != nullptr || !tc_supports(g)) return FGQ_ERR_UNSUPPORTED;
   TcArgs a;
+  memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
   a.codes = codes;
   a.alpha = alpha;
@@ -441,14 +590,32 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   a.kt_per_group = g.G / TC_KT;
   a.ktiles = g.ng * a.kt_per_group;
   a.wait_limit = TC_WAIT_LIMIT;
+  const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
+  if (!make_map_2d(&a.codes_map, CU_TENSOR_MAP_DATA_TYPE_UINT32, codes, (uint64_t)g.wrow, (uint64_t)g.M,
+                   (uint64_t)g.wrow * 4, TC_KT / 16, TC_BM, CU_TENSOR_MAP_SWIZZLE_NONE))
+    return FGQ_ERR_CUDA;
+  // im2col rows are consecutive input rows for a 1x1, stride-1, unpadded convolution or a GEMM
+  if (g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
+    const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
+    a.act_tma = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, row_bytes, (uint64_t)g.B * g.H * g.W,
+                            row_bytes, (uint32_t)(TC_KT * abits / 8), TC_BN,
+                            abits == 8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B)
+                    ? 1
+                    : 0;
+  }
+  if (a.act_tma && g.groups == 1 && g.M % 4 == 0) {
+    a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
+                            (uint64_t)g.M * 4, TC_BM, TC_BN, CU_TENSOR_MAP_SWIZZLE_NONE)
+                    ? 1
+                    : 0;
+  }
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = a.ntiles < sms ? a.ntiles : sms;
   const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
-  const bool four = g.act_type == FGQ_U4 || g.act_type == FGQ_S4;
-  if (four) return sgn ? launch_tc<4, true>(a, grid, s) : launch_tc<4, false>(a, grid, s);
-  return sgn ? launch_tc<8, true>(a, grid, s) : launch_tc<8, false>(a, grid, s);
+  if (abits == 4) return sgn ? launch_tc_path<4, true>(a, grid, s) : launch_tc_path<4, false>(a, grid, s);
+  return sgn ? launch_tc_path<8, true>(a, grid, s) : launch_tc_path<8, false>(a, grid, s);
 }
 
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s) {

@@ -35,20 +35,37 @@ __device__ __forceinline__ bool j_greater(uint64_t Sa, uint32_t ka, uint64_t Sb,
 }
 
 // fp32 nearest (ties to even) to S * 2^u / k, for 1 <= S < 2^40, 1 <= k <= 128, u >= -157.
+// Only the top 32 bits of S enter a 32-bit division: with N = those bits (N >= 2^31) and
+// the dropped low bits folded into a sticky flag, the exact quotient is
+// q + (r + f) / k with q = N / k >= 2^24, r = N % k and 0 <= f < 1, so q is its floor and
+// the quotient is exact iff r == 0 and nothing was dropped -- enough to round to 24 bits.
 __device__ __forceinline__ float round_ratio_f32(uint64_t S, uint32_t k, int u) {
   if (S == 0 || k == 0) return 0.0f;
-  const int sh = __clzll((long long)S) - 8;  // S << sh has 56 significant bits
-  const uint64_t num = S << sh;
-  const uint64_t q = num / k;
-  const uint64_t r = num - q * k;
-  const int nb = 64 - __clzll((long long)q);  // >= 49
-  const int lead = nb - 1 + u - sh;           // binary exponent of the leading bit
+  const int nbS = 64 - __clzll((long long)S);
+  int shift = nbS - 32;  // value = (N + dropped) * 2^(u + shift) / k
+  uint32_t N;
+  bool dropped;
+  if (shift >= 0) {
+    N = (uint32_t)(S >> shift);
+    dropped = (S & ((1ull << shift) - 1)) != 0;
+  } else {
+    N = (uint32_t)(S << -shift);
+    dropped = false;
+  }
+  const uint32_t q = N / k;
+  const uint32_t r = N - q * k;
+  const bool sticky = dropped || r != 0;
+  const int nb = 32 - __clz((int)q);           // >= 25
+  const int lead = nb - 1 + u + shift;         // binary exponent of the leading bit
   int lsb = lead >= -126 ? lead - 23 : -149;
-  const int drop = lsb - (u - sh);            // bits of q below the fp32 lsb, in [25, 63]
-  uint64_t mant = drop < 64 ? (q >> drop) : 0;
-  const uint64_t rem = drop < 64 ? (q & ((1ull << drop) - 1)) : q;
-  const uint64_t half = 1ull << (drop - 1);
-  if (rem > half || (rem == half && (r != 0 || (mant & 1)))) mant += 1;
+  const int drop = lsb - (u + shift);          // bits of q below the fp32 lsb, >= 1
+  uint64_t mant = 0, rem = 0, half = 1;
+  if (drop < 64) {
+    mant = (uint64_t)q >> drop;
+    rem = (uint64_t)q & ((1ull << drop) - 1);
+    half = 1ull << (drop - 1);
+  }  // else: the value is below a quarter of the smallest subnormal step and rounds to 0
+  if (rem > half || (rem == half && (sticky || (mant & 1)))) mant += 1;
   if (mant == (1ull << 24)) {
     mant >>= 1;
     lsb += 1;
