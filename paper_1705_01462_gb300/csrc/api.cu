@@ -54,12 +54,18 @@ fgq_status make_geom(int type, int B, int H, int W, int C, int R, int S, int str
   return FGQ_OK;
 }
 
+bool tc_any(const Geom& g) { return g.G == 4 ? tc4_supports(g) : tc_supports(g); }
+
 int choose_path(const Geom& g, bool sums) {
   const int forced = g_path.load();
   if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
-  if (forced == FGQ_PATH_TC) return tc_supports(g) ? FGQ_PATH_TC : -1;
-  return tc_supports(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
+  if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
+  // automatic choice: G = 4 stays on the dp4a kernel (the block-diagonal tensor-core form
+  // is reached by forcing FGQ_PATH_TC); G in {64, 128} takes the tensor cores when the
+  // shape is covered
+  if (g.G == 4) return FGQ_PATH_SIMT;
+  return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
 }
 
 fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
@@ -69,7 +75,10 @@ fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const
   if (path < 0) return FGQ_ERR_UNSUPPORTED;
   t_last_path = path;
   unsigned int* err = device_error_word();
-  if (path == FGQ_PATH_TC) return launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
+  if (path == FGQ_PATH_TC) {
+    if (g.G == 4) return launch_tc4_contract(act, g, codes, alpha, act_scale, out, err, s);
+    return launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
+  }
   return launch_simt_contract(act, g, codes, alpha, 0, act_scale, out, sums, s);
 }
 

@@ -49,6 +49,11 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                               const float* alpha, const float* act_scale, float* out,
                               int32_t* sums, unsigned int* err, cudaStream_t s);
 
+// Tensor-core contraction for G = 4 (block-diagonal activation operand).
+bool tc4_supports(const Geom& g);
+fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
+                               const float* act_scale, float* out, unsigned int* err, cudaStream_t s);
+
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
 
 }  // namespace fgq

@@ -32,18 +32,19 @@
 // Every mbarrier wait is bounded; on expiry the kernel records FGQ_ERR_TIMEOUT, each role
 // leaves its loop (uniformly within a role that uses named barriers), in-flight copies
 // and MMAs are waited for, and TMEM is freed.
-#include <cuda.h>
-#include <cudaTypedefs.h>
-
 #include <cstdint>
 #include <cstring>
-#include <mutex>
 
-#include "fgq_device.cuh"
-#include "ptx_sm100.cuh"
+#include "tc_common.cuh"
 
 namespace fgq {
 namespace {
+
+using tc::encode_tiled;
+using tc::make_map_2d;
+using tc::st_off;
+using tc::sw128;
+using tc::u8pair_to_h2;
 
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 128;        // positions per tile (MMA N)
@@ -100,21 +101,6 @@ struct TcArgs {
   uint32_t wait_limit;
 };
 
-// Byte offset of 16-byte chunk c (0..7) of row r in a 128B-swizzled K-major tile.
-__device__ __forceinline__ uint32_t sw128(int r, int c) {
-  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
-}
-
-// Byte offset of 16-byte chunk c of staging row t.  Rows are 64 bytes (8-bit activations,
-// 4 chunks) or 32 bytes (4-bit, 2 chunks); the chunk index is XOR-ed with row bits so that
-// eight consecutive rows read the same chunk from eight different bank groups.  This is
-// the layout a TMA box load with the 64-byte (32-byte) swizzle produces.
-template <int ABITS>
-__device__ __forceinline__ uint32_t st_off(int t, int c) {
-  if (ABITS == 8) return (uint32_t)(t * 64 + ((c ^ ((t >> 1) & 3)) << 4));
-  return (uint32_t)(t * 32 + ((c ^ ((t >> 2) & 1)) << 4));
-}
-
 __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, int& m0, int64_t& p0) {
   const int per_p = a.g.groups * a.mtiles;
   const int pt = tile / per_p;
@@ -123,14 +109,6 @@ __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, 
   const int mt = r - gi * a.mtiles;
   m0 = gi * a.g.Mg + mt * TC_BM;
   p0 = (int64_t)pt * TC_BN;
-}
-
-// fp16 pair (lo, hi) from two 8-bit lanes of x selected by sel (unsigned: 1024 + v - 1024).
-__device__ __forceinline__ uint32_t u8pair_to_h2(uint32_t x, uint32_t sel, uint32_t bias2) {
-  const uint32_t h = __byte_perm(x, 0x64646464u, sel);  // halves 1024 + v
-  uint32_t r;
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(h), "r"(bias2));
-  return r;
 }
 
 // TMAP: the layer's im2col rows are contiguous input rows (TMA loads, TMA-store epilogue);
@@ -176,17 +154,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     *abort_flag = 0;
     fence_mbar_init();
   }
-  // two 2-bit codes (a nibble) -> two fp16 {0, +1, -1}; 32 copies so every lane reads its own bank
-  for (int i = threadIdx.x; i < 16 * 32; i += blockDim.x) {
-    const uint32_t x = (uint32_t)i >> 5;
-    uint32_t h[2];
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const uint32_t c = (x >> (2 * e)) & 3u;
-      h[e] = c == 1u ? 0x3C00u : (c == 3u ? 0xBC00u : 0u);
-    }
-    lut[i] = h[0] | (h[1] << 16);
-  }
+  tc::fill_code_lut(lut);
   if (warp == TC_MMA_WARP) {
     tmem_alloc(tmem_slot, TC_TMEM_COLS);
     tmem_relinquish();
@@ -531,33 +499,6 @@ __global__ void wait_timeout_selftest_kernel(uint32_t max_iter, unsigned int* er
   __syncthreads();
   const bool ok = mbar_wait_bounded(&bar, 0, max_iter);
   if (!ok && threadIdx.x == 0) record_error(err, FGQ_ERR_TIMEOUT);
-}
-
-// cuTensorMapEncodeTiled from the driver, looked up once through the runtime.
-PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
-}
-
-// 2D tiled map: dims {d0 (innermost), d1}, row pitch in bytes, box {b0, b1}.
-bool make_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t d0, uint64_t d1,
-                 uint64_t pitch, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {
-  auto enc = encode_tiled();
-  if (!enc) return false;
-  const cuuint64_t dims[2] = {d0, d1};
-  const cuuint64_t strides[1] = {pitch};
-  const cuuint32_t box[2] = {b0, b1};
-  const cuuint32_t estr[2] = {1, 1};
-  return enc(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace

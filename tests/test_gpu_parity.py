@@ -252,6 +252,10 @@ TC_CASES = [
 ]
 
 
+# every tensor-core case also at G = 4 (the block-diagonal G = 4 kernel)
+TC_CASES = TC_CASES + [c[:10] + (4,) + c[11:] for c in TC_CASES]
+
+
 @pytest.mark.parametrize("case", TC_CASES, ids=lambda c: "x".join(map(str, c)))
 def test_tc_conv2d_parity(case):
     B, H, W, C, M, R, S, stride, pad, groups, G, act = case
@@ -270,7 +274,8 @@ def test_tc_conv2d_parity(case):
 
 
 @pytest.mark.parametrize("case", [(128, 64, 128, 64, "u8"), (1, 9216, 4096, 64, "u8"), (300, 256, 64, 128, "s8"),
-                                  (257, 1024, 1000, 64, "u8"), (64, 512, 130, 64, "u4")],
+                                  (257, 1024, 1000, 64, "u8"), (64, 512, 130, 64, "u4"), (128, 64, 128, 4, "u8"),
+                                  (1, 9216, 4096, 4, "u8"), (257, 1024, 1000, 4, "s8"), (64, 512, 130, 4, "u4")],
                          ids=lambda c: "x".join(map(str, c)))
 def test_tc_gemm_parity(case):
     P, K, M, G, act = case
@@ -296,3 +301,23 @@ def test_tc_forced_on_unsupported_shape():
     with pytest.raises(fgq.FGQError) as e:
         fgq.fgq_gemm(q, "u8", torch.ones(1, device=dev()), 64, 48, codes, al, 8, 64)
     assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("path", ["simt", "tc"])
+@pytest.mark.parametrize("case", [(1, 56, 56, 64, 64, 3, 3, 1, 1, 1, 4, "u8"), (2, 28, 28, 128, 96, 1, 1, 1, 0, 1, 4, "u8"),
+                                  (2, 14, 14, 256, 64, 1, 1, 2, 0, 1, 4, "s8")],
+                         ids=lambda c: "x".join(map(str, c)))
+def test_g4_both_kernel_families(case, path):
+    """G = 4 through the dp4a kernel and through the block-diagonal tensor-core kernel."""
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()) + 2)
+    w = (rng.standard_normal((M, R * S * C)) * np.sqrt(2.0 / (R * S * C))).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    fgq.fgq_set_path(fgq.PATH_SIMT if path == "simt" else fgq.PATH_TC)
+    gout = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride,
+                          pad, groups, to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    assert fgq.fgq_last_path() == (fgq.PATH_SIMT if path == "simt" else fgq.PATH_TC)
+    check_within(gout.cpu().numpy(), y, ym, f"G=4 {path} {case}")
