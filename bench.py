@@ -239,7 +239,7 @@ class Workload:
                         self.q[i].data_ptr(), fgq.U8, self.sc[i].data_ptr(), self.B, l.H, l.W, l.C, l.R, l.S,
                         l.stride, l.pad, l.groups, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(), l.M, G,
                         self.out[G][i].data_ptr(), sh), "conv"))
-                    self.paths.setdefault(f"conv_g{G}", {})[L.fgq_last_path()] = True
+                    self.paths[(G, i)] = L.fgq_last_path()
 
 
 def alu_peak_tops(G, sm_count, clk_hz):
@@ -251,19 +251,37 @@ def alu_peak_tops(G, sm_count, clk_hz):
     return sm_count * clk_hz * (2.0 * G) / clk_per_unit / 1e12
 
 
+def tc_peak_tops(G, sm_count, clk_hz, bf16_tflops):
+    """Peak of the tensor-core contraction in effective TOPS, and what bounds it.  The MMAs
+    (fp16 operands, the bf16 rate) do the 2G ops of a (filter, position, group) unit, but for
+    G = 4 three quarters of each block-diagonal MMA multiply zeros, so the MMA bound is a
+    quarter of the bf16 peak; the epilogue spends one fp32 FMA per unit on a 128-lane/clk/SM
+    pipe."""
+    mma = bf16_tflops * (0.25 if G == 4 else 1.0)
+    fma = sm_count * clk_hz * 128 * 2.0 * G / 1e12
+    return (mma, "tensor") if mma <= fma else (fma, "alu")
+
+
 def family_roofline(fam, layers, B, peaks, sm_count, sec_per_step, paths):
     """Roofline entry of a kernel family over one step: bound, achieved, peak, unit, and the
-    algorithmic work (ops or bytes) and bytes per step."""
+    algorithmic work (ops or bytes) and bytes per step.  A conv family whose layers run on
+    different kernels gets the ops-weighted harmonic blend of the kernels' peaks (the step
+    time if every layer ran at its kernel's peak)."""
     clk = peaks["sm_max_mhz"] * 1e6
     if fam.startswith("conv_g"):
         G = int(fam[6:])
         ops = sum(l.ops(B) for l in layers[1:])
         nbytes = sum(algorithmic_bytes(l, B, G) for l in layers[1:])
-        if paths.get(fam) == 2:  # tensor-core family: bf16-rate MMAs on exact integers
-            return {"bound": "tensor", "achieved": ops / sec_per_step / 1e12, "peak": peaks["bf16_tflops"],
-                    "unit": "TFLOP/s", "bytes": nbytes}
-        return {"bound": "alu", "achieved": ops / sec_per_step / 1e12, "peak": alu_peak_tops(G, sm_count, clk),
-                "unit": "TOPS", "bytes": nbytes}
+        ideal_s, ops_by_bound = 0.0, {}
+        for i, l in enumerate(layers[1:], start=1):
+            if paths.get((G, i)) == 2:
+                pk, bound = tc_peak_tops(G, sm_count, clk, peaks["bf16_tflops"])
+            else:
+                pk, bound = alu_peak_tops(G, sm_count, clk), "alu"
+            ideal_s += l.ops(B) / (pk * 1e12)
+            ops_by_bound[bound] = ops_by_bound.get(bound, 0) + l.ops(B)
+        return {"bound": max(ops_by_bound, key=ops_by_bound.get), "achieved": ops / sec_per_step / 1e12,
+                "peak": ops / ideal_s / 1e12, "unit": "TOPS", "bytes": nbytes}
     if fam == "quantize_act":  # fp32 in, uint8 out
         nbytes = sum(B * l.H * l.W * l.C * 5 for l in layers)
     elif fam.startswith("ternarize_g"):  # fp32 in; 2-bit codes and one fp32 alpha per group out
@@ -339,6 +357,28 @@ def dist_setup(args):
     return ws, rank, local
 
 
+def rank_seed_offset(rank):
+    """Seed offset of a rank's synthetic inputs: every rank works on its own batch."""
+    return rank * 7
+
+
+def max_over_ranks(dist, value, device):
+    """The maximum of a per-rank time over all ranks (the job is as slow as its slowest
+    rank); dist is torch.distributed with an initialized group, or None for one rank."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(ops_per_rank, world, ms_per_step):
+    """Whole-job throughput in effective TOPS: the units all ranks processed over the
+    (max-over-ranks) step time."""
+    return ops_per_rank * world / (ms_per_step / 1e3) / 1e12
+
+
 def run_reference(args, ws, rank):
     if rank != 0:
         return
@@ -385,7 +425,7 @@ def main():
     peaks = load_peaks()
     sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
     layers = workload_layers()
-    W = Workload(dev, BATCH, layers, seed_offset=rank * 7)
+    W = Workload(dev, BATCH, layers, seed_offset=rank_seed_offset(rank))
     stream = torch.cuda.Stream(device=dev)
 
     with torch.cuda.stream(stream):
@@ -416,17 +456,14 @@ def main():
     status = fgq.fgq_stream_status(stream)
     if status != fgq.FGQ_OK:
         raise RuntimeError(f"device error during the timed region: {status}")
-    if pg:
-        t = torch.tensor([total_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(pg, total_ms, dev)
     ms_per_step = total_ms / args.steps
     ops_rank = total_ops(layers, BATCH)
-    value = ops_rank * ws / (ms_per_step / 1e3) / 1e12
+    value = whole_job_rate(ops_rank, ws, ms_per_step)
 
     fam_ms = {f: sum(a.elapsed_time(b) for a, b in ev) for f, ev in timers.items()}
     dom = max(fam_ms, key=fam_ms.get)
-    paths = {f: (2 if 2 in v else 1) for f, v in W.paths.items()}
+    paths = W.paths
     roof = family_roofline(dom, layers, BATCH, peaks, sm_count, fam_ms[dom] / 1e3 / args.steps, paths)
     traffic = load_traffic().get(dom)
     n_launch_per_step = len(timers[dom]) / args.steps
@@ -436,7 +473,9 @@ def main():
                 "algorithmic_bytes_per_launch": roof["bytes"] / n_launch_per_step,
                 "launches_per_step": n_launch_per_step,
                 "family_ms_per_step": {f: v / args.steps for f, v in sorted(fam_ms.items())},
-                "conv_paths": {f: ("tc" if p == 2 else "simt") for f, p in paths.items()}}
+                "conv_layers_on_tc": {f"conv_g{G}": sum(1 for (g, _), p in paths.items() if g == G and p == 2)
+                                      for G in GROUPS},
+                "conv_layers": len(layers) - 1}
 
     # ---- end-to-end through the C ABI with host buffers (pinned), copies inside the timed region
     h_x = [x.to("cpu").pin_memory() for x in W.x]
@@ -464,11 +503,8 @@ def main():
         e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / ne2e
-    if pg:
-        t = torch.tensor([e2e_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = ops_rank * ws / (e2e_ms / 1e3) / 1e12
+    e2e_ms = max_over_ranks(pg, e2e_ms, dev)
+    e2e_value = whole_job_rate(ops_rank, ws, e2e_ms)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:

@@ -65,8 +65,9 @@ typedef enum { FGQ_U8 = 0, FGQ_S8 = 1, FGQ_U4 = 2, FGQ_S4 = 3 } fgq_act_type;
 
 /* Contraction kernel families (see fgq_set_path / fgq_last_path). */
 typedef enum {
-  FGQ_PATH_AUTO = 0,   /* choose per shape: G = 4 on the CUDA cores, G in {64, 128} on the
-                          tensor cores where the shape is covered */
+  FGQ_PATH_AUTO = 0,   /* choose per shape: the tensor cores where the shape is covered
+                          (G = 4 only with at least 128 filters per conv group), else the
+                          CUDA cores */
   FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
   FGQ_PATH_TC = 2      /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
                           the group; G = 4 with a block-diagonal activation operand

@@ -61,10 +61,10 @@ int choose_path(const Geom& g, bool sums) {
   if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
   if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
-  // automatic choice: G = 4 stays on the dp4a kernel (the block-diagonal tensor-core form
-  // is reached by forcing FGQ_PATH_TC); G in {64, 128} takes the tensor cores when the
-  // shape is covered
-  if (g.G == 4) return FGQ_PATH_SIMT;
+  // automatic choice: the tensor cores where the shape is covered, except G = 4 layers with
+  // fewer than 128 filters per conv group, where the 128-row MMA tile would leave half its
+  // rows idle and the dp4a kernel is faster
+  if (g.G == 4 && g.Mg < 128) return FGQ_PATH_SIMT;
   return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
 }
 
