@@ -167,6 +167,10 @@ fgq_status fgq_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, 
  *   codes, alpha as produced by fgq_ternarize for (M, Kred, G).
  *   y          out, fp32 [P][M].
  * The fp32 result is within 1e-5 * act_scale * sum_g |alpha_g * s_g| of the exact value.
+ * Memory: the tensor-core G = 4 kernel expands the codes to fp16 (2 * M * Kred bytes) in a
+ * temporary taken from a library-owned stream-ordered pool of the current device and
+ * returned to it on the same stream; the pool keeps freed blocks, so only a call that needs
+ * more than the pool holds reaches the device allocator.  No other path allocates.
  * Errors: FGQ_ERR_ARG (null pointers, bad sizes, Kred odd for 4-bit types),
  * FGQ_ERR_ALIGN (any pointer not 16-byte aligned), FGQ_ERR_CUDA.
  */

@@ -3,34 +3,40 @@
 // Math (Eq. 2, 32-bit group accumulators of Section 4): y[p][m] = s_x * sum_g alpha[m][g]
 // * s[m][g][p] with s an exact integer sum over a group of 4 reduction elements.  A dense
 // MMA would sum across groups, so each K = 16 MMA step (4 groups) uses a block-diagonal
-// activation operand B' of 256 rows: row (h, j, p) = 128 h + 32 j + p holds the
-// activations of tile position 32 h + p only in the 4 columns of group slot j (zeros
-// elsewhere).  Then D[m][128 h + 32 j + p] = s[m][group 4 step + j][32 h + p] exactly (fp16
-// operands on exact integers, |s| <= 4 * 255), each step into its own TMEM buffer, and
-// the epilogue applies alpha once per group-output on the CUDA cores (Section 4.1) with
-// packed fp32 FMAs.  The zeros of B' never change, so they are written once per CTA; each
-// K-tile writes only the diagonal 8-byte pieces.
+// activation operand B' of 256 rows: row 64 j + P holds the activations of tile position P
+// only in the 4 columns of group slot j (zeros elsewhere).  Each step is one MMA (M = 128,
+// N = 256, K = 16) into its own 256-column TMEM buffer: D[m][64 j + P] = s[m][group
+// 4 step + j][P] exactly (fp16 operands on exact integers, |s| <= 4 * 255), and the
+// epilogue applies alpha once per group-output on the CUDA cores (Section 4.1) with packed
+// fp32 FMAs.  The zeros of B' never change, so they are written once per CTA; each K-tile
+// writes only the diagonal 8-byte pieces.
 //
-// Tile: 128 filters x 64 positions; K-tile 64 (16 groups, 4 MMA steps of M = 128,
-// N = 256, K = 16).  TMEM: two 256-column buffers, the MMA of step s + 1 runs while the
-// epilogue drains step s.
+// The ternary operand A is expanded once per call from the 2-bit codes to fp16 {0, +1, -1}
+// in a stream-ordered temporary (expand_codes_kernel) and reaches shared memory by TMA box
+// loads in the MMA's swizzled layout.
+//
+// Tile: 128 filters x 64 positions; K-tile 64 (16 groups, 4 steps).  TMEM: two 256-column
+// buffers; the MMA of step s + 1 runs while the epilogue drains step s.  N = 256 keeps the
+// tensor pipe at its full rate, and one commit per step keeps the commits (each of which
+// drains the pipe) to four per K-tile.
 // Warp roles (416 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w owns TMEM lanes 32 (w % 4) .. (filters) and the 32
-//              positions of half w / 4; per step it reads the 4 group slots (4 x 32
-//              columns, each load overlapped with the FMAs of the previous one) and adds
-//              alpha * s into 32 position accumulators; at tile end it scales by s_x and
-//              writes its 32 x 32 block (through shared memory and a TMA box store when
-//              the output allows).
-//   warps 8-11 loaders/converters: thread t owns code row t of A and, for position
-//              t % 64, the two MMA steps 2 (t / 64), 2 (t / 64) + 1 of B'; copies come
-//              by TMA boxes (1x1 stride-1 layers and GEMMs) or by per-thread cp.async
-//              gathers whose completion is tracked on the stage's mbarrier.
+//              positions of half w / 4; per step it loads its four 32-column slices (two
+//              at a time, each later load overlapped with the FMAs of an earlier one), frees
+//              the buffer, and adds alpha * s into 32 position accumulators; at tile end it
+//              scales by s_x and writes its 32 x 32 block (through shared memory and a TMA
+//              box store when the output allows).
+//   warps 8-11 loaders/converters: thread t builds, for position t % 64, MMA steps
+//              2 (t / 64), 2 (t / 64) + 1 of B'; activations come by TMA boxes (1x1
+//              stride-1 layers and GEMMs) or by per-thread cp.async gathers whose completion
+//              is tracked on the stage's mbarrier; thread 0 also issues the A box loads.
 //   warp 12    TMEM allocation and the MMA issuer.
 // Every mbarrier wait is bounded in time; on expiry the kernel records FGQ_ERR_TIMEOUT,
 // each role leaves its loop (uniformly within the epilogue, which uses named barriers),
 // in-flight copies and MMAs are waited for, and TMEM is freed.
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "tc_common.cuh"
 
@@ -48,7 +54,7 @@ constexpr int T4_BP = 64;       // positions per tile
 constexpr int T4_KT = 64;       // reduction elements per K-tile: 16 groups, 4 MMA steps
 constexpr int T4_NO = 3;        // operand ring depth
 constexpr int T4_NS = 6;        // staging ring depth
-constexpr int T4_NACC = 2;      // TMEM accumulator buffers of 256 columns
+constexpr int T4_NACC = 2;      // TMEM buffers of 256 columns (one step each)
 constexpr int T4_EPI_WARPS = 8;
 constexpr int T4_LOAD_WARP0 = 8;  // loaders: warps 8-11
 constexpr int T4_LOADERS = 128;
@@ -61,24 +67,20 @@ constexpr uint32_t BAR_EPI4 = 2;
 constexpr int A_TILE4 = 128 * T4_KT * 2;   // 16 KB fp16 codes [128 filters][64 K]
 constexpr int B_TILE4 = 256 * T4_KT * 2;   // 32 KB fp16 block-diagonal activations
 constexpr int OP_STAGE4 = A_TILE4 + B_TILE4;
-constexpr int ST_ACT4 = T4_BP * T4_KT;     // 4 KB: 64 raw activation rows (8-bit: 64 B each)
-constexpr int ST_CODE4 = 128 * 16;         // 2 KB raw code words
-constexpr int ST_STAGE4 = ST_ACT4 + ST_CODE4;
+constexpr int ST_STAGE4 = T4_BP * T4_KT;   // 4 KB: 64 raw activation rows (8-bit: 64 B each)
 constexpr int OUT_TILE4 = T4_BP * T4_BM * 4;  // 32 KB fp32 [64 positions][128 filters]
 constexpr int SMEM_OP4 = T4_NO * OP_STAGE4;
 constexpr int SMEM_ST4 = T4_NS * ST_STAGE4;
-constexpr int SMEM_LUT4 = 16 * 32 * 4;
-constexpr int SMEM_BAR4 = 8 * (2 * T4_NO + 2 * T4_NS + 2 * T4_NACC + 1) + 16;
-constexpr int T4_SMEM = 1024 + SMEM_OP4 + SMEM_ST4 + OUT_TILE4 + SMEM_LUT4 + SMEM_BAR4;
+constexpr int SMEM_BAR4 = 8 * (3 * T4_NO + 2 * T4_NS + 2 * T4_NACC + 1) + 16;
+constexpr int T4_SMEM = 1024 + SMEM_OP4 + SMEM_ST4 + OUT_TILE4 + SMEM_BAR4;
 static_assert(T4_SMEM <= 232448, "shared memory budget");
 static_assert(ST_STAGE4 % 1024 == 0 && OP_STAGE4 % 1024 == 0, "stage alignment");
 
 struct T4Args {
-  CUtensorMap codes_map;  // uint32 [M][wrow], box {4 words, 128 rows}
+  CUtensorMap a16_map;    // fp16 [M][Kp] expanded codes, box {64, 128 rows}, 128-byte swizzle
   CUtensorMap act_map;    // uint8 [pixels][row bytes], box {64 (or 32) bytes, 64 rows}; TMA path
   CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 64 positions}; if out_tma
   const uint8_t* act;
-  const uint32_t* codes;
   const float* alpha;
   const float* act_scale;
   float* out;
@@ -107,6 +109,25 @@ __device__ __forceinline__ void scale_add(float (&acc)[32], const uint32_t (&r)[
     ffma2(acc[2 * i], acc[2 * i + 1], __uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]), al);
 }
 
+// Expands 2-bit codes (00 = 0, 01 = +1, 11 = -1; element k in word k / 16, bits 2 (k % 16))
+// to fp16 {0, +1, -1}: one thread per code word, 16 halves (32 bytes) out.
+__global__ void __launch_bounds__(256) expand_codes_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
+                                                           uint4* __restrict__ a16) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= nwords) return;
+  const uint32_t w = __ldg(codes + i);
+  uint32_t h[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const uint32_t c0 = (w >> (4 * e)) & 3u, c1 = (w >> (4 * e + 2)) & 3u;
+    const uint32_t lo = (c0 & 1u) ? ((c0 & 2u) ? 0xBC00u : 0x3C00u) : 0u;
+    const uint32_t hi = (c1 & 1u) ? ((c1 & 2u) ? 0xBC00u : 0x3C00u) : 0u;
+    h[e] = lo | (hi << 16);
+  }
+  a16[2 * i] = make_uint4(h[0], h[1], h[2], h[3]);
+  a16[2 * i + 1] = make_uint4(h[4], h[5], h[6], h[7]);
+}
+
 template <int ABITS, bool SIGNED, bool TMAP>
 __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __grid_constant__ T4Args a) {
   extern __shared__ uint8_t smem_raw4[];
@@ -114,11 +135,11 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   uint8_t* op = smem;
   uint8_t* st = smem + SMEM_OP4;
   float* otile = reinterpret_cast<float*>(smem + SMEM_OP4 + SMEM_ST4);
-  uint32_t* lut = reinterpret_cast<uint32_t*>(smem + SMEM_OP4 + SMEM_ST4 + OUT_TILE4);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP4 + SMEM_ST4 + OUT_TILE4 + SMEM_LUT4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP4 + SMEM_ST4 + OUT_TILE4);
   uint64_t* op_full = bars;
   uint64_t* op_empty = bars + T4_NO;
-  uint64_t* st_full = bars + 2 * T4_NO;
+  uint64_t* a_full = bars + 2 * T4_NO;
+  uint64_t* st_full = bars + 3 * T4_NO;
   uint64_t* st_empty = st_full + T4_NS;
   uint64_t* acc_full = st_empty + T4_NS;
   uint64_t* acc_empty = acc_full + T4_NACC;
@@ -133,8 +154,9 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < T4_NO; ++i) {
-      mbar_init(&op_full[i], T4_LOADERS);
+      mbar_init(&op_full[i], T4_LOADERS);  // B' pieces
       mbar_init(&op_empty[i], 1);
+      mbar_init(&a_full[i], 1);            // the A box's byte count
     }
     for (int i = 0; i < T4_NS; ++i) {
       mbar_init(&st_full[i], TMAP ? 1 : T4_LOADERS);
@@ -148,7 +170,6 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     *abort_flag = 0;
     fence_mbar_init();
   }
-  tc::fill_code_lut(lut);
   // the off-diagonal zeros of every B' tile, written once
   for (int s = 0; s < T4_NO; ++s) {
     uint4* bt = reinterpret_cast<uint4*>(op + s * OP_STAGE4 + A_TILE4);
@@ -175,18 +196,18 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     const int t = threadIdx.x - 32 * T4_LOAD_WARP0;
     const int P = t & (T4_BP - 1);  // tile position whose activations this thread copies/converts
     const int cpair = t >> 6;       // MMA steps 2 cpair, 2 cpair + 1 of the K-tile
-    const int hsub = P >> 5, pl = P & 31;
     const int total = my_tiles * a.ktiles;
     constexpr int ROW_BYTES = T4_KT * ABITS / 8;
     constexpr int CPT = ROW_BYTES / 32;  // 16-byte chunks per thread and K-tile (2 or 1)
-    constexpr uint32_t TX_BYTES = 128 * 16 + T4_BP * ROW_BYTES;
+    constexpr uint32_t TX_ACT = T4_BP * ROW_BYTES;
 
+    // walk of the K-tiles this thread issues copies for
     int cur_tile = -1, gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0;
     int64_t p0 = 0;
     int pb = 0, phb = 0, pwb = 0;
     bool pvalid = false;
-    int issued = 0;
-    // copies of K-tile j (of this CTA's sequence) into staging slot j % NS; false on timeout
+    int issued = 0, a_armed = 0;
+    // activation copies of K-tile j (of this CTA's sequence) into staging slot j % NS
     auto issue = [&](int j) -> bool {
       const int tl = j / a.ktiles;
       if (tl != cur_tile) {
@@ -205,13 +226,11 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       }
       const int slot = j % T4_NS;
       uint8_t* sa = st + slot * ST_STAGE4;
-      const int kk = j - tl * a.ktiles;
       if (TMAP) {
         if (t == 0) {
           if (j >= T4_NS && !mbar_wait_timed(&st_empty[slot], ((j / T4_NS) & 1) ^ 1, tmo, abort_flag, 64))
             return false;
-          mbar_arrive_expect_tx(&st_full[slot], TX_BYTES);
-          tma_load_2d(smem_u32(sa + ST_ACT4), &a.codes_map, kk * (T4_KT / 16), m0, &st_full[slot]);
+          mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
           tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
           issued = j + 1;
         }
@@ -234,10 +253,6 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
           cp_async16(smem_u32(sa + st_off<ABITS>(P, c)), inside ? (const void*)(src + 16 * c) : (const void*)a.act,
                      inside ? 16u : 0u);
         }
-        const int m = m0 + t;
-        const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
-        const uint32_t* csrc = mok ? a.codes + (int64_t)m * g.wrow + kk * (T4_KT / 16) : a.codes;
-        cp_async16(smem_u32(sa + ST_ACT4 + t * 16), csrc, mok ? 16u : 0u);
         cp_async_mbar_arrive_noinc(&st_full[slot]);
         issued = j + 1;
       }
@@ -262,18 +277,29 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       }
       const int slot = j % T4_NS;
       const int os = j % T4_NO;
-      if (!mbar_wait_timed(&st_full[slot], (j / T4_NS) & 1, tmo, abort_flag, 32) ||
-          !mbar_wait_timed(&op_empty[os], ((j / T4_NO) & 1) ^ 1, tmo, abort_flag, 64)) {
+      if (!mbar_wait_timed(&op_empty[os], ((j / T4_NO) & 1) ^ 1, tmo, abort_flag, 64)) {
+        ok = false;
+        break;
+      }
+      uint8_t* A = op + os * OP_STAGE4;
+      uint8_t* Bt = A + A_TILE4;
+      if (t == 0) {  // the A box of K-tile j: expanded codes of the tile's 128 filters
+        const int tl = j / a.ktiles;
+        int gj, mj;
+        int64_t pj;
+        tile_coords4(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
+        mbar_arrive_expect_tx(&a_full[os], A_TILE4);
+        tma_load_2d(smem_u32(A), &a.a16_map, (j - tl * a.ktiles) * T4_KT, mj, &a_full[os]);
+        a_armed = j + 1;
+      }
+      if (!mbar_wait_timed(&st_full[slot], (j / T4_NS) & 1, tmo, abort_flag, 32)) {
         ok = false;
         break;
       }
       consumed = j + 1;
       const uint8_t* sa = st + slot * ST_STAGE4;
-      uint8_t* A = op + os * OP_STAGE4;
-      uint8_t* Bt = A + A_TILE4;
-      tc::codes_row_to_fp16(sa + ST_ACT4 + t * 16, A, t, lut + lane);
-      // B' rows (hsub, j, pl) for j = 0..3, MMA steps s of this thread: the 4 activations of
-      // group slot j at K offsets 16 s + 4 j .. +3
+      // B' rows 64 jj + P for slots jj = 0..3, MMA steps s of this thread: the 4 activations
+      // of group slot jj at K offsets 16 s + 4 jj .. +3
       uint32_t wv[2][4];
       if (ABITS == 8) {
 #pragma unroll
@@ -286,7 +312,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         }
       } else {
         // one 16-byte chunk = steps 2 cpair (bytes 0-7) and 2 cpair + 1 (bytes 8-15); the 4
-        // nibbles of slot j are 16-bit half j of the step's 8 bytes
+        // nibbles of slot jj are 16-bit half jj of the step's 8 bytes
         const uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<4>(P, cpair));
         const uint32_t half[2][2] = {{v.x, v.y}, {v.z, v.w}};
 #pragma unroll
@@ -307,7 +333,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         for (int jj = 0; jj < 4; ++jj) {
           const uint32_t w = SIGNED ? (wv[ss][jj] ^ flip) : wv[ss][jj];
           const uint2 hv = make_uint2(u8pair_to_h2(w, 0x4140, bias2), u8pair_to_h2(w, 0x4342, bias2));
-          *reinterpret_cast<uint2*>(Bt + sw128(128 * hsub + 32 * jj + pl, 2 * s + (jj >> 1)) + 8 * (jj & 1)) = hv;
+          *reinterpret_cast<uint2*>(Bt + sw128(64 * jj + P, 2 * s + (jj >> 1)) + 8 * (jj & 1)) = hv;
         }
       }
       fence_proxy_async_smem();
@@ -318,6 +344,10 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     if (!TMAP) cp_async_wait_all();
     if (TMAP && t == 0) {
       for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % T4_NS], (j / T4_NS) & 1, 1u << 16);
+    }
+    if (t == 0 && !ok && a_armed > 0) {  // the last A box may still be in flight
+      const int j = a_armed - 1;
+      mbar_wait_bounded(&a_full[j % T4_NO], (j / T4_NO) & 1, 1u << 16);
     }
   }
 
@@ -330,7 +360,8 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     bool ok = true;
     for (int j = 0; j < total && ok; ++j) {
       const int os = j % T4_NO;
-      if (!mbar_wait_timed(&op_full[os], (j / T4_NO) & 1, tmo, abort_flag, 32)) {
+      if (!mbar_wait_timed(&op_full[os], (j / T4_NO) & 1, tmo, abort_flag, 0) ||
+          !mbar_wait_timed(&a_full[os], (j / T4_NO) & 1, tmo, abort_flag, 0)) {
         ok = false;
         break;
       }
@@ -340,7 +371,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       const uint64_t bd = sdesc_k_sw128(abase + A_TILE4);
       for (int s = 0; s < 4; ++s, ++sc) {
         const int b = sc & 1;
-        if (!mbar_wait_timed(&acc_empty[b], ((sc >> 1) & 1) ^ 1, tmo, abort_flag, 32)) {
+        if (!mbar_wait_timed(&acc_empty[b], ((sc >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
           ok = false;
           break;
         }
@@ -359,7 +390,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   if (warp < T4_EPI_WARPS) {
     const int quarter = warp & 3, hsub = warp >> 2;
     const int t = 32 * quarter + lane;  // TMEM lane = filter row of the tile
-    const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(128 * hsub);
+    const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(32 * hsub);
     const float sx = __ldg(a.act_scale);
     const bool leader = threadIdx.x == 0;
     const int nsteps = a.ktiles * 4;
@@ -379,29 +410,30 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       float4 al_next = mok ? __ldg(arow) : make_float4(0.f, 0.f, 0.f, 0.f);
       for (int gs = 0; gs < nsteps; ++gs, ++sc) {
         if (!ok) continue;
-        const int b = sc & 1;
         const float4 al = al_next;
         if (mok && gs + 1 < nsteps) al_next = __ldg(arow + gs + 1);
+        const int b = sc & 1;
         if (!mbar_wait_timed(&acc_full[b], (sc >> 1) & 1, tmo, abort_flag, 0)) {
           ok = false;
           continue;
         }
         tc_fence_after();
+        // slot j at columns 64 j .. 64 j + 63; this warp's 32 positions at + 32 hsub
         const uint32_t ta = tbase + (uint32_t)(b * 256);
         uint32_t r0[32], r1[32];
         tmem_ld32(ta, r0);
+        tmem_ld32(ta + 64, r1);
         tmem_ld_wait_regs(r0);
-        tmem_ld32(ta + 32, r1);
+        reg_fence(r1);
         scale_add(acc, r0, al.x);
-        tmem_ld_wait_regs(r1);
-        tmem_ld32(ta + 64, r0);
+        tmem_ld32(ta + 128, r0);
         scale_add(acc, r1, al.y);
+        tmem_ld32(ta + 192, r1);
         tmem_ld_wait_regs(r0);
-        tmem_ld32(ta + 96, r1);
-        scale_add(acc, r0, al.z);
-        tmem_ld_wait_regs(r1);
+        reg_fence(r1);
         tc_fence_before();
         if (lane == 0) mbar_arrive(&acc_empty[b]);
+        scale_add(acc, r0, al.z);
         scale_add(acc, r1, al.w);
       }
       if (!ok && !*abort_flag) fail();
@@ -454,6 +486,29 @@ fgq_status launch_tc4_path(const T4Args& args, int grid, cudaStream_t s) {
   return args.act_tma ? launch_tc4<ABITS, SIGNED, true>(args, grid, s) : launch_tc4<ABITS, SIGNED, false>(args, grid, s);
 }
 
+// Stream-ordered memory pool of the current device for the expanded-code temporaries; it
+// keeps freed blocks (no release threshold), so steady-state calls do not reach the OS.
+cudaMemPool_t a16_pool() {
+  static std::mutex mu;
+  static cudaMemPool_t pools[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!pools[dev]) {
+    cudaMemPoolProps props;
+    memset(&props, 0, sizeof props);
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    cudaMemPool_t p = nullptr;
+    if (cudaMemPoolCreate(&p, &props) != cudaSuccess) return nullptr;
+    uint64_t keep = ~0ull;
+    cudaMemPoolSetAttribute(p, cudaMemPoolAttrReleaseThreshold, &keep);
+    pools[dev] = p;
+  }
+  return pools[dev];
+}
+
 }  // namespace
 
 bool tc4_supports(const Geom& g) {
@@ -471,7 +526,6 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   T4Args a;
   memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
-  a.codes = codes;
   a.alpha = alpha;
   a.act_scale = act_scale;
   a.out = out;
@@ -483,10 +537,20 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   a.ktiles = g.Kp / T4_KT;
   a.timeout_ns = T4_TIMEOUT_NS;
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
-  if (!make_map_2d(&a.codes_map, CU_TENSOR_MAP_DATA_TYPE_UINT32, codes, (uint64_t)g.wrow, (uint64_t)g.M,
-                   (uint64_t)g.wrow * 4, T4_KT / 16, T4_BM, CU_TENSOR_MAP_SWIZZLE_NONE))
-    return FGQ_ERR_CUDA;
-  if (g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
+
+  // expanded codes: fp16 [M][Kp] (Kp = 16 wrow), in a temporary from the stream-ordered pool
+  cudaMemPool_t pool = a16_pool();
+  if (!pool) return FGQ_ERR_CUDA;
+  const int64_t nwords = (int64_t)g.M * g.wrow;
+  void* a16 = nullptr;
+  if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 32, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
+  expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
+  fgq_status st = after_launch();
+  if (st == FGQ_OK &&
+      !make_map_2d(&a.a16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a16, (uint64_t)g.wrow * 16, (uint64_t)g.M,
+                   (uint64_t)g.wrow * 32, T4_KT, T4_BM, CU_TENSOR_MAP_SWIZZLE_128B))
+    st = FGQ_ERR_CUDA;
+  if (st == FGQ_OK && g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
     const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
     a.act_tma = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, row_bytes, (uint64_t)g.B * g.H * g.W,
                             row_bytes, (uint32_t)(T4_KT * abits / 8), T4_BP,
@@ -494,19 +558,26 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
                     ? 1
                     : 0;
   }
-  if (g.groups == 1 && g.M % 4 == 0) {
+  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, T4_BM, T4_BP, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1
                     : 0;
   }
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int grid = a.ntiles < sms ? a.ntiles : sms;
-  const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
-  if (abits == 4) return sgn ? launch_tc4_path<4, true>(a, grid, s) : launch_tc4_path<4, false>(a, grid, s);
-  return sgn ? launch_tc4_path<8, true>(a, grid, s) : launch_tc4_path<8, false>(a, grid, s);
+  if (st == FGQ_OK) {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = a.ntiles < sms ? a.ntiles : sms;
+    const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
+    if (abits == 4)
+      st = sgn ? launch_tc4_path<4, true>(a, grid, s) : launch_tc4_path<4, false>(a, grid, s);
+    else
+      st = sgn ? launch_tc4_path<8, true>(a, grid, s) : launch_tc4_path<8, false>(a, grid, s);
+  }
+  // the temporary returns to the pool once the work queued on s before this point is done
+  if (cudaFreeAsync(a16, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  return st;
 }
 
 }  // namespace fgq

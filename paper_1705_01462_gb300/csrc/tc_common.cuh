@@ -66,6 +66,19 @@ __device__ __forceinline__ void codes_row_to_fp16(const uint8_t* codes16, uint8_
   }
 }
 
+// Half h (codes 32 h .. 32 h + 31, 8 bytes) of one K-tile row: 16-byte chunks 4 h .. 4 h + 3
+// of row t of the 128B-swizzled operand tile.
+__device__ __forceinline__ void codes_half_row_to_fp16(const uint8_t* codes16, int h, uint8_t* tile, int t,
+                                                       const uint32_t* lt) {
+  const uint2 cw = *reinterpret_cast<const uint2*>(codes16 + 8 * h);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t bits = ((i < 2 ? cw.x : cw.y) >> (16 * (i & 1))) & 0xffffu;  // 8 codes
+    *reinterpret_cast<uint4*>(tile + sw128(t, 4 * h + i)) =
+        make_uint4(lt[32 * (bits & 15u)], lt[32 * ((bits >> 4) & 15u)], lt[32 * ((bits >> 8) & 15u)], lt[32 * (bits >> 12)]);
+  }
+}
+
 // cuTensorMapEncodeTiled from the driver, looked up once through the runtime.
 inline PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
