@@ -44,6 +44,9 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--batch", type=int, default=BATCH,
+                    help="images per GPU (the benchmark workload is 64; smaller batches serve profiler "
+                         "captures that must stay small)")
     return ap.parse_args()
 
 
@@ -425,7 +428,8 @@ def main():
     peaks = load_peaks()
     sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
     layers = workload_layers()
-    W = Workload(dev, BATCH, layers, seed_offset=rank_seed_offset(rank))
+    B = args.batch
+    W = Workload(dev, B, layers, seed_offset=rank_seed_offset(rank))
     stream = torch.cuda.Stream(device=dev)
 
     with torch.cuda.stream(stream):
@@ -458,13 +462,13 @@ def main():
         raise RuntimeError(f"device error during the timed region: {status}")
     total_ms = max_over_ranks(pg, total_ms, dev)
     ms_per_step = total_ms / args.steps
-    ops_rank = total_ops(layers, BATCH)
+    ops_rank = total_ops(layers, B)
     value = whole_job_rate(ops_rank, ws, ms_per_step)
 
     fam_ms = {f: sum(a.elapsed_time(b) for a, b in ev) for f, ev in timers.items()}
     dom = max(fam_ms, key=fam_ms.get)
     paths = W.paths
-    roof = family_roofline(dom, layers, BATCH, peaks, sm_count, fam_ms[dom] / 1e3 / args.steps, paths)
+    roof = family_roofline(dom, layers, B, peaks, sm_count, fam_ms[dom] / 1e3 / args.steps, paths)
     traffic = load_traffic().get(dom)
     n_launch_per_step = len(timers[dom]) / args.steps
     roofline = {"kernel": dom, "bound": roof["bound"], "achieved": roof["achieved"], "peak": roof["peak"],
@@ -508,14 +512,14 @@ def main():
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        v, desc, cores = oracle_sample(layers, BATCH, args.cpu_seconds)
+        v, desc, cores = oracle_sample(layers, B, args.cpu_seconds)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "u8xternary->int32->f32", "data": "synthetic",
-                "config": {"workload": "ResNet-50 conv stack (53 convs), batch 64 per GPU, 224x224, uint8 DFP "
+                "config": {"workload": f"ResNet-50 conv stack (53 convs), batch {B} per GPU, 224x224, uint8 DFP "
                                        "activations, ternary weights at G=4 and G=64, first layer 8-bit weights",
                            "ops_per_step_per_gpu": ops_rank,
                            "l2": "no flush: per-step working set ~9 GB >> 129 MB L2",
