@@ -193,56 +193,68 @@ class Workload:
                 self.out[G].append(torch.empty((B, l.Ho, l.Wo, l.M), dtype=torch.float32, device=dev))
         torch.cuda.synchronize()
 
-    def step(self, stream, timers=None):
-        """Issue one step on `stream`; timers: dict family -> list of (start, end) events."""
+    def step(self, stream, timers=None, counts=None):
+        """Issue one step on `stream`.  The calls of one kernel family run back to back, and
+        with `timers` (dict family -> list of (start, end) events) one event pair brackets
+        each contiguous run of a family, so the per-family times cost a handful of events
+        per step instead of two per call; `counts` (dict family -> calls) is filled on the
+        way."""
         fgq = self.fgq
         L = fgq.lib()
         sh = stream.cuda_stream
         torch = self.torch
-
-        def timed(fam, fn):
-            if timers is None:
-                return fn()
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            r = fn()
-            e1.record(stream)
-            timers.setdefault(fam, []).append((e0, e1))
-            return r
+        calls = []  # (family, function) in issue order
 
         def chk(code, what):
             if code != 0:
                 raise RuntimeError(f"{what} failed: {L.fgq_status_string(code).decode()}")
 
-        for i, l in enumerate(self.layers):
-            for G in GROUPS:
-                if i == 0:
-                    timed("quantize_weights_w8", lambda: chk(L.fgq_quantize_weights_w8(
-                        self.w[i].data_ptr(), l.M, l.Kred, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(),
-                        sh), "w8"))
-                else:
-                    timed(f"ternarize_g{G}", lambda: chk(L.fgq_ternarize(
-                        self.w[i].data_ptr(), l.M, l.Kred, G, self.codes[G][i].data_ptr(),
-                        self.alpha[G][i].data_ptr(), sh), "ternarize"))
-        for i, l in enumerate(self.layers):
-            n = self.x[i].numel()
-            timed("quantize_act", lambda: chk(L.fgq_quantize_act(
-                self.x[i].data_ptr(), n, fgq.U8, 0.0, self.q[i].data_ptr(), self.sc[i].data_ptr(),
-                self.ws[i].data_ptr(), self.ws[i].numel(), sh), "quantize"))
+        for G in GROUPS:  # first layer: 8-bit weights (8w-8a)
+            l = self.layers[0]
+            calls.append(("quantize_weights_w8", lambda G=G, l=l: chk(L.fgq_quantize_weights_w8(
+                self.w[0].data_ptr(), l.M, l.Kred, self.codes[G][0].data_ptr(), self.alpha[G][0].data_ptr(), sh),
+                "w8")))
         for G in GROUPS:
-            for i, l in enumerate(self.layers):
-                if i == 0:
-                    timed("conv_w8_stem", lambda: chk(L.fgq_conv2d_w8(
-                        self.q[i].data_ptr(), fgq.U8, self.sc[i].data_ptr(), self.B, l.H, l.W, l.C, l.R, l.S,
-                        l.stride, l.pad, l.groups, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(), l.M,
-                        self.out[G][i].data_ptr(), sh), "conv_w8"))
-                else:
-                    timed(f"conv_g{G}", lambda: chk(L.fgq_conv2d(
-                        self.q[i].data_ptr(), fgq.U8, self.sc[i].data_ptr(), self.B, l.H, l.W, l.C, l.R, l.S,
-                        l.stride, l.pad, l.groups, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(), l.M, G,
-                        self.out[G][i].data_ptr(), sh), "conv"))
+            for i, l in enumerate(self.layers[1:], start=1):
+                calls.append((f"ternarize_g{G}", lambda G=G, i=i, l=l: chk(L.fgq_ternarize(
+                    self.w[i].data_ptr(), l.M, l.Kred, G, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(),
+                    sh), "ternarize")))
+        for i, l in enumerate(self.layers):
+            calls.append(("quantize_act", lambda i=i: chk(L.fgq_quantize_act(
+                self.x[i].data_ptr(), self.x[i].numel(), fgq.U8, 0.0, self.q[i].data_ptr(), self.sc[i].data_ptr(),
+                self.ws[i].data_ptr(), self.ws[i].numel(), sh), "quantize")))
+        for G in GROUPS:
+            l = self.layers[0]
+            calls.append(("conv_w8_stem", lambda G=G, l=l: chk(L.fgq_conv2d_w8(
+                self.q[0].data_ptr(), fgq.U8, self.sc[0].data_ptr(), self.B, l.H, l.W, l.C, l.R, l.S, l.stride,
+                l.pad, l.groups, self.codes[G][0].data_ptr(), self.alpha[G][0].data_ptr(), l.M,
+                self.out[G][0].data_ptr(), sh), "conv_w8")))
+        for G in GROUPS:
+            for i, l in enumerate(self.layers[1:], start=1):
+                def conv(G=G, i=i, l=l):
+                    chk(L.fgq_conv2d(self.q[i].data_ptr(), fgq.U8, self.sc[i].data_ptr(), self.B, l.H, l.W, l.C, l.R,
+                                     l.S, l.stride, l.pad, l.groups, self.codes[G][i].data_ptr(),
+                                     self.alpha[G][i].data_ptr(), l.M, G, self.out[G][i].data_ptr(), sh), "conv")
                     self.paths[(G, i)] = L.fgq_last_path()
+                calls.append((f"conv_g{G}", conv))
+
+        cur, e0 = None, None
+        for fam, fn in calls:
+            if timers is not None and fam != cur:
+                if cur is not None:
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e1.record(stream)
+                    timers.setdefault(cur, []).append((e0, e1))
+                e0 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                cur = fam
+            fn()
+            if counts is not None:
+                counts[fam] = counts.get(fam, 0) + 1
+        if timers is not None and cur is not None:
+            e1 = torch.cuda.Event(enable_timing=True)
+            e1.record(stream)
+            timers.setdefault(cur, []).append((e0, e1))
 
 
 def alu_peak_tops(G, sm_count, clk_hz):
@@ -444,14 +456,14 @@ def main():
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    timers = {}
+    timers, counts = {}, {}
     launches0 = fgq.fgq_launch_count()
     e_start = torch.cuda.Event(enable_timing=True)
     e_end = torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         e_start.record(stream)
         for _ in range(args.steps):
-            W.step(stream, timers)
+            W.step(stream, timers, counts)
         e_end.record(stream)
     torch.cuda.synchronize()
     launches = fgq.fgq_launch_count() - launches0
@@ -470,7 +482,7 @@ def main():
     paths = W.paths
     roof = family_roofline(dom, layers, B, peaks, sm_count, fam_ms[dom] / 1e3 / args.steps, paths)
     traffic = load_traffic().get(dom)
-    n_launch_per_step = len(timers[dom]) / args.steps
+    n_launch_per_step = counts[dom] / args.steps  # API calls of the family per step
     roofline = {"kernel": dom, "bound": roof["bound"], "achieved": roof["achieved"], "peak": roof["peak"],
                 "unit": roof["unit"], "frac": roof["achieved"] / roof["peak"],
                 "traffic": traffic, "peak_source": peaks["source"],

@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     }
     for (int i = 0; i < TC_NACC; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], 32 * TC_EPI_WARPS);
+      mbar_init(&acc_empty[i], TC_EPI_WARPS);  // one arrival per epilogue warp
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -271,7 +271,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       const int slot = j % TC_NS;
       const int os = j % TC_NO;
       if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag)) ||
-          !mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)) {
+          !(a.kt_per_group > 1
+                ? mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)
+                : (j < TC_NO || mbar_wait_or_abort(&acc_full[(j - TC_NO) % TC_NACC], ((j - TC_NO) / TC_NACC) & 1,
+                                                   a.wait_limit, abort_flag)))) {
         if (!*abort_flag) fail();
         break;
       }
@@ -383,7 +386,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
             // advance 16 fp16 (32 bytes) along K inside the swizzled rows
             mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (sub > 0 || k > 0) ? 1u : 0u);
           }
-          mma_commit(&op_empty[os]);
+          // with one K-tile per group the group's acc_full commit also frees the operand
+          // stage (the loaders wait on it), so a second commit is not spent on op_empty
+          if (a.kt_per_group > 1) mma_commit(&op_empty[os]);
         }
         if (ok) mma_commit(&acc_full[b]);
       }
@@ -432,7 +437,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         tmem_ld32(tbase + (uint32_t)(b * TC_BN + 32), r);
         tmem_ld_wait();
         tc_fence_before();
-        mbar_arrive(&acc_empty[b]);  // the buffer is free once the values are in registers
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[b]);  // the buffer is free once the values are in registers
 #pragma unroll
         for (int j = 0; j < 32; ++j) acc[32 + j] = fmaf(al, __uint_as_float(r[j]), acc[32 + j]);
       }

@@ -432,6 +432,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         tmem_ld_wait_regs(r0);
         reg_fence(r1);
         tc_fence_before();
+        __syncwarp();
         if (lane == 0) mbar_arrive(&acc_empty[b]);
         scale_add(acc, r0, al.z);
         scale_add(acc, r1, al.w);
