@@ -31,6 +31,26 @@ __device__ __forceinline__ uint32_t mag_bits(float x, bool is_unsigned) {
   return b & 0x7fffffffu;
 }
 
+// float4 loads with an L2 eviction-priority hint: pass 1 marks the input evict-last so that
+// as much of it as fits is still in L2 when pass 2 reads it (evict-first: not needed again).
+__device__ __forceinline__ float4 ld_f4_policy(const float4* p, uint64_t pol) {
+  float4 v;
+  asm volatile("ld.global.nc.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
 __global__ void __launch_bounds__(kThreads) qa_max_kernel(const float* __restrict__ x, size_t n, int is_unsigned,
                                                           uint32_t* __restrict__ partials, unsigned int* err) {
   uint32_t mx = 0;
@@ -39,8 +59,9 @@ __global__ void __launch_bounds__(kThreads) qa_max_kernel(const float* __restric
   const float4* x4 = reinterpret_cast<const float4*>(x);
   const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const size_t nth = (size_t)gridDim.x * blockDim.x;
+  const uint64_t keep = policy_evict_last();
   for (size_t i = tid; i < n4; i += nth) {
-    const float4 f = __ldg(x4 + i);
+    const float4 f = ld_f4_policy(x4 + i, keep);
     const float e[4] = {f.x, f.y, f.z, f.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -118,11 +139,15 @@ __global__ void __launch_bounds__(kThreads) qa_quant_kernel(const float* __restr
   const size_t tid = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const size_t nth = (size_t)gridDim.x * blockDim.x;
   const float4* x4 = reinterpret_cast<const float4*>(x);
-  for (size_t c = tid; c < n16; c += nth) {
+  const uint64_t drop = policy_evict_first();
+  // chunks in reverse of pass 1's order: the part of x pass 1 read last is the part most
+  // likely still in L2
+  for (size_t c0 = tid; c0 < n16; c0 += nth) {
+    const size_t c = n16 - 1 - c0;
     float e[16];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const float4 f = __ldg(x4 + 4 * c + j);
+      const float4 f = ld_f4_policy(x4 + 4 * c + j, drop);
       e[4 * j] = f.x; e[4 * j + 1] = f.y; e[4 * j + 2] = f.z; e[4 * j + 3] = f.w;
     }
     if (T::bits == 8) {
