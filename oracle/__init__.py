@@ -67,6 +67,9 @@ def lib() -> ctypes.CDLL:
         L.oracle_conv2d_w8.argtypes = conv_args + [_P(ctypes.c_int8), _P(c_f), c_i, _P(c_d), _P(c_d)]
         L.oracle_gemm.argtypes = [_P(ctypes.c_int32), c_d, c_i, c_i, _P(ctypes.c_int8), _P(c_f), c_i, c_i,
                                   _P(c_d), _P(c_d)]
+        L.oracle_ternarize_threshold.argtypes = [_P(c_f), c_i, c_i, c_i, c_i, c_i, _P(ctypes.c_int8), _P(c_f),
+                                                 ctypes.c_void_p]
+        L.oracle_ternary_error.argtypes = [_P(c_f), c_i, c_i, c_i, _P(ctypes.c_int8), _P(c_f), _P(c_d)]
         L.oracle_group_sums.argtypes = [_P(ctypes.c_int32), c_i, c_i, _P(ctypes.c_int8), c_i, c_i,
                                         _P(ctypes.c_int64)]
         _lib = L
@@ -132,6 +135,38 @@ def ternarize(w: np.ndarray, G: int, check: bool = True):
     if check:
         _check(st, "ternarize")
     return t, alpha, st
+
+
+RULE_EXP, RULE_GAUSS = 0, 1
+
+
+def ternarize_threshold(w: np.ndarray, G: int, rule: int, per_layer: bool = False, check: bool = True):
+    """Analytical-threshold ternarization (Section 3, Lemma 1; see the C file):
+    w fp32 [M][Kred] -> (t int8 [M][Kp], alpha fp32 [M][Kp/G], delta fp64 [M][Kp/G] or [1], status)."""
+    w = np.ascontiguousarray(w, dtype=np.float32)
+    M, Kred = w.shape
+    ng = num_groups(Kred, G)
+    t = np.zeros((M, ng * G), dtype=np.int8)
+    alpha = np.zeros((M, ng), dtype=np.float32)
+    delta = np.zeros(1 if per_layer else (M, ng), dtype=np.float64)
+    st = lib().oracle_ternarize_threshold(_ptr(w, ctypes.c_float), M, Kred, G, rule, int(per_layer),
+                                          _ptr(t, ctypes.c_int8), _ptr(alpha, ctypes.c_float),
+                                          delta.ctypes.data_as(ctypes.c_void_p))
+    if check:
+        _check(st, "ternarize_threshold")
+    return t, alpha, delta, st
+
+
+def ternary_error(w: np.ndarray, t: np.ndarray, alpha: np.ndarray, G: int) -> np.ndarray:
+    """Per-group ||w - alpha t||^2 (fp64 [M][Kp/G])."""
+    w = np.ascontiguousarray(w, dtype=np.float32)
+    t = np.ascontiguousarray(t, dtype=np.int8)
+    alpha = np.ascontiguousarray(alpha, dtype=np.float32)
+    M, Kred = w.shape
+    err = np.zeros((M, num_groups(Kred, G)), dtype=np.float64)
+    _check(lib().oracle_ternary_error(_ptr(w, ctypes.c_float), M, Kred, G, _ptr(t, ctypes.c_int8),
+                                      _ptr(alpha, ctypes.c_float), _ptr(err, ctypes.c_double)), "ternary_error")
+    return err
 
 
 def pack_codes(t: np.ndarray) -> np.ndarray:

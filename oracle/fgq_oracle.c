@@ -24,6 +24,9 @@
  *   oracle_gemm                 grouped contraction for a [P][Kred] activation matrix
  *   oracle_group_sums           the int32-accumulator group sums s[m][g][p]
  *   oracle_conv2d_w8            dense 8-bit-weight convolution (first layer, Section 4)
+ *   oracle_ternarize_threshold  ternarization at an analytical threshold (Section 3, Lemma 1),
+ *                               per group or with one threshold and one alpha per layer
+ *   oracle_ternary_error        per-group ternary error ||w - alpha t||^2 (Section 3)
  *
  * Readings of the paper that this file fixes (where the paper is silent):
  *   - Ties between candidate thresholds with exactly equal objective are broken towards
@@ -556,5 +559,132 @@ int oracle_conv2d_w8(const int32_t* q, double act_scale, int B, int H, int W, in
         }
       }
   free(col);
+  return ORACLE_OK;
+}
+
+/*
+ * Threshold ternarization with an analytical threshold (Section 3: t_i = sign(w_i) if
+ * |w_i| > Delta, else 0; Lemma 1 and its Gaussian counterpart).  One threshold per group
+ * of G (per_layer = 0) or one for the whole M x Kred layer (per_layer = 1):
+ *   rule 0, exponential magnitudes (Lemma 1): Delta = mean |w|;
+ *   rule 1, Gaussian weights: Delta = ORACLE_Z_GAUSS * rms(w), rms(w) the maximum-
+ *     likelihood sigma of N(0, sigma) that the paper names, and ORACLE_Z_GAUSS the z that
+ *     maximises phi(z)^2 / (1 - Phi(z)): for w ~ N(0, sigma^2) and many elements, the
+ *     threshold objective (sum_{|w| > Delta} |w|)^2 / |I_Delta| is proportional to that
+ *     function of z = Delta / sigma (the Gaussian counterpart of the Lemma 1 derivation).
+ * alpha = mean of the kept |w| (for a fixed support, the alpha of Eq. 4; 0 if none is
+ * kept): per group when per_layer = 0, one value for the layer (written to every
+ * alpha[m][g]) when per_layer = 1 -- the one-scaling-factor-per-layer baseline.  The
+ * statistics cover the real weights only (a row's zero padding is not counted).  All sums
+ * are fp64 in element order (row-major over the layer when per_layer = 1); the threshold
+ * is kept in fp64 and compared with |w| (fp32 promoted exactly); alpha = (float)(S / k).
+ * delta_out (may be NULL) receives the per-group thresholds [M][ng] (or one per layer).
+ * Non-finite weights: ORACLE_ERR_NONFINITE, and the affected groups (or the layer) get
+ * t = 0, alpha = 0.
+ */
+#define ORACLE_Z_GAUSS 0.6120031809624808
+
+static double threshold_of(double sum_abs, double sum_sq, int64_t n, int rule) {
+  if (n == 0) return 0.0;
+  if (rule == 0) return sum_abs / (double)n;
+  return ORACLE_Z_GAUSS * sqrt(sum_sq / (double)n);
+}
+
+int oracle_ternarize_threshold(const float* w, int M, int Kred, int G, int rule, int per_layer,
+                               int8_t* t, float* alpha, double* delta_out) {
+  int m, g, j;
+  int ng, Kp;
+  if (M < 0 || Kred < 0 || G < 1 || (rule != 0 && rule != 1)) return ORACLE_ERR_ARG;
+  ng = (Kred + G - 1) / G;
+  Kp = ng * G;
+  memset(t, 0, (size_t)M * Kp);
+  if (per_layer) {
+    double sa = 0.0, sq = 0.0, kept = 0.0, delta;
+    int64_t n = (int64_t)M * Kred, k = 0;
+    size_t i;
+    float a;
+    for (i = 0; i < (size_t)n; i++) {
+      if (!isfinite(w[i])) {
+        for (i = 0; i < (size_t)M * ng; i++) alpha[i] = 0.0f;
+        if (delta_out) delta_out[0] = 0.0;
+        return ORACLE_ERR_NONFINITE;
+      }
+      sa += fabs((double)w[i]);
+      sq += (double)w[i] * (double)w[i];
+    }
+    delta = threshold_of(sa, sq, n, rule);
+    for (m = 0; m < M; m++)
+      for (j = 0; j < Kred; j++) {
+        const double v = (double)w[(size_t)m * Kred + j];
+        if (fabs(v) > delta) {
+          t[(size_t)m * Kp + j] = v > 0 ? 1 : -1;
+          kept += fabs(v);
+          k++;
+        }
+      }
+    a = k ? (float)(kept / (double)k) : 0.0f;
+    for (i = 0; i < (size_t)M * ng; i++) alpha[i] = a;
+    if (delta_out) delta_out[0] = delta;
+    return ORACLE_OK;
+  }
+  {
+    int status = ORACLE_OK;
+    for (m = 0; m < M; m++) {
+      for (g = 0; g < ng; g++) {
+        const int j0 = g * G, j1 = j0 + G < Kred ? j0 + G : Kred;
+        double sa = 0.0, sq = 0.0, kept = 0.0, delta;
+        int64_t k = 0;
+        int bad = 0;
+        for (j = j0; j < j1; j++) {
+          const float v = w[(size_t)m * Kred + j];
+          if (!isfinite(v)) bad = 1;
+          sa += fabs((double)v);
+          sq += (double)v * (double)v;
+        }
+        if (bad) {
+          alpha[(size_t)m * ng + g] = 0.0f;
+          if (delta_out) delta_out[(size_t)m * ng + g] = 0.0;
+          status = ORACLE_ERR_NONFINITE;
+          continue;
+        }
+        delta = threshold_of(sa, sq, j1 - j0, rule);
+        for (j = j0; j < j1; j++) {
+          const double v = (double)w[(size_t)m * Kred + j];
+          if (fabs(v) > delta) {
+            t[(size_t)m * Kp + j] = v > 0 ? 1 : -1;
+            kept += fabs(v);
+            k++;
+          }
+        }
+        alpha[(size_t)m * ng + g] = k ? (float)(kept / (double)k) : 0.0f;
+        if (delta_out) delta_out[(size_t)m * ng + g] = delta;
+      }
+    }
+    return status;
+  }
+}
+
+/*
+ * Ternary error of each group, err[m][g] = sum_{j in g} (w_j - alpha[m][g] * t_j)^2 in
+ * fp64, element order, over the real weights (Section 3: the element-wise error E).
+ */
+int oracle_ternary_error(const float* w, int M, int Kred, int G, const int8_t* t, const float* alpha,
+                         double* err) {
+  int m, g, j;
+  int ng, Kp;
+  if (M < 0 || Kred < 0 || G < 1) return ORACLE_ERR_ARG;
+  ng = (Kred + G - 1) / G;
+  Kp = ng * G;
+  for (m = 0; m < M; m++)
+    for (g = 0; g < ng; g++) {
+      const int j0 = g * G, j1 = j0 + G < Kred ? j0 + G : Kred;
+      const double a = (double)alpha[(size_t)m * ng + g];
+      double e = 0.0;
+      for (j = j0; j < j1; j++) {
+        const double d = (double)w[(size_t)m * Kred + j] - a * (double)t[(size_t)m * Kp + j];
+        e += d * d;
+      }
+      err[(size_t)m * ng + g] = e;
+    }
   return ORACLE_OK;
 }
