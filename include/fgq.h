@@ -149,6 +149,51 @@ fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float s
 fgq_status fgq_quantize_act_noalloc(const float* x, size_t n, fgq_act_type type, float scale_in,
                                     void* q, float* scale_out, cudaStream_t stream);
 
+/* Threshold rules of fgq_ternarize_threshold. */
+typedef enum { FGQ_RULE_EXP = 0, FGQ_RULE_GAUSS = 1 } fgq_threshold_rule;
+
+/*
+ * Ternarization at an analytical threshold instead of the exact search (Section 3:
+ * t_j = sign(w_j) where |w_j| > Delta, else 0; Lemma 1 and its proof in the appendix).
+ *   rule FGQ_RULE_EXP    Delta = mean |w| (Lemma 1: exponential magnitudes);
+ *   rule FGQ_RULE_GAUSS  Delta = 0.6120031809624808 * rms(w) (Gaussian weights: rms is the
+ *                        maximum-likelihood sigma the paper names; the constant is the z
+ *                        maximising phi(z)^2 / (1 - Phi(z)), the Gaussian limit of the
+ *                        threshold objective (sum of kept |w|)^2 / (number kept)).
+ *   per_layer = 0        one Delta and one alpha per group of G;
+ *   per_layer = 1        one Delta and one alpha for the whole M x Kred matrix (alpha
+ *                        written to every entry): the one-scaling-factor-per-layer baseline.
+ * alpha = fp32(mean of the kept |w|), 0 when nothing is kept.  The statistics cover the
+ * real weights only (a row's zero padding is not counted).  Per group they are fp64 sums
+ * in element order with explicitly rounded operations, so results are bit-reproducible;
+ * per layer the sums run in a fixed tree order (deterministic, a few ulps from a
+ * sequential sum).  codes and alpha layouts as fgq_ternarize (codes fully written).
+ *   workspace  per_layer = 1: device scratch of fgq_ternarize_threshold_workspace_bytes()
+ *              bytes, 16-byte aligned; ignored (may be NULL) when per_layer = 0.
+ *   delta_out  per_layer = 1: device fp64 [1] receiving Delta (may be NULL); ignored
+ *              otherwise.
+ * A group (per_layer = 0) or layer (per_layer = 1) holding NaN/Inf gets zero codes and
+ * alpha, and FGQ_ERR_NONFINITE is recorded.
+ * Errors: as fgq_ternarize; FGQ_ERR_ARG for a bad rule or a missing or short workspace.
+ */
+size_t fgq_ternarize_threshold_workspace_bytes(void);
+fgq_status fgq_ternarize_threshold(const float* w, int M, int Kred, int G, int rule, int per_layer,
+                                   uint32_t* codes, float* alpha, void* workspace,
+                                   size_t workspace_bytes, double* delta_out, cudaStream_t stream);
+
+/*
+ * Ternary error of each group (Section 3: the element-wise error ||W - alpha What||^2
+ * restricted to the group):
+ *   err[m][g] = sum_{j in g, j < Kred} (w[m][j] - alpha[m][g] * t[m][j])^2,
+ * fp64, accumulated in element order with explicitly rounded operations.  codes and alpha
+ * as from fgq_ternarize or fgq_ternarize_threshold for (M, Kred, G); err device fp64
+ * [M][fgq_num_groups(Kred, G)].
+ * Errors: FGQ_ERR_ARG, FGQ_ERR_ALIGN (w, codes, alpha not 4-byte aligned, err not 8-byte
+ * aligned), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_ternary_error(const float* w, int M, int Kred, int G, const uint32_t* codes,
+                             const float* alpha, double* err, cudaStream_t stream);
+
 /*
  * 8-bit weights for the first layer (Section 4: the first layer is kept at 8w-8a): each
  * filter row of w fp32 [M][Kred] is quantized as a signed 8-bit DFP vector, the same rule

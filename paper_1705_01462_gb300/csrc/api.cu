@@ -143,6 +143,34 @@ fgq_status fgq_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes
   return launch_ternarize(w, M, Kred, G, codes, alpha, device_error_word(), stream);
 }
 
+size_t fgq_ternarize_threshold_workspace_bytes(void) { return threshold_workspace_bytes(); }
+
+fgq_status fgq_ternarize_threshold(const float* w, int M, int Kred, int G, int rule, int per_layer, uint32_t* codes,
+                                   float* alpha, void* workspace, size_t workspace_bytes, double* delta_out,
+                                   cudaStream_t stream) {
+  if (M < 0 || Kred < 0 || !valid_G(G) || (rule != FGQ_RULE_EXP && rule != FGQ_RULE_GAUSS)) return FGQ_ERR_ARG;
+  if ((int64_t)M * Kred == 0) return FGQ_OK;
+  if (!w || !codes || !alpha) return FGQ_ERR_ARG;
+  if (!aligned(w, 4) || !aligned(codes, 4) || !aligned(alpha, 4)) return FGQ_ERR_ALIGN;
+  if ((int64_t)Kred + G > INT32_MAX) return FGQ_ERR_ARG;
+  if (per_layer) {
+    if (!workspace || workspace_bytes < threshold_workspace_bytes()) return FGQ_ERR_ARG;
+    if (!aligned(workspace, 16) || (delta_out && !aligned(delta_out, 8))) return FGQ_ERR_ALIGN;
+  }
+  return launch_ternarize_threshold(w, M, Kred, G, rule, per_layer ? 1 : 0, codes, alpha, workspace,
+                                    per_layer ? delta_out : nullptr, device_error_word(), stream);
+}
+
+fgq_status fgq_ternary_error(const float* w, int M, int Kred, int G, const uint32_t* codes, const float* alpha,
+                             double* err, cudaStream_t stream) {
+  if (M < 0 || Kred < 0 || !valid_G(G)) return FGQ_ERR_ARG;
+  if ((int64_t)M * Kred == 0) return FGQ_OK;
+  if (!w || !codes || !alpha || !err) return FGQ_ERR_ARG;
+  if (!aligned(w, 4) || !aligned(codes, 4) || !aligned(alpha, 4) || !aligned(err, 8)) return FGQ_ERR_ALIGN;
+  if ((int64_t)Kred + G > INT32_MAX) return FGQ_ERR_ARG;
+  return launch_ternary_error(w, M, Kred, G, codes, alpha, err, stream);
+}
+
 size_t fgq_quantize_act_workspace_bytes(size_t n) { return quantize_workspace_bytes(n); }
 
 fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float scale_in, void* q,

@@ -33,6 +33,12 @@ fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* co
 fgq_status launch_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
                                       unsigned int* err, cudaStream_t s);
 size_t quantize_workspace_bytes(size_t n);
+size_t threshold_workspace_bytes();
+fgq_status launch_ternarize_threshold(const float* w, int M, int Kred, int G, int rule, int per_layer,
+                                      uint32_t* codes, float* alpha, void* ws, double* delta_out, unsigned int* err,
+                                      cudaStream_t s);
+fgq_status launch_ternary_error(const float* w, int M, int Kred, int G, const uint32_t* codes, const float* alpha,
+                                double* errv, cudaStream_t s);
 fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool derive, void* q,
                            float* scale_out, uint32_t* partials, unsigned int* err, cudaStream_t s);
 

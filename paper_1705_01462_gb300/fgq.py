@@ -32,6 +32,9 @@ SIGNATURES = [
     ("fgq_codes_words_per_row", _i64, [_i, _i]),
     ("fgq_num_groups", _i64, [_i, _i]),
     ("fgq_ternarize", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_ternarize_threshold_workspace_bytes", _sz, []),
+    ("fgq_ternarize_threshold", _i, [_vp, _i, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp, _vp]),
+    ("fgq_ternary_error", _i, [_vp, _i, _i, _i, _vp, _vp, _vp, _vp]),
     ("fgq_quantize_act_workspace_bytes", _sz, [_sz]),
     ("fgq_quantize_act", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp, _sz, _vp]),
     ("fgq_quantize_act_noalloc", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp]),
@@ -136,6 +139,40 @@ def fgq_ternarize(w: torch.Tensor, G: int, codes: Optional[torch.Tensor] = None,
     _check(lib().fgq_ternarize(_dev(w, torch.float32, "w"), M, Kred, G, _dev(codes, torch.int32, "codes"),
                                _dev(alpha, torch.float32, "alpha"), _stream(stream)), "fgq_ternarize")
     return codes, alpha
+
+
+RULE_EXP, RULE_GAUSS = 0, 1
+
+
+def fgq_ternarize_threshold(w: torch.Tensor, G: int, rule: int, per_layer: bool = False, stream=None):
+    """Analytical-threshold ternarization: w fp32 [M][Kred] -> (codes, alpha, delta); delta is a
+    device fp64 [1] tensor for per_layer, else None."""
+    _require_cuda()
+    M, Kred = w.shape
+    codes = torch.empty((M, codes_words_per_row(Kred, G)), dtype=torch.int32, device=w.device)
+    alpha = torch.empty((M, num_groups(Kred, G)), dtype=torch.float32, device=w.device)
+    ws, wsb, delta = None, 0, None
+    if per_layer:
+        wsb = lib().fgq_ternarize_threshold_workspace_bytes()
+        ws = torch.empty(wsb, dtype=torch.uint8, device=w.device)
+        delta = torch.empty(1, dtype=torch.float64, device=w.device)
+    _check(lib().fgq_ternarize_threshold(_dev(w, torch.float32, "w"), M, Kred, G, rule, int(per_layer),
+                                         _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"),
+                                         ws.data_ptr() if ws is not None else None, wsb,
+                                         delta.data_ptr() if delta is not None else None, _stream(stream)),
+           "fgq_ternarize_threshold")
+    return codes, alpha, delta
+
+
+def fgq_ternary_error(w: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, G: int, stream=None) -> torch.Tensor:
+    """Per-group ||w - alpha t||^2, device fp64 [M][ng]."""
+    _require_cuda()
+    M, Kred = w.shape
+    err = torch.empty((M, num_groups(Kred, G)), dtype=torch.float64, device=w.device)
+    _check(lib().fgq_ternary_error(_dev(w, torch.float32, "w"), M, Kred, G, _dev(codes, torch.int32, "codes"),
+                                   _dev(alpha, torch.float32, "alpha"), err.data_ptr(), _stream(stream)),
+           "fgq_ternary_error")
+    return err
 
 
 def fgq_quantize_act(x: torch.Tensor, act_type="u8", scale_in: float = 0.0, q: Optional[torch.Tensor] = None,
