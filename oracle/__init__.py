@@ -70,6 +70,7 @@ def lib() -> ctypes.CDLL:
         L.oracle_ternarize_threshold.argtypes = [_P(c_f), c_i, c_i, c_i, c_i, c_i, _P(ctypes.c_int8), _P(c_f),
                                                  ctypes.c_void_p]
         L.oracle_ternary_error.argtypes = [_P(c_f), c_i, c_i, c_i, _P(ctypes.c_int8), _P(c_f), _P(c_d)]
+        L.oracle_quantize_alpha.argtypes = [_P(c_f), c_i, c_i, c_i, _P(ctypes.c_int32), _P(c_f)]
         L.oracle_group_sums.argtypes = [_P(ctypes.c_int32), c_i, c_i, _P(ctypes.c_int8), c_i, c_i,
                                         _P(ctypes.c_int64)]
         _lib = L
@@ -167,6 +168,33 @@ def ternary_error(w: np.ndarray, t: np.ndarray, alpha: np.ndarray, G: int) -> np
     _check(lib().oracle_ternary_error(_ptr(w, ctypes.c_float), M, Kred, G, _ptr(t, ctypes.c_int8),
                                       _ptr(alpha, ctypes.c_float), _ptr(err, ctypes.c_double)), "ternary_error")
     return err
+
+
+def quantize_alpha(alpha: np.ndarray, bits: int, check: bool = True):
+    """Fixed-point alphas (Section 4): alpha fp32 [M][ng] -> (a int32 [M][ng], scale fp32 [M], status)."""
+    alpha = np.ascontiguousarray(alpha, dtype=np.float32)
+    M, ng = alpha.shape
+    a = np.zeros((M, ng), dtype=np.int32)
+    scale = np.zeros(M, dtype=np.float32)
+    st = lib().oracle_quantize_alpha(_ptr(alpha, ctypes.c_float), M, ng, bits, _ptr(a, ctypes.c_int32),
+                                     _ptr(scale, ctypes.c_float))
+    if check:
+        _check(st, "quantize_alpha")
+    return a, scale, st
+
+
+def dequantize_alpha(a: np.ndarray, scale: np.ndarray) -> np.ndarray:
+    """alpha' = a * 2^E per row (exact in fp32)."""
+    return (a.astype(np.float32) * scale.astype(np.float32)[:, None]).astype(np.float32)
+
+
+def pack_alpha4(a: np.ndarray) -> np.ndarray:
+    """4-bit alphas two per byte along each row (element 2i in the low nibble)."""
+    M, ng = a.shape
+    out = np.zeros((M, (ng + 1) // 2), dtype=np.uint8)
+    for g in range(ng):
+        out[:, g // 2] |= (a[:, g].astype(np.uint8) & 0xf) << (4 * (g % 2))
+    return out
 
 
 def pack_codes(t: np.ndarray) -> np.ndarray:

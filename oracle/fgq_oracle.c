@@ -27,6 +27,8 @@
  *   oracle_ternarize_threshold  ternarization at an analytical threshold (Section 3, Lemma 1),
  *                               per group or with one threshold and one alpha per layer
  *   oracle_ternary_error        per-group ternary error ||w - alpha t||^2 (Section 3)
+ *   oracle_quantize_alpha       8/4-bit fixed-point alphas, one DFP exponent per filter
+ *                               (Section 4)
  *
  * Readings of the paper that this file fixes (where the paper is silent):
  *   - Ties between candidate thresholds with exactly equal objective are broken towards
@@ -687,4 +689,29 @@ int oracle_ternary_error(const float* w, int M, int Kred, int G, const int8_t* t
       err[(size_t)m * ng + g] = e;
     }
   return ORACLE_OK;
+}
+
+/*
+ * Fixed-point scaling factors (Section 4: the alphas of the groups are quantized to 8/4-bit
+ * fixed point).  Reading (the paper does not say how the exponent is shared): the ng
+ * alphas of one filter row share one DFP exponent, and the rule is oracle_quantize's with
+ * the unsigned 8-bit (bits = 8) or 4-bit (bits = 4) type, since alpha >= 0:
+ *   a[m][g] = clamp(round_half_even(alpha[m][g] * 2^-E_m), 0, 2^bits - 1), scale[m] = 2^E_m.
+ * The contraction then uses alpha' = a * 2^E_m (exact in fp32).  a holds one int32 per
+ * value (unpacked).
+ */
+int oracle_quantize_alpha(const float* alpha, int M, int ng, int bits, int32_t* a, float* scale) {
+  int m, st = ORACLE_OK;
+  if (M < 0 || ng < 0 || (bits != 8 && bits != 4)) return ORACLE_ERR_ARG;
+  for (m = 0; m < M; m++) {
+    int E;
+    const int r = oracle_quantize(alpha + (size_t)m * ng, (size_t)ng, bits == 8 ? ORACLE_U8 : ORACLE_U4, 0.0f,
+                                  a + (size_t)m * ng, scale + m, &E);
+    if (r != ORACLE_OK) {
+      memset(a + (size_t)m * ng, 0, sizeof(int32_t) * (size_t)ng);
+      scale[m] = 0.0f;
+      if (st == ORACLE_OK) st = r;
+    }
+  }
+  return st;
 }
