@@ -65,13 +65,16 @@ typedef enum { FGQ_U8 = 0, FGQ_S8 = 1, FGQ_U4 = 2, FGQ_S4 = 3 } fgq_act_type;
 
 /* Contraction kernel families (see fgq_set_path / fgq_last_path). */
 typedef enum {
-  FGQ_PATH_AUTO = 0,   /* choose per shape: the tensor cores where the shape is covered
-                          (G = 4 only with at least 128 filters per conv group), else the
-                          CUDA cores */
+  FGQ_PATH_AUTO = 0,   /* choose per shape: the few-row path for small GEMMs, else the
+                          tensor cores where the shape is covered (G = 4 only with at least
+                          128 filters per conv group), else the CUDA cores */
   FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
-  FGQ_PATH_TC = 2      /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
+  FGQ_PATH_TC = 2,     /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
                           the group; G = 4 with a block-diagonal activation operand
                           (Cg a multiple of 64) */
+  FGQ_PATH_GEMV = 3    /* few-row path for GEMMs with P <= 8 (8-bit activations, Kred a
+                          multiple of 16, G >= 4): one warp per filter row streams the
+                          weights once; the automatic choice for such calls */
 } fgq_path;
 
 /* ABI version of this header (incremented on any signature change). */
@@ -239,6 +242,41 @@ fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale
                       int W, int C, int R, int S, int stride, int pad, int groups,
                       const uint32_t* codes, const float* alpha, int M, int G, float* out,
                       cudaStream_t stream);
+
+/*
+ * Fixed-point scaling factors (Section 4: the alphas are quantized to 8/4-bit fixed point).
+ * The ng alphas of each filter row share one DFP exponent (this library's reading; the
+ * paper does not say how the exponent is shared), chosen by fgq_quantize_act's rule for
+ * the unsigned type of that width (alphas are >= 0):
+ *   aq[m][g] = clamp(round_half_even(alpha[m][g] * 2^-E_m), 0, 2^bits - 1),
+ *   ascale[m] = 2^E_m, E_m the smallest integer with max_g alpha[m][g] * 2^-E_m <= 2^bits - 1.
+ *   alpha   fp32 [M][ng] (as from fgq_ternarize).
+ *   bits    8 (aq: one byte per alpha, [M][ng]) or 4 (aq: two per byte along the row,
+ *           element 2i in the low nibble, [M][ceil(ng/2)]).
+ *   ascale  out, fp32 [M].
+ * A row holding NaN/Inf gets zero codes and scale 0 and records FGQ_ERR_NONFINITE.
+ * Errors: FGQ_ERR_ARG, FGQ_ERR_ALIGN (alpha, ascale not 4-byte aligned), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8_t* aq, float* ascale,
+                              cudaStream_t stream);
+
+/*
+ * fgq_gemm and fgq_conv2d with fixed-point alphas (aq, abits, ascale as produced by
+ * fgq_quantize_alpha): the same contraction with alpha'[m][g] = aq[m][g] * ascale[m] (exact
+ * in fp32).  On the few-row path (P <= 8, see FGQ_PATH_GEMV) the weights stream as 2-bit
+ * codes plus 1 (or 1/2) byte per group instead of 4, and sum_g aq * s is accumulated
+ * exactly in 64-bit integers: y = act_scale * ascale[m] * sum, rounded once.  On the other
+ * paths the alphas are expanded to fp32 in a temporary from the library's stream-ordered
+ * pool (2-bit codes stay as they are).  Tolerance as fgq_gemm with alpha'; errors as
+ * fgq_gemm / fgq_conv2d, FGQ_ERR_ARG for abits not 8 or 4.
+ */
+fgq_status fgq_gemm_qa(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                       const uint32_t* codes, const uint8_t* aq, int abits, const float* ascale, int M,
+                       int G, float* y, cudaStream_t stream);
+fgq_status fgq_conv2d_qa(const void* act, fgq_act_type type, const float* act_scale, int B, int H,
+                         int W, int C, int R, int S, int stride, int pad, int groups,
+                         const uint32_t* codes, const uint8_t* aq, int abits, const float* ascale,
+                         int M, int G, float* out, cudaStream_t stream);
 
 /*
  * Dense 8-bit-weight convolution for the first layer (8w-8a, Section 4):

@@ -56,11 +56,15 @@ fgq_status make_geom(int type, int B, int H, int W, int C, int R, int S, int str
 
 bool tc_any(const Geom& g) { return g.G == 4 ? tc4_supports(g) : tc_supports(g); }
 
+bool gemv_any(const Geom& g) { return !g.is_conv && gemv_supports((int)g.P, g.Kred, g.G, g.act_type); }
+
 int choose_path(const Geom& g, bool sums) {
   const int forced = g_path.load();
   if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
   if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
+  if (forced == FGQ_PATH_GEMV) return gemv_any(g) ? FGQ_PATH_GEMV : -1;
+  if (gemv_any(g)) return FGQ_PATH_GEMV;  // a few activation rows: stream the weights once
   // automatic choice: the tensor cores where the shape is covered, except G = 4 layers with
   // fewer than 128 filters per conv group, where the 128-row MMA tile would leave half its
   // rows idle and the dp4a kernel is faster
@@ -68,21 +72,68 @@ int choose_path(const Geom& g, bool sums) {
   return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
 }
 
+// Fixed-point alphas of a contraction call (nullptr: fp32 alphas).
+struct QAlpha {
+  const uint8_t* aq;
+  int bits;
+  const float* ascale;
+};
+
 fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
-                    const float* act_scale, float* out, int32_t* sums, cudaStream_t s) {
+                    const float* act_scale, float* out, int32_t* sums, cudaStream_t s, const QAlpha* qa = nullptr) {
   if (g.P == 0 || g.M == 0) return FGQ_OK;
   const int path = choose_path(g, sums != nullptr);
   if (path < 0) return FGQ_ERR_UNSUPPORTED;
   t_last_path = path;
   unsigned int* err = device_error_word();
-  if (path == FGQ_PATH_TC) {
-    if (g.G == 4) return launch_tc4_contract(act, g, codes, alpha, act_scale, out, err, s);
-    return launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
+  if (path == FGQ_PATH_GEMV)
+    return launch_gemv(act, g.act_type, (int)g.P, g.Kred, g.M, g.G, codes, alpha, qa ? qa->aq : nullptr,
+                       qa ? qa->bits : 0, qa ? qa->ascale : nullptr, act_scale, out, s);
+  float* a32 = nullptr;  // fixed-point alphas on the fp32-alpha kernels: alpha' = a 2^E, exact
+  if (qa) {
+    cudaMemPool_t pool = scratch_pool();
+    if (!pool || cudaMallocFromPoolAsync(reinterpret_cast<void**>(&a32), sizeof(float) * (size_t)g.M * g.ng, pool, s) !=
+                     cudaSuccess)
+      return FGQ_ERR_CUDA;
+    fgq_status st = launch_dequantize_alpha(qa->aq, qa->bits, g.M, g.ng, qa->ascale, a32, s);
+    if (st != FGQ_OK) {
+      cudaFreeAsync(a32, s);
+      return st;
+    }
+    alpha = a32;
   }
-  return launch_simt_contract(act, g, codes, alpha, 0, act_scale, out, sums, s);
+  fgq_status st;
+  if (path == FGQ_PATH_TC)
+    st = g.G == 4 ? launch_tc4_contract(act, g, codes, alpha, act_scale, out, err, s)
+                  : launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
+  else
+    st = launch_simt_contract(act, g, codes, alpha, 0, act_scale, out, sums, s);
+  if (a32 && cudaFreeAsync(a32, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  return st;
 }
 
 }  // namespace
+
+cudaMemPool_t scratch_pool() {
+  static std::mutex mu;
+  static cudaMemPool_t pools[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!pools[dev]) {
+    cudaMemPoolProps props;
+    memset(&props, 0, sizeof props);
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    cudaMemPool_t p = nullptr;
+    if (cudaMemPoolCreate(&p, &props) != cudaSuccess) return nullptr;
+    uint64_t keep = ~0ull;
+    cudaMemPoolSetAttribute(p, cudaMemPoolAttrReleaseThreshold, &keep);
+    pools[dev] = p;
+  }
+  return pools[dev];
+}
 
 unsigned int* device_error_word() {
   int dev = 0;
@@ -240,6 +291,47 @@ fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale
   return contract(act, g, codes, alpha, act_scale, out, nullptr, stream);
 }
 
+fgq_status fgq_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8_t* aq, float* ascale,
+                              cudaStream_t stream) {
+  if (M < 0 || ng < 0 || (bits != 8 && bits != 4)) return FGQ_ERR_ARG;
+  if ((int64_t)M * ng == 0) return FGQ_OK;
+  if (!alpha || !aq || !ascale) return FGQ_ERR_ARG;
+  if (!aligned(alpha, 4) || !aligned(ascale, 4)) return FGQ_ERR_ALIGN;
+  return launch_quantize_alpha(alpha, M, ng, bits, aq, ascale, device_error_word(), stream);
+}
+
+fgq_status fgq_gemm_qa(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                       const uint32_t* codes, const uint8_t* aq, int abits, const float* ascale, int M, int G,
+                       float* y, cudaStream_t stream) {
+  if (!valid_G(G) || P < 0 || Kred <= 0 || M < 0 || (abits != 8 && abits != 4)) return FGQ_ERR_ARG;
+  if (is4(type) && Kred % 2) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, P, 1, 1, Kred, 1, 1, 1, 0, 1, M, G, 0, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!q || !act_scale || !codes || !aq || !ascale || !y) return FGQ_ERR_ARG;
+  if (!aligned(q, 16) || !aligned(codes, 16) || !aligned(y, 16) || !aligned(act_scale, 4) || !aligned(ascale, 4))
+    return FGQ_ERR_ALIGN;
+  const QAlpha qa{aq, abits, ascale};
+  return contract(q, g, codes, nullptr, act_scale, y, nullptr, stream, &qa);
+}
+
+fgq_status fgq_conv2d_qa(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
+                         int R, int S, int stride, int pad, int groups, const uint32_t* codes, const uint8_t* aq,
+                         int abits, const float* ascale, int M, int G, float* out, cudaStream_t stream) {
+  if (!valid_G(G) || (abits != 8 && abits != 4)) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !act_scale || !codes || !aq || !ascale || !out) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(codes, 16) || !aligned(out, 16) || !aligned(act_scale, 4) ||
+      !aligned(ascale, 4))
+    return FGQ_ERR_ALIGN;
+  const QAlpha qa{aq, abits, ascale};
+  return contract(act, g, codes, nullptr, act_scale, out, nullptr, stream, &qa);
+}
+
 fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
                          int R, int S, int stride, int pad, int groups, const int8_t* wq, const float* wscale,
                          int M, float* out, cudaStream_t stream) {
@@ -281,7 +373,7 @@ fgq_status fgq_stream_status(cudaStream_t stream) {
 }
 
 int fgq_set_path(int path) {
-  if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC) return -1;
+  if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC && path != FGQ_PATH_GEMV) return -1;
   return g_path.exchange(path);
 }
 

@@ -62,4 +62,21 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
 
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
 
+// Stream-ordered memory pool of the current device for per-call temporaries (it keeps
+// freed blocks: no release threshold).  nullptr if it cannot be created.
+cudaMemPool_t scratch_pool();
+
+// Fixed-point alphas (8- or 4-bit codes, one scale 2^E per filter row).
+fgq_status launch_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8_t* aq, float* ascale,
+                                 unsigned int* err, cudaStream_t s);
+fgq_status launch_dequantize_alpha(const uint8_t* aq, int bits, int M, int ng, const float* ascale, float* alpha,
+                                   cudaStream_t s);
+
+// Few-row contraction (P <= 8, 8-bit activations, Kred % 16 == 0, G >= 4); alphas fp32
+// (abits = 0) or fixed point (abits 8 or 4 with aq, ascale).
+bool gemv_supports(int P, int Kred, int G, int act_type);
+fgq_status launch_gemv(const void* q, int act_type, int P, int Kred, int M, int G, const uint32_t* codes,
+                       const float* alpha, const uint8_t* aq, int abits, const float* ascale, const float* act_scale,
+                       float* y, cudaStream_t s);
+
 }  // namespace fgq

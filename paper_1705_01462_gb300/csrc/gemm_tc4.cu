@@ -36,7 +36,6 @@
 // in-flight copies and MMAs are waited for, and TMEM is freed.
 #include <cstdint>
 #include <cstring>
-#include <mutex>
 
 #include "tc_common.cuh"
 
@@ -487,29 +486,6 @@ fgq_status launch_tc4_path(const T4Args& args, int grid, cudaStream_t s) {
   return args.act_tma ? launch_tc4<ABITS, SIGNED, true>(args, grid, s) : launch_tc4<ABITS, SIGNED, false>(args, grid, s);
 }
 
-// Stream-ordered memory pool of the current device for the expanded-code temporaries; it
-// keeps freed blocks (no release threshold), so steady-state calls do not reach the OS.
-cudaMemPool_t a16_pool() {
-  static std::mutex mu;
-  static cudaMemPool_t pools[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  std::lock_guard<std::mutex> lk(mu);
-  if (!pools[dev]) {
-    cudaMemPoolProps props;
-    memset(&props, 0, sizeof props);
-    props.allocType = cudaMemAllocationTypePinned;
-    props.location.type = cudaMemLocationTypeDevice;
-    props.location.id = dev;
-    cudaMemPool_t p = nullptr;
-    if (cudaMemPoolCreate(&p, &props) != cudaSuccess) return nullptr;
-    uint64_t keep = ~0ull;
-    cudaMemPoolSetAttribute(p, cudaMemPoolAttrReleaseThreshold, &keep);
-    pools[dev] = p;
-  }
-  return pools[dev];
-}
-
 }  // namespace
 
 bool tc4_supports(const Geom& g) {
@@ -540,7 +516,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
 
   // expanded codes: fp16 [M][Kp] (Kp = 16 wrow), in a temporary from the stream-ordered pool
-  cudaMemPool_t pool = a16_pool();
+  cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
   const int64_t nwords = (int64_t)g.M * g.wrow;
   void* a16 = nullptr;

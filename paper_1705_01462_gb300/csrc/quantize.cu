@@ -196,6 +196,91 @@ int max_blocks(size_t n) {
 
 }  // namespace
 
+namespace {
+
+// Fixed-point alphas (Section 4): one warp per filter row; the row's DFP exponent from its
+// maximum (the activation quantizer's rule, unsigned 8- or 4-bit), then the codes (4-bit:
+// two per byte, element 2i in the low nibble) and the row scale 2^E.  A row holding
+// NaN/Inf gets zero codes and scale 0 and records FGQ_ERR_NONFINITE.
+template <int TYPE>
+__global__ void __launch_bounds__(256) quantize_alpha_kernel(const float* __restrict__ alpha, int M, int ng,
+                                                            uint8_t* __restrict__ aq, float* __restrict__ ascale,
+                                                            unsigned int* err) {
+  using T = QTraits<TYPE>;
+  const int m = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float* row = alpha + (int64_t)m * ng;
+  uint32_t mx = 0;
+  bool bad = false;
+  for (int g = lane; g < ng; g += 32) {
+    const float v = __ldg(row + g);
+    bad |= (__float_as_uint(v) & 0x7fffffffu) >= 0x7f800000u;
+    mx = max(mx, mag_bits(v, true));
+  }
+  mx = __reduce_max_sync(FULL_MASK, mx);
+  bad = __any_sync(FULL_MASK, bad);
+  const int rb = T::bits == 8 ? ng : (ng + 1) / 2;  // code bytes per row
+  uint8_t* out = aq + (int64_t)m * rb;
+  if (bad) {
+    if (lane == 0) {
+      record_error(err, FGQ_ERR_NONFINITE);
+      ascale[m] = 0.0f;
+    }
+    for (int i = lane; i < rb; i += 32) out[i] = 0;
+    return;
+  }
+  const int E = dfp_exponent(mx, T::qmax);
+  const float mul1 = (-E <= 127) ? pow2f(-E) : pow2f(64);
+  const float mul2 = (-E <= 127) ? 1.0f : pow2f(-E - 64);
+  if (lane == 0) ascale[m] = pow2f(E);
+  for (int i = lane; i < rb; i += 32) {
+    if (T::bits == 8) {
+      out[i] = (uint8_t)qcode<TYPE>(__ldg(row + i), mul1, mul2);
+    } else {
+      const uint32_t lo = qcode<TYPE>(__ldg(row + 2 * i), mul1, mul2);
+      const uint32_t hi = 2 * i + 1 < ng ? qcode<TYPE>(__ldg(row + 2 * i + 1), mul1, mul2) : 0u;
+      out[i] = (uint8_t)(lo | (hi << 4));
+    }
+  }
+}
+
+// alpha' = a * scale per row (exact in fp32), for the paths that take fp32 alphas.
+__global__ void __launch_bounds__(256) dequantize_alpha_kernel(const uint8_t* __restrict__ aq, int bits, int M, int ng,
+                                                              const float* __restrict__ ascale,
+                                                              float* __restrict__ alpha) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)M * ng) return;
+  const int m = (int)(i / ng), g = (int)(i - (int64_t)m * ng);
+  uint32_t a;
+  if (bits == 8) {
+    a = __ldg(aq + i);
+  } else {
+    const uint8_t b = __ldg(aq + (int64_t)m * ((ng + 1) / 2) + g / 2);
+    a = (g & 1) ? (b >> 4) : (b & 0xfu);
+  }
+  alpha[i] = (float)a * __ldg(ascale + m);
+}
+
+}  // namespace
+
+fgq_status launch_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8_t* aq, float* ascale,
+                                 unsigned int* err, cudaStream_t s) {
+  const unsigned blocks = (unsigned)((M + 7) / 8);
+  if (bits == 8)
+    quantize_alpha_kernel<FGQ_U8><<<blocks, 256, 0, s>>>(alpha, M, ng, aq, ascale, err);
+  else
+    quantize_alpha_kernel<FGQ_U4><<<blocks, 256, 0, s>>>(alpha, M, ng, aq, ascale, err);
+  return after_launch();
+}
+
+fgq_status launch_dequantize_alpha(const uint8_t* aq, int bits, int M, int ng, const float* ascale, float* alpha,
+                                   cudaStream_t s) {
+  const int64_t n = (int64_t)M * ng;
+  dequantize_alpha_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(aq, bits, M, ng, ascale, alpha);
+  return after_launch();
+}
+
 size_t quantize_workspace_bytes(size_t n) {
   if (n == 0) return 0;
   return sizeof(uint32_t) * (size_t)max_blocks(n);

@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "libfgq.so")
 
 FGQ_OK, FGQ_ERR_ARG, FGQ_ERR_ALIGN, FGQ_ERR_UNSUPPORTED, FGQ_ERR_NONFINITE, FGQ_ERR_TIMEOUT, FGQ_ERR_CUDA = range(7)
 U8, S8, U4, S4 = 0, 1, 2, 3
-PATH_AUTO, PATH_SIMT, PATH_TC = 0, 1, 2
+PATH_AUTO, PATH_SIMT, PATH_TC, PATH_GEMV = 0, 1, 2, 3
 ACT_TYPES = {"u8": U8, "s8": S8, "u4": U4, "s4": S4}
 
 _lib: Optional[ctypes.CDLL] = None
@@ -42,6 +42,9 @@ SIGNATURES = [
     ("fgq_gemm", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d_w8", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _vp]),
+    ("fgq_quantize_alpha", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_gemm_qa", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
+    ("fgq_conv2d_qa", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_group_sums", _i, [_vp, _i, _i, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_stream_status", _i, [_vp]),
     ("fgq_set_path", _i, [_i]),
@@ -218,6 +221,45 @@ def fgq_gemm(q: torch.Tensor, act_type, act_scale: torch.Tensor, P: int, Kred: i
                           P, Kred, _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
                           _dev(y, torch.float32, "y"), _stream(stream)), "fgq_gemm")
     return y
+
+
+def fgq_quantize_alpha(alpha: torch.Tensor, bits: int, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """Fixed-point alphas: fp32 [M][ng] -> (aq uint8 [M][ng] or [M][ceil(ng/2)], ascale fp32 [M])."""
+    _require_cuda()
+    M, ng = alpha.shape
+    aq = torch.empty((M, ng if bits == 8 else (ng + 1) // 2), dtype=torch.uint8, device=alpha.device)
+    ascale = torch.empty(M, dtype=torch.float32, device=alpha.device)
+    _check(lib().fgq_quantize_alpha(_dev(alpha, torch.float32, "alpha"), M, ng, bits, _dev(aq, torch.uint8, "aq"),
+                                    _dev(ascale, torch.float32, "ascale"), _stream(stream)), "fgq_quantize_alpha")
+    return aq, ascale
+
+
+def fgq_gemm_qa(q: torch.Tensor, act_type, act_scale: torch.Tensor, P: int, Kred: int, codes: torch.Tensor,
+                aq: torch.Tensor, abits: int, ascale: torch.Tensor, M: int, G: int, y: Optional[torch.Tensor] = None,
+                stream=None) -> torch.Tensor:
+    _require_cuda()
+    if y is None:
+        y = torch.empty((P, M), dtype=torch.float32, device=q.device)
+    _check(lib().fgq_gemm_qa(_dev(q, torch.uint8, "q"), _act_type(act_type), _dev(act_scale, torch.float32, "act_scale"),
+                             P, Kred, _dev(codes, torch.int32, "codes"), _dev(aq, torch.uint8, "aq"), abits,
+                             _dev(ascale, torch.float32, "ascale"), M, G, _dev(y, torch.float32, "y"), _stream(stream)),
+           "fgq_gemm_qa")
+    return y
+
+
+def fgq_conv2d_qa(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, H: int, W: int, C: int, R: int,
+                  S: int, stride: int, pad: int, groups: int, codes: torch.Tensor, aq: torch.Tensor, abits: int,
+                  ascale: torch.Tensor, M: int, G: int, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if out is None:
+        out = torch.empty((B, Ho, Wo, M), dtype=torch.float32, device=act.device)
+    _check(lib().fgq_conv2d_qa(_dev(act, torch.uint8, "act"), _act_type(act_type),
+                               _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
+                               _dev(codes, torch.int32, "codes"), _dev(aq, torch.uint8, "aq"), abits,
+                               _dev(ascale, torch.float32, "ascale"), M, G, _dev(out, torch.float32, "out"),
+                               _stream(stream)), "fgq_conv2d_qa")
+    return out
 
 
 def conv_out_hw(H, W, R, S, stride, pad):

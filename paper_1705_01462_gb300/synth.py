@@ -152,6 +152,15 @@ def activations(shape, seed: int) -> np.ndarray:
     return np.abs(g.standard_normal(shape, dtype=np.float32)).astype(np.float32)
 
 
+def torch_weights_matrix(M: int, K: int, seed: int, device, fan_in: int | None = None):
+    """Same distribution as `weights_matrix`, drawn on `device` with a seeded torch generator."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    std = float(np.sqrt(2.0 / (fan_in or K)))
+    return torch.randn((M, K), generator=gen, device=device, dtype=torch.float32) * std
+
+
 def torch_weights(layer: ConvLayer, seed: int, device):
     """Same distribution as `weights`, drawn on `device` with a seeded torch generator."""
     import torch
