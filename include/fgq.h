@@ -244,6 +244,28 @@ fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale
                       cudaStream_t stream);
 
 /*
+ * fgq_gemm and fgq_conv2d with the output requantized inside the kernel (Section 4: the
+ * 32-bit outputs are converted to 8 bits and rounded before they are passed to the next
+ * layer): instead of fp32 y the kernels write
+ *   out_q[p][m] = clamp(round_half_even(y[p][m] * 2^-E), qmin, qmax)
+ * of out_type FGQ_U8 (0..255: negative outputs become 0, a fused ReLU) or FGQ_S8
+ * (-128..127), one byte each, for the given output scale out_scale[0] = 2^E (device fp32,
+ * a power of two, e.g. a per-layer DFP scale found on a calibration batch).  y is the fp32
+ * value the fp32-output call returns (same kernel, same rounding), so the codes equal
+ * fgq_quantize_act applied to that output with scale_in = 2^E.  out_q: [P][M] bytes,
+ * 4-byte aligned.  Errors as fgq_gemm / fgq_conv2d; FGQ_ERR_ARG for another out_type.
+ */
+fgq_status fgq_gemm_rq(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                       const uint32_t* codes, const float* alpha, int M, int G,
+                       fgq_act_type out_type, const float* out_scale, void* out_q,
+                       cudaStream_t stream);
+fgq_status fgq_conv2d_rq(const void* act, fgq_act_type type, const float* act_scale, int B, int H,
+                         int W, int C, int R, int S, int stride, int pad, int groups,
+                         const uint32_t* codes, const float* alpha, int M, int G,
+                         fgq_act_type out_type, const float* out_scale, void* out_q,
+                         cudaStream_t stream);
+
+/*
  * Fixed-point scaling factors (Section 4: the alphas are quantized to 8/4-bit fixed point).
  * The ng alphas of each filter row share one DFP exponent (this library's reading; the
  * paper does not say how the exponent is shared), chosen by fgq_quantize_act's rule for

@@ -51,6 +51,9 @@ fgq_status make_geom(int type, int B, int H, int W, int C, int R, int S, int str
   g.act_type = type;
   g.is_conv = is_conv;
   g.P = (int64_t)B * g.Ho * g.Wo;
+  g.rq_out = nullptr;
+  g.rq_scale = nullptr;
+  g.rq_signed = 0;
   return FGQ_OK;
 }
 
@@ -88,7 +91,8 @@ fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const
   unsigned int* err = device_error_word();
   if (path == FGQ_PATH_GEMV)
     return launch_gemv(act, g.act_type, (int)g.P, g.Kred, g.M, g.G, codes, alpha, qa ? qa->aq : nullptr,
-                       qa ? qa->bits : 0, qa ? qa->ascale : nullptr, act_scale, out, s);
+                       qa ? qa->bits : 0, qa ? qa->ascale : nullptr, act_scale, out, g.rq_out, g.rq_scale,
+                       g.rq_signed, s);
   float* a32 = nullptr;  // fixed-point alphas on the fp32-alpha kernels: alpha' = a 2^E, exact
   if (qa) {
     cudaMemPool_t pool = scratch_pool();
@@ -289,6 +293,44 @@ fgq_status fgq_conv2d(const void* act, fgq_act_type type, const float* act_scale
       !aligned(act_scale, 4))
     return FGQ_ERR_ALIGN;
   return contract(act, g, codes, alpha, act_scale, out, nullptr, stream);
+}
+
+fgq_status fgq_gemm_rq(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,
+                       const uint32_t* codes, const float* alpha, int M, int G, fgq_act_type out_type,
+                       const float* out_scale, void* out_q, cudaStream_t stream) {
+  if (!valid_G(G) || P < 0 || Kred <= 0 || M < 0 || (out_type != FGQ_U8 && out_type != FGQ_S8)) return FGQ_ERR_ARG;
+  if (is4(type) && Kred % 2) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, P, 1, 1, Kred, 1, 1, 1, 0, 1, M, G, 0, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!q || !act_scale || !codes || !alpha || !out_scale || !out_q) return FGQ_ERR_ARG;
+  if (!aligned(q, 16) || !aligned(codes, 16) || !aligned(alpha, 16) || !aligned(out_q, 4) ||
+      !aligned(act_scale, 4) || !aligned(out_scale, 4))
+    return FGQ_ERR_ALIGN;
+  g.rq_out = static_cast<uint8_t*>(out_q);
+  g.rq_scale = out_scale;
+  g.rq_signed = out_type == FGQ_S8;
+  return contract(q, g, codes, alpha, act_scale, nullptr, nullptr, stream);
+}
+
+fgq_status fgq_conv2d_rq(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
+                         int R, int S, int stride, int pad, int groups, const uint32_t* codes, const float* alpha,
+                         int M, int G, fgq_act_type out_type, const float* out_scale, void* out_q,
+                         cudaStream_t stream) {
+  if (!valid_G(G) || (out_type != FGQ_U8 && out_type != FGQ_S8)) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !act_scale || !codes || !alpha || !out_scale || !out_q) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(codes, 16) || !aligned(alpha, 16) || !aligned(out_q, 4) ||
+      !aligned(act_scale, 4) || !aligned(out_scale, 4))
+    return FGQ_ERR_ALIGN;
+  g.rq_out = static_cast<uint8_t*>(out_q);
+  g.rq_scale = out_scale;
+  g.rq_signed = out_type == FGQ_S8;
+  return contract(act, g, codes, alpha, act_scale, nullptr, nullptr, stream);
 }
 
 fgq_status fgq_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8_t* aq, float* ascale,

@@ -77,4 +77,27 @@ __host__ __device__ constexpr uint32_t expand_code_byte(uint32_t b) {
   return r;
 }
 
+// Fused output requantization (Section 4: the 32-bit outputs are converted to 8 bits and
+// rounded before they are passed to the next layer): q = clamp(round_half_even(v * 2^-E),
+// qmin, qmax) for the output scale 2^E, the rule of the activation quantizer; the two
+// multipliers keep 2^-E representable for every E in [-149, 127].
+struct RqMul {
+  float m1, m2;
+  int qmin, qmax;
+};
+__device__ __forceinline__ RqMul rq_mul(const float* scale, int is_signed) {
+  const int E = ilogbf(__ldg(scale));
+  RqMul r;
+  r.m1 = (-E <= 127) ? pow2f(-E) : pow2f(64);
+  r.m2 = (-E <= 127) ? 1.0f : pow2f(-E - 64);
+  r.qmin = is_signed ? -128 : 0;
+  r.qmax = is_signed ? 127 : 255;
+  return r;
+}
+__device__ __forceinline__ uint8_t rq_code(float v, const RqMul& r) {
+  int x = __float2int_rn(v * r.m1 * r.m2);
+  x = max(r.qmin, min(r.qmax, x));
+  return (uint8_t)(x & 0xff);
+}
+
 }  // namespace fgq

@@ -18,6 +18,11 @@ struct Geom {
   int act_type;  // fgq_act_type
   int is_conv;
   int64_t P;     // B * Ho * Wo
+  // fused output requantization (nullptr: fp32 output): codes [P][M] of 8-bit type
+  // rq_signed ? FGQ_S8 : FGQ_U8 at the scale *rq_scale = 2^E
+  uint8_t* rq_out;
+  const float* rq_scale;
+  int rq_signed;
 };
 
 // Device error word of the current device (first error wins; cleared by
@@ -77,6 +82,6 @@ fgq_status launch_dequantize_alpha(const uint8_t* aq, int bits, int M, int ng, c
 bool gemv_supports(int P, int Kred, int G, int act_type);
 fgq_status launch_gemv(const void* q, int act_type, int P, int Kred, int M, int G, const uint32_t* codes,
                        const float* alpha, const uint8_t* aq, int abits, const float* ascale, const float* act_scale,
-                       float* y, cudaStream_t s);
+                       float* y, uint8_t* rq_out, const float* rq_scale, int rq_signed, cudaStream_t s);
 
 }  // namespace fgq

@@ -368,6 +368,27 @@ __global__ void __launch_bounds__(NT, FGQ_SIMT_MIN_BLOCKS) simt_contract_kernel(
   const float sx = __ldg(act_scale);
   const int m = mlo + ty * 4;
   const bool vec = (g.M % 4 == 0) && (m + 3 < mhi);
+  if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
+    const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t p = p0 + 64 * (j / 4) + 4 * tx + (j % 4);
+      if (p >= g.P) continue;
+      uint32_t b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        b[i] = rq_code(DW ? sx * __ldg(scales + min(m + i, g.M - 1)) * (float)iacc[i][j] : sx * acc[i][j], r);
+      uint8_t* orow = g.rq_out + p * g.M;
+      if (vec) {
+        *reinterpret_cast<uint32_t*>(orow + m) = b[0] | (b[1] << 8) | (b[2] << 16) | (b[3] << 24);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (m + i < mhi) orow[m + i] = (uint8_t)b[i];
+      }
+    }
+    return;
+  }
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const int64_t p = p0 + 64 * (j / 4) + 4 * tx + (j % 4);
@@ -417,7 +438,12 @@ __global__ void simple_contract_kernel(const uint8_t* __restrict__ act, const Ge
     if (sums) sums[((int64_t)m * g.ng + gg) * g.P + p] = s;
     else acc = fmaf(alpha[(int64_t)m * g.ng + gg], (float)s, acc);
   }
-  if (!sums) out[p * g.M + m] = acc * act_scale[0];
+  if (sums) return;
+  const float v = acc * act_scale[0];
+  if (g.rq_out)
+    g.rq_out[p * g.M + m] = rq_code(v, rq_mul(g.rq_scale, g.rq_signed));
+  else
+    out[p * g.M + m] = v;
 }
 
 template <int G, bool SA, bool DW, bool SUMS>

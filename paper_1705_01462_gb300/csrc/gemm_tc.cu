@@ -458,10 +458,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         }
       } else if (mok) {
         const int64_t pbase = p0 + 64 * half;
+        if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
+          const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
 #pragma unroll
-        for (int j = 0; j < 64; ++j) {
-          const int64_t p = pbase + j;
-          if (p < g.P) a.out[p * g.M + m] = sx * acc[j];
+          for (int j = 0; j < 64; ++j) {
+            const int64_t p = pbase + j;
+            if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sx * acc[j], r);
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 64; ++j) {
+            const int64_t p = pbase + j;
+            if (p < g.P) a.out[p * g.M + m] = sx * acc[j];
+          }
         }
       }
     }
@@ -550,7 +559,7 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                     ? 1
                     : 0;
   }
-  if (a.act_tma && g.groups == 1 && g.M % 4 == 0) {
+  if (a.act_tma && g.groups == 1 && g.M % 4 == 0 && !g.rq_out) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, TC_BM, TC_BN, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1

@@ -450,10 +450,19 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
           bulk_commit();
         }
       } else if (mok) {
+        if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
+          const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int64_t p = p0 + 32 * hsub + i;
-          if (p < g.P) a.out[p * g.M + m] = sx * acc[i];
+          for (int i = 0; i < 32; ++i) {
+            const int64_t p = p0 + 32 * hsub + i;
+            if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sx * acc[i], r);
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int64_t p = p0 + 32 * hsub + i;
+            if (p < g.P) a.out[p * g.M + m] = sx * acc[i];
+          }
         }
       }
     }
@@ -535,7 +544,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
                     ? 1
                     : 0;
   }
-  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0) {
+  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, T4_BM, T4_BP, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1

@@ -45,7 +45,8 @@ __global__ void __launch_bounds__(32 * GV_WARPS) gemv_kernel(const uint8_t* __re
                                                              const uint8_t* __restrict__ aq,
                                                              const float* __restrict__ ascale,
                                                              const float* __restrict__ act_scale,
-                                                             float* __restrict__ y) {
+                                                             float* __restrict__ y, uint8_t* __restrict__ rq_out,
+                                                             const float* __restrict__ rq_scale, int rq_signed) {
   __shared__ uint32_t lut[256];  // byte of 4 codes -> 4 int8 weights
   for (int i = threadIdx.x; i < 256; i += blockDim.x) {
     uint32_t v = 0;
@@ -143,7 +144,10 @@ __global__ void __launch_bounds__(32 * GV_WARPS) gemv_kernel(const uint8_t* __re
   for (int p = 0; p < GV_MAXP; ++p) {
     if (p < P && lane == p) {
       const float v = QA ? (float)iacc[p] * (sx * __ldg(ascale + m)) : sx * acc[p];
-      y[(int64_t)p * M + m] = v;
+      if (rq_out)  // fused requantization
+        rq_out[(int64_t)p * M + m] = rq_code(v, rq_mul(rq_scale, rq_signed));
+      else
+        y[(int64_t)p * M + m] = v;
     }
   }
 }
@@ -151,15 +155,18 @@ __global__ void __launch_bounds__(32 * GV_WARPS) gemv_kernel(const uint8_t* __re
 template <int G, bool SIGNED>
 fgq_status launch_gemv_g(const void* q, int P, int Kred, int M, const uint32_t* codes, const float* alpha,
                          const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* y,
-                         cudaStream_t s) {
+                         uint8_t* rq_out, const float* rq_scale, int rq_signed, cudaStream_t s) {
   const unsigned blocks = (unsigned)((M + GV_WARPS - 1) / GV_WARPS);
   const uint8_t* qb = static_cast<const uint8_t*>(q);
   if (abits == 8)
-    gemv_kernel<G, SIGNED, 8><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y);
+    gemv_kernel<G, SIGNED, 8><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y,
+                                                                 rq_out, rq_scale, rq_signed);
   else if (abits == 4)
-    gemv_kernel<G, SIGNED, 4><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y);
+    gemv_kernel<G, SIGNED, 4><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y,
+                                                                 rq_out, rq_scale, rq_signed);
   else
-    gemv_kernel<G, SIGNED, 0><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y);
+    gemv_kernel<G, SIGNED, 0><<<blocks, 32 * GV_WARPS, 0, s>>>(qb, P, Kred, M, codes, alpha, aq, ascale, act_scale, y,
+                                                                 rq_out, rq_scale, rq_signed);
   return after_launch();
 }
 
@@ -171,13 +178,13 @@ bool gemv_supports(int P, int Kred, int G, int act_type) {
 
 fgq_status launch_gemv(const void* q, int act_type, int P, int Kred, int M, int G, const uint32_t* codes,
                        const float* alpha, const uint8_t* aq, int abits, const float* ascale, const float* act_scale,
-                       float* y, cudaStream_t s) {
+                       float* y, uint8_t* rq_out, const float* rq_scale, int rq_signed, cudaStream_t s) {
   if (!gemv_supports(P, Kred, G, act_type)) return FGQ_ERR_UNSUPPORTED;
   const bool sg = act_type == FGQ_S8;
 #define FGQ_GEMV_CASE(GG)                                                                                   \
   case GG:                                                                                                  \
-    return sg ? launch_gemv_g<GG, true>(q, P, Kred, M, codes, alpha, aq, abits, ascale, act_scale, y, s)    \
-              : launch_gemv_g<GG, false>(q, P, Kred, M, codes, alpha, aq, abits, ascale, act_scale, y, s);
+    return sg ? launch_gemv_g<GG, true>(q, P, Kred, M, codes, alpha, aq, abits, ascale, act_scale, y, rq_out, rq_scale, rq_signed, s)    \
+              : launch_gemv_g<GG, false>(q, P, Kred, M, codes, alpha, aq, abits, ascale, act_scale, y, rq_out, rq_scale, rq_signed, s);
   switch (G) {
     FGQ_GEMV_CASE(4)
     FGQ_GEMV_CASE(8)

@@ -43,6 +43,8 @@ SIGNATURES = [
     ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d_w8", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _vp]),
     ("fgq_quantize_alpha", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_gemm_rq", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_conv2d_rq", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
     ("fgq_gemm_qa", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d_qa", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_group_sums", _i, [_vp, _i, _i, _i, _vp, _i, _i, _vp, _vp]),
@@ -221,6 +223,36 @@ def fgq_gemm(q: torch.Tensor, act_type, act_scale: torch.Tensor, P: int, Kred: i
                           P, Kred, _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
                           _dev(y, torch.float32, "y"), _stream(stream)), "fgq_gemm")
     return y
+
+
+def fgq_gemm_rq(q: torch.Tensor, act_type, act_scale: torch.Tensor, P: int, Kred: int, codes: torch.Tensor,
+                alpha: torch.Tensor, M: int, G: int, out_type, out_scale: torch.Tensor,
+                out_q: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """fgq_gemm with the output requantized in the kernel: uint8 [P][M] codes at out_scale."""
+    _require_cuda()
+    if out_q is None:
+        out_q = torch.empty((P, M), dtype=torch.uint8, device=q.device)
+    _check(lib().fgq_gemm_rq(_dev(q, torch.uint8, "q"), _act_type(act_type), _dev(act_scale, torch.float32, "act_scale"),
+                             P, Kred, _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
+                             _act_type(out_type), _dev(out_scale, torch.float32, "out_scale"),
+                             _dev(out_q, torch.uint8, "out_q"), _stream(stream)), "fgq_gemm_rq")
+    return out_q
+
+
+def fgq_conv2d_rq(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, H: int, W: int, C: int, R: int,
+                  S: int, stride: int, pad: int, groups: int, codes: torch.Tensor, alpha: torch.Tensor, M: int, G: int,
+                  out_type, out_scale: torch.Tensor, out_q: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """fgq_conv2d with the output requantized in the kernel: uint8 NHWC [B][Ho][Wo][M] codes."""
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if out_q is None:
+        out_q = torch.empty((B, Ho, Wo, M), dtype=torch.uint8, device=act.device)
+    _check(lib().fgq_conv2d_rq(_dev(act, torch.uint8, "act"), _act_type(act_type),
+                               _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
+                               _dev(codes, torch.int32, "codes"), _dev(alpha, torch.float32, "alpha"), M, G,
+                               _act_type(out_type), _dev(out_scale, torch.float32, "out_scale"),
+                               _dev(out_q, torch.uint8, "out_q"), _stream(stream)), "fgq_conv2d_rq")
+    return out_q
 
 
 def fgq_quantize_alpha(alpha: torch.Tensor, bits: int, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
