@@ -265,6 +265,34 @@ fgq_status fgq_conv2d_rq(const void* act, fgq_act_type type, const float* act_sc
                          fgq_act_type out_type, const float* out_scale, void* out_q,
                          cudaStream_t stream);
 
+/* fgq_conv2d_w8 (the 8-bit-weight first layer) with the output requantized in the kernel,
+ * as fgq_conv2d_rq. */
+fgq_status fgq_conv2d_w8_rq(const void* act, fgq_act_type type, const float* act_scale, int B, int H,
+                            int W, int C, int R, int S, int stride, int pad, int groups,
+                            const int8_t* wq, const float* wscale, int M, fgq_act_type out_type,
+                            const float* out_scale, void* out_q, cudaStream_t stream);
+
+/*
+ * Max pooling of unsigned 8-bit codes (the pooling after the first layer of the ResNet
+ * forward): out[b][ho][wo][c] = max over the R x R window at stride, padding pad (padded
+ * positions do not take part) of in[b][h][w][c], NHWC, C a multiple of 4, pad < R.  Exact
+ * in the code domain (one shared scale).  in, out 4-byte aligned.
+ */
+fgq_status fgq_maxpool_u8(const uint8_t* in, int B, int H, int W, int C, int R, int stride, int pad,
+                          uint8_t* out, cudaStream_t stream);
+
+/*
+ * Residual addition of two 8-bit code tensors of n elements (the shortcut of a ResNet
+ * block): v = a * a_scale[0] + b * b_scale[0] in fp32 (each product exact, the sum rounded
+ * once).  out != NULL: fp32 v is stored there; otherwise v is requantized to out_q at
+ * out_scale[0] = 2^E as fgq_conv2d_rq does (out_type FGQ_U8: negative sums become 0, the
+ * ReLU after the addition; or FGQ_S8).  a_type, b_type: FGQ_U8 or FGQ_S8.
+ */
+fgq_status fgq_add_codes(const void* a, fgq_act_type a_type, const float* a_scale, const void* b,
+                         fgq_act_type b_type, const float* b_scale, size_t n, float* out,
+                         fgq_act_type out_type, const float* out_scale, void* out_q,
+                         cudaStream_t stream);
+
 /*
  * Fixed-point scaling factors (Section 4: the alphas are quantized to 8/4-bit fixed point).
  * The ng alphas of each filter row share one DFP exponent (this library's reading; the

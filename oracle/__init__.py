@@ -326,3 +326,42 @@ def quantize_weights_w8(w: np.ndarray):
         wq[m] = q.astype(np.int8)
         sc[m] = s
     return wq, sc
+
+
+# --------------------------------------------------------------------------- chained forward steps
+# The steps between the contractions of a quantized ResNet forward (Section 4 keeps the
+# activations between layers as 8-bit dynamic fixed point).  The paper states no rule for
+# them; these are the plain definitions this library follows.
+
+def maxpool_codes(q: np.ndarray, R: int, stride: int, pad: int) -> np.ndarray:
+    """Max pooling of integer codes, NHWC: out[b][ho][wo][c] = max of q[b][h][w][c] over the
+    R x R window at (ho*stride - pad, wo*stride - pad), positions outside the map not taking
+    part.  Written as a loop over the output pixels; each window is a numpy slice."""
+    q = np.asarray(q)
+    B, H, W, C = q.shape
+    Ho, Wo = conv_out_hw(H, W, R, R, stride, pad)
+    out = np.zeros((B, Ho, Wo, C), dtype=q.dtype)
+    for ho in range(Ho):
+        h0, h1 = max(ho * stride - pad, 0), min(ho * stride - pad + R, H)
+        for wo in range(Wo):
+            w0, w1 = max(wo * stride - pad, 0), min(wo * stride - pad + R, W)
+            out[:, ho, wo, :] = q[:, h0:h1, w0:w1, :].max(axis=(1, 2))
+    return out
+
+
+def add_codes(qa: np.ndarray, sa: float, qb: np.ndarray, sb: float) -> np.ndarray:
+    """Residual sum of two code tensors at scales sa, sb as fp32: the exact value
+    qa*sa + qb*sb (fp64 holds it exactly for 8-bit codes and power-of-two scales whose
+    exponents differ by less than 40) rounded once to fp32, to nearest even."""
+    sa, sb = float(sa), float(sb)
+    fa, fb = np.frexp(sa)[1], np.frexp(sb)[1]
+    assert abs(int(fa) - int(fb)) < 40, "scales too far apart for an exact fp64 sum"
+    v = np.asarray(qa, dtype=np.float64) * sa + np.asarray(qb, dtype=np.float64) * sb
+    return v.astype(np.float32)
+
+
+def add_requant(qa, sa, qb, sb, out_type: int, scale_out: float) -> np.ndarray:
+    """add_codes followed by the activation quantizer at the fixed scale scale_out (U8: a
+    negative sum becomes 0, the ReLU after the addition)."""
+    q, _, _, _ = quantize(add_codes(qa, sa, qb, sb), out_type, scale_in=scale_out)
+    return q

@@ -388,6 +388,51 @@ fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_sc
   return launch_simt_contract(act, g, wq, wscale, 1, act_scale, out, nullptr, stream);
 }
 
+fgq_status fgq_conv2d_w8_rq(const void* act, fgq_act_type type, const float* act_scale, int B, int H, int W, int C,
+                            int R, int S, int stride, int pad, int groups, const int8_t* wq, const float* wscale,
+                            int M, fgq_act_type out_type, const float* out_scale, void* out_q, cudaStream_t stream) {
+  if (out_type != FGQ_U8 && out_type != FGQ_S8) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, 4, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !act_scale || !wq || !wscale || !out_scale || !out_q) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(wscale, 4) || !aligned(out_q, 4) || !aligned(act_scale, 4) ||
+      !aligned(out_scale, 4))
+    return FGQ_ERR_ALIGN;
+  g.rq_out = static_cast<uint8_t*>(out_q);
+  g.rq_scale = out_scale;
+  g.rq_signed = out_type == FGQ_S8;
+  t_last_path = FGQ_PATH_SIMT;
+  return launch_simt_contract(act, g, wq, wscale, 1, act_scale, nullptr, nullptr, stream);
+}
+
+fgq_status fgq_maxpool_u8(const uint8_t* in, int B, int H, int W, int C, int R, int stride, int pad, uint8_t* out,
+                          cudaStream_t stream) {
+  if (B < 0 || H <= 0 || W <= 0 || C <= 0 || C % 4 || R <= 0 || stride <= 0 || pad < 0 || pad >= R ||
+      H + 2 * pad < R || W + 2 * pad < R)
+    return FGQ_ERR_ARG;
+  if (B == 0) return FGQ_OK;
+  if (!in || !out) return FGQ_ERR_ARG;
+  if (!aligned(in, 4) || !aligned(out, 4)) return FGQ_ERR_ALIGN;
+  return launch_maxpool_u8(in, B, H, W, C, R, stride, pad, out, stream);
+}
+
+fgq_status fgq_add_codes(const void* a, fgq_act_type a_type, const float* a_scale, const void* b,
+                         fgq_act_type b_type, const float* b_scale, size_t n, float* out, fgq_act_type out_type,
+                         const float* out_scale, void* out_q, cudaStream_t stream) {
+  auto is8 = [](int t) { return t == FGQ_U8 || t == FGQ_S8; };
+  if (!is8(a_type) || !is8(b_type) || (!out && !is8(out_type))) return FGQ_ERR_ARG;
+  if (n == 0) return FGQ_OK;
+  if (!a || !b || !a_scale || !b_scale || (!out && (!out_q || !out_scale))) return FGQ_ERR_ARG;
+  if (!aligned(a_scale, 4) || !aligned(b_scale, 4) || (out && !aligned(out, 4)) ||
+      (!out && !aligned(out_scale, 4)))
+    return FGQ_ERR_ALIGN;
+  return launch_add_codes(static_cast<const uint8_t*>(a), a_type == FGQ_S8, a_scale, static_cast<const uint8_t*>(b),
+                          b_type == FGQ_S8, b_scale, (int64_t)n, out, out ? nullptr : static_cast<uint8_t*>(out_q),
+                          out_scale, out_type == FGQ_S8, stream);
+}
+
 fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred, const uint32_t* codes, int M, int G,
                           int32_t* s, cudaStream_t stream) {
   if (!valid_G(G) || P < 0 || Kred <= 0 || M < 0) return FGQ_ERR_ARG;

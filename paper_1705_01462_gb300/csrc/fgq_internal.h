@@ -67,6 +67,14 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
 
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
 
+// Chained-forward steps: max pooling of u8 codes, residual addition of two 8-bit code
+// tensors (fp32 sum, or requantized when out_q is given).
+fgq_status launch_maxpool_u8(const uint8_t* in, int B, int H, int W, int C, int R, int stride, int pad, uint8_t* out,
+                             cudaStream_t s);
+fgq_status launch_add_codes(const uint8_t* a, int a_signed, const float* a_scale, const uint8_t* b, int b_signed,
+                            const float* b_scale, int64_t n, float* out, uint8_t* out_q, const float* out_scale,
+                            int o_signed, cudaStream_t s);
+
 // Stream-ordered memory pool of the current device for per-call temporaries (it keeps
 // freed blocks: no release threshold).  nullptr if it cannot be created.
 cudaMemPool_t scratch_pool();

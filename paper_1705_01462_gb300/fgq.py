@@ -43,6 +43,9 @@ SIGNATURES = [
     ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d_w8", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _vp]),
     ("fgq_quantize_alpha", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_conv2d_w8_rq", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp, _vp]),
+    ("fgq_maxpool_u8", _i, [_vp] + [_i] * 7 + [_vp, _vp]),
+    ("fgq_add_codes", _i, [_vp, _i, _vp, _vp, _i, _vp, _sz, _vp, _i, _vp, _vp, _vp]),
     ("fgq_gemm_rq", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
     ("fgq_conv2d_rq", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
     ("fgq_gemm_qa", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
@@ -323,6 +326,60 @@ def fgq_conv2d_w8(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, 
                                _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
                                _dev(wq, torch.int8, "wq"), _dev(wscale, torch.float32, "wscale"), M,
                                _dev(out, torch.float32, "out"), _stream(stream)), "fgq_conv2d_w8")
+    return out
+
+
+def fgq_conv2d_w8_rq(act: torch.Tensor, act_type, act_scale: torch.Tensor, B: int, H: int, W: int, C: int, R: int,
+                     S: int, stride: int, pad: int, groups: int, wq: torch.Tensor, wscale: torch.Tensor, M: int,
+                     out_type, out_scale: torch.Tensor, out_q: Optional[torch.Tensor] = None,
+                     stream=None) -> torch.Tensor:
+    """fgq_conv2d_w8 with the output requantized in the kernel: uint8 NHWC [B][Ho][Wo][M] codes."""
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if out_q is None:
+        out_q = torch.empty((B, Ho, Wo, M), dtype=torch.uint8, device=act.device)
+    _check(lib().fgq_conv2d_w8_rq(_dev(act, torch.uint8, "act"), _act_type(act_type),
+                                  _dev(act_scale, torch.float32, "act_scale"), B, H, W, C, R, S, stride, pad, groups,
+                                  _dev(wq, torch.int8, "wq"), _dev(wscale, torch.float32, "wscale"), M,
+                                  _act_type(out_type), _dev(out_scale, torch.float32, "out_scale"),
+                                  _dev(out_q, torch.uint8, "out_q"), _stream(stream)), "fgq_conv2d_w8_rq")
+    return out_q
+
+
+def fgq_maxpool_u8(x: torch.Tensor, B: int, H: int, W: int, C: int, R: int, stride: int, pad: int,
+                   out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """R x R max pooling of unsigned codes, NHWC -> uint8 [B][Ho][Wo][C]."""
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, R, stride, pad)
+    if out is None:
+        out = torch.empty((B, Ho, Wo, C), dtype=torch.uint8, device=x.device)
+    _check(lib().fgq_maxpool_u8(_dev(x, torch.uint8, "x"), B, H, W, C, R, stride, pad, _dev(out, torch.uint8, "out"),
+                                _stream(stream)), "fgq_maxpool_u8")
+    return out
+
+
+def fgq_add_codes(a: torch.Tensor, a_type, a_scale: torch.Tensor, b: torch.Tensor, b_type, b_scale: torch.Tensor,
+                  out_type=None, out_scale: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None,
+                  stream=None) -> torch.Tensor:
+    """a * a_scale + b * b_scale: fp32 (out_type None) or codes requantized at out_scale."""
+    _require_cuda()
+    n = a.numel()
+    if b.numel() != n:
+        raise ValueError("fgq_add_codes: a and b differ in size")
+    if out_type is None:
+        if out is None:
+            out = torch.empty(a.shape, dtype=torch.float32, device=a.device)
+        st = lib().fgq_add_codes(_dev(a, torch.uint8, "a"), _act_type(a_type), _dev(a_scale, torch.float32, "a_scale"),
+                                 _dev(b, torch.uint8, "b"), _act_type(b_type), _dev(b_scale, torch.float32, "b_scale"),
+                                 n, _dev(out, torch.float32, "out"), 0, None, None, _stream(stream))
+    else:
+        if out is None:
+            out = torch.empty(a.shape, dtype=torch.uint8, device=a.device)
+        st = lib().fgq_add_codes(_dev(a, torch.uint8, "a"), _act_type(a_type), _dev(a_scale, torch.float32, "a_scale"),
+                                 _dev(b, torch.uint8, "b"), _act_type(b_type), _dev(b_scale, torch.float32, "b_scale"),
+                                 n, None, _act_type(out_type), _dev(out_scale, torch.float32, "out_scale"),
+                                 _dev(out, torch.uint8, "out"), _stream(stream))
+    _check(st, "fgq_add_codes")
     return out
 
 

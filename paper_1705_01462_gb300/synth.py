@@ -146,6 +146,17 @@ def weights_matrix(M: int, K: int, seed: int, fan_in: int | None = None) -> np.n
     return (g.standard_normal((M, K), dtype=np.float32) * np.float32(std)).astype(np.float32)
 
 
+def pow2_ternary_weights(layer: ConvLayer, seed: int) -> np.ndarray:
+    """fp32 [M][Kred] with values in {-c, 0, +c}, c = 2^round(log2(sqrt(2 / fan_in))): each
+    weight zero with probability 1/3, else of random sign.  Already ternary with one
+    magnitude, so every group's scaling factor is c and every contraction sum is a multiple
+    of c below 2^24 c: exact in fp32 in any order."""
+    g = rng(seed)
+    c = np.float32(2.0 ** round(np.log2(np.sqrt(2.0 / layer.fan_in))))
+    u = g.integers(0, 3, size=(layer.M, layer.Kred))
+    return ((u == 1).astype(np.float32) - (u == 2).astype(np.float32)) * c
+
+
 def activations(shape, seed: int) -> np.ndarray:
     """fp32 half-normal (sigma = 1) post-ReLU activations of the given shape."""
     g = rng(seed)
