@@ -65,16 +65,29 @@ typedef enum { FGQ_U8 = 0, FGQ_S8 = 1, FGQ_U4 = 2, FGQ_S4 = 3 } fgq_act_type;
 
 /* Contraction kernel families (see fgq_set_path / fgq_last_path). */
 typedef enum {
-  FGQ_PATH_AUTO = 0,   /* choose per shape: the few-row path for small GEMMs, else the
-                          tensor cores where the shape is covered (G = 4 only with at least
-                          128 filters per conv group), else the CUDA cores */
+  FGQ_PATH_AUTO = 0,   /* choose per shape: the few-row path for small GEMMs; with
+                          fixed-point alphas the dense tensor-core path where it applies;
+                          else the tensor cores where the shape is covered (G = 4 only with
+                          at least 128 filters per conv group), else the CUDA cores */
   FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
   FGQ_PATH_TC = 2,     /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
                           the group; G = 4 with a block-diagonal activation operand
                           (Cg a multiple of 64) */
-  FGQ_PATH_GEMV = 3    /* few-row path for GEMMs with P <= 8 (8-bit activations, Kred a
+  FGQ_PATH_GEMV = 3,   /* few-row path for GEMMs with P <= 8 (8-bit activations, Kred a
                           multiple of 16, G >= 4): one warp per filter row streams the
                           weights once; the automatic choice for such calls */
+  FGQ_PATH_DENSE = 4   /* dense tensor-core path (tcgen05, any G, 8-bit activations, Cg a
+                          multiple of 64): the alphas are folded into fp16 weights
+                          alpha(m, k / G) * t[m][k] built per call, and one dense
+                          contraction replaces the per-group multiplies.  Fixed-point alphas
+                          fold exactly (integer weights |a t| <= 255; the result is the exact
+                          value rounded once while |sum a t q| < 2^24): the automatic choice
+                          for fgq_gemm_qa / fgq_conv2d_qa.  fp32 alphas (only when forced)
+                          are split per filter row into two fp16 parts after scaling the
+                          row's largest alpha into [2^14, 2^15), about 22 bits of alpha, and
+                          the fp32 accumulator rounds once per 16 reduction elements: a
+                          numerical ablation of folding, outside the fgq_gemm tolerance
+                          guarantee. */
 } fgq_path;
 
 /* ABI version of this header (incremented on any signature change). */

@@ -61,13 +61,16 @@ bool tc_any(const Geom& g) { return g.G == 4 ? tc4_supports(g) : tc_supports(g);
 
 bool gemv_any(const Geom& g) { return !g.is_conv && gemv_supports((int)g.P, g.Kred, g.G, g.act_type); }
 
-int choose_path(const Geom& g, bool sums) {
+int choose_path(const Geom& g, bool sums, bool qa) {
   const int forced = g_path.load();
   if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
   if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
   if (forced == FGQ_PATH_GEMV) return gemv_any(g) ? FGQ_PATH_GEMV : -1;
+  if (forced == FGQ_PATH_DENSE) return dense_supports(g) ? FGQ_PATH_DENSE : -1;
   if (gemv_any(g)) return FGQ_PATH_GEMV;  // a few activation rows: stream the weights once
+  // fixed-point alphas fold exactly into fp16 weights: one dense tensor-core contraction
+  if (qa && dense_supports(g)) return FGQ_PATH_DENSE;
   // automatic choice: the tensor cores where the shape is covered, except G = 4 layers with
   // fewer than 128 filters per conv group, where the 128-row MMA tile would leave half its
   // rows idle and the dp4a kernel is faster
@@ -85,10 +88,13 @@ struct QAlpha {
 fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                     const float* act_scale, float* out, int32_t* sums, cudaStream_t s, const QAlpha* qa = nullptr) {
   if (g.P == 0 || g.M == 0) return FGQ_OK;
-  const int path = choose_path(g, sums != nullptr);
+  const int path = choose_path(g, sums != nullptr, qa != nullptr);
   if (path < 0) return FGQ_ERR_UNSUPPORTED;
   t_last_path = path;
   unsigned int* err = device_error_word();
+  if (path == FGQ_PATH_DENSE)
+    return launch_dense_contract(act, g, codes, alpha, qa ? qa->aq : nullptr, qa ? qa->bits : 0,
+                                 qa ? qa->ascale : nullptr, act_scale, out, err, s);
   if (path == FGQ_PATH_GEMV)
     return launch_gemv(act, g.act_type, (int)g.P, g.Kred, g.M, g.G, codes, alpha, qa ? qa->aq : nullptr,
                        qa ? qa->bits : 0, qa ? qa->ascale : nullptr, act_scale, out, g.rq_out, g.rq_scale,
@@ -460,7 +466,9 @@ fgq_status fgq_stream_status(cudaStream_t stream) {
 }
 
 int fgq_set_path(int path) {
-  if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC && path != FGQ_PATH_GEMV) return -1;
+  if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC && path != FGQ_PATH_GEMV &&
+      path != FGQ_PATH_DENSE)
+    return -1;
   return g_path.exchange(path);
 }
 

@@ -65,6 +65,14 @@ bool tc4_supports(const Geom& g);
 fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                                const float* act_scale, float* out, unsigned int* err, cudaStream_t s);
 
+// Dense tensor-core contraction with the alphas folded into fp16 weights: fixed-point alphas
+// (aq, abits 8 or 4, ascale) exactly, or fp32 alphas (aq == nullptr) split into two fp16
+// parts.  8-bit activations, Cg % 64 == 0.
+bool dense_supports(const Geom& g);
+fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
+                                 const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
+                                 unsigned int* err, cudaStream_t s);
+
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
 
 // Chained-forward steps: max pooling of u8 codes, residual addition of two 8-bit code

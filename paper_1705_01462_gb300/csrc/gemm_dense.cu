@@ -1,0 +1,620 @@
+// Dense tensor-core (tcgen05) contraction with the group scales folded into the weights.
+//
+// Eq. 2 sums alpha_g * (sum over group g of t * x); with A[m][k] = alpha(m, k / G) * t[m][k] the
+// same value is one dense contraction y[p][m] = s_x * rs[m] * sum_k A[m][k] q[p][k], with no
+// multiply per group.  A is built once per call in fp16, in one or two parts (A = A0 + A1):
+//
+//   * fixed-point alphas (Section 4: 8/4-bit codes a[m][g], one exponent E_m per filter row):
+//     A = a * t, integers of magnitude <= 255 and exact in fp16; rs = 2^E_m.  Products and
+//     every partial sum below 2^24 are exact in the fp32 accumulator, so y is the exact value
+//     rounded once whenever |sum_k A q| < 2^24.
+//   * fp32 alphas (an ablation): alpha * 2^e_m = hi + lo with hi = fp16(alpha 2^e_m) and lo =
+//     fp16(the remainder); e_m puts the row's largest alpha in [2^14, 2^15), so the pair
+//     carries about 22 bits of alpha; A0 = hi t, A1 = lo t, rs = 2^-e_m.  The accumulator
+//     rounds once per K = 16 step.
+//
+// Tile: 128 filters x 256 positions, K-tile 64.  Each K-tile is 4 (or 8, two parts) MMAs
+// M = 128, N = 256, K = 16 into the tile's TMEM accumulator (256 columns); the epilogue runs
+// once per tile.  Two accumulators: the epilogue of tile i overlaps the MMAs of tile i + 1.
+// Warp roles (448 threads, one CTA per SM, persistent over tiles):
+//   warps 0-7  epilogue: warp w reads TMEM lanes 32 (w % 4) .. (filters), columns 128 (w / 4)
+//              .. +127 (positions), scales by s_x rs[m] and stores fp32 (through shared memory
+//              and TMA box stores where the output allows, single-part weights) or requantized
+//              codes;
+//   warps 8-11 loaders/converters: thread t brings the activation rows of tile positions t and
+//              t + 128 (TMA boxes for 1x1 stride-1 layers and GEMMs, else cp.async gathers) and
+//              converts them to the fp16 operand B (two stages);
+//   warp 12    TMEM allocation and the MMA issuer;
+//   warp 13    streams the folded-weight boxes (A) by TMA into their own ring of four stages
+//              (two for split weights), released by the MMAs' commits, so the boxes arrive
+//              ahead of the K-tiles that use them.
+// Every mbarrier wait is bounded in time; on expiry the kernel records FGQ_ERR_TIMEOUT, each
+// role leaves its loop, in-flight copies and MMAs are waited for, and TMEM is freed.
+#include <cuda_fp16.h>
+
+#include <cstdint>
+#include <cstring>
+
+#include "tc_common.cuh"
+
+namespace fgq {
+namespace {
+
+using tc::encode_tiled;
+using tc::make_map_2d;
+using tc::st_off;
+using tc::sw128;
+using tc::u8pair_to_h2;
+
+constexpr int TD_BM = 128;   // filters per tile (MMA M, TMEM lanes)
+constexpr int TD_BN = 256;   // positions per tile (MMA N)
+constexpr int TD_KT = 64;    // reduction elements per K-tile (4 MMA steps of K = 16)
+constexpr int TD_NS = 4;     // staging ring depth
+constexpr int TD_NACC = 2;   // TMEM accumulators of 256 columns (one tile each)
+constexpr int TD_EPI_WARPS = 8;
+constexpr int TD_LOAD_WARP0 = 8;
+constexpr int TD_LOADERS = 128;
+constexpr int TD_MMA_WARP = 12;
+constexpr int TD_A_WARP = 13;  // lane 0 streams the folded-weight boxes
+constexpr int TD_THREADS = 32 * (TD_A_WARP + 1);
+constexpr int TD_TMEM_COLS = TD_NACC * 256;
+constexpr uint64_t TD_TIMEOUT_NS = 1000000000ull;  // 1 s per wait
+constexpr uint32_t BAR_EPID = 3;
+
+constexpr int A_TILED = TD_BM * TD_KT * 2;  // 16 KB fp16 [128 filters][64 K] per part
+constexpr int B_TILED = TD_BN * TD_KT * 2;  // 32 KB fp16 [256 positions][64 K]
+constexpr int ST_STAGED = TD_BN * TD_KT;    // 16 KB: 256 raw activation rows of 64 bytes
+constexpr int OUT_BOXD = 64 * TD_BM * 4;    // 32 KB: fp32 [64 positions][128 filters]
+
+template <int NA>
+struct DenseCfg {
+  static constexpr int NAS = NA == 1 ? 4 : 2;  // folded-weight (A) ring depth
+  static constexpr int NB = 2;                 // activation operand (B) ring depth
+  static constexpr int A_STAGE = NA * A_TILED;
+  static constexpr int SMEM_A = NAS * A_STAGE;
+  static constexpr int SMEM_B = NB * B_TILED;
+  static constexpr int SMEM_ST = TD_NS * ST_STAGED;
+  // output staging for TMA box stores: one [64 positions][128 filters] fp32 box, single-part
+  // weights only (two parts leave no room)
+  static constexpr int SMEM_OUT = NA == 1 ? OUT_BOXD : 0;
+  static constexpr int SMEM_BAR = 8 * (2 * NAS + 2 * NB + 2 * TD_NS + 2 * TD_NACC + 1) + 16;
+  static constexpr int SMEM = 1024 + SMEM_A + SMEM_B + SMEM_ST + SMEM_OUT + SMEM_BAR;
+};
+static_assert(DenseCfg<1>::SMEM <= 232448 && DenseCfg<2>::SMEM <= 232448, "shared memory budget");
+static_assert(A_TILED % 1024 == 0 && B_TILED % 1024 == 0 && ST_STAGED % 1024 == 0, "stage alignment");
+
+struct TDArgs {
+  CUtensorMap a_map[2];  // fp16 [M][Kp] folded weights (part 0, part 1), box {64, 128 rows}, 128-byte swizzle
+  CUtensorMap act_map;   // uint8 [pixels][C], box {64 bytes, 256 rows}, 64-byte swizzle; TMA path
+  CUtensorMap out_map;   // fp32 [P][M], box {128 filters, 64 positions}; if out_tma
+  const uint8_t* act;
+  const float* row_scale;  // rs [M]
+  const float* act_scale;
+  float* out;
+  unsigned int* err;
+  Geom g;
+  int mtiles, ptiles, ntiles, ktiles;
+  int out_tma;
+  uint64_t timeout_ns;
+};
+
+// Filter tiles of one position tile are consecutive, so CTAs running at the same time share
+// activation rows in L2.
+__device__ __forceinline__ void tile_coords_d(const TDArgs& a, int tile, int& gi, int& m0, int64_t& p0) {
+  const int per_p = a.g.groups * a.mtiles;
+  const int pt = tile / per_p;
+  const int r = tile - pt * per_p;
+  gi = r / a.mtiles;
+  m0 = gi * a.g.Mg + (r - gi * a.mtiles) * TD_BM;
+  p0 = (int64_t)pt * TD_BN;
+}
+
+// Folded weights, one warp per filter row.  MODE 8 / 4: fixed-point alpha codes (8-bit, or
+// 4-bit packed two per byte, element 2i in the low nibble) times t, and rs = ascale; MODE 0:
+// fp32 alphas split into hi + lo after scaling the row by 2^e, rs = 2^-e.  Row m of part i
+// is fp16 [Kp] at a_i + m Kp; codes 00 and padding give 0.
+template <int MODE>
+__global__ void __launch_bounds__(256) fold_weights_kernel(const uint32_t* __restrict__ codes, int M, int wrow, int G,
+                                                           int ng, const float* __restrict__ alpha,
+                                                           const uint8_t* __restrict__ aq,
+                                                           const float* __restrict__ ascale, __half* __restrict__ a0,
+                                                           __half* __restrict__ a1, float* __restrict__ row_scale) {
+  const int m = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  float mul = 1.0f;
+  if (MODE == 0) {
+    float mx = 0.0f;
+    for (int g = lane; g < ng; g += 32) mx = fmaxf(mx, __ldg(alpha + (int64_t)m * ng + g));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    int e = mx > 0.0f ? 14 - ilogbf(mx) : 0;  // mx 2^e in [2^14, 2^15)
+    e = e < -100 ? -100 : (e > 100 ? 100 : e);
+    mul = ldexpf(1.0f, e);
+    if (lane == 0) row_scale[m] = ldexpf(1.0f, -e);
+  } else if (lane == 0) {
+    row_scale[m] = __ldg(ascale + m);
+  }
+  const int64_t arow = MODE == 4 ? (ng + 1) / 2 : ng;
+  for (int w = lane; w < wrow; w += 32) {
+    const uint32_t cw = __ldg(codes + (int64_t)m * wrow + w);
+    uint32_t h0[8], h1[8];
+#pragma unroll
+    for (int e2 = 0; e2 < 8; ++e2) {
+      uint32_t v0[2], v1[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int e = 2 * e2 + u;
+        const uint32_t c = (cw >> (2 * e)) & 3u;
+        const int g = (16 * w + e) / G;
+        v0[u] = v1[u] = 0u;
+        if ((c == 1u || c == 3u) && g < ng) {
+          float v;
+          if (MODE == 8) {
+            v = (float)__ldg(aq + (int64_t)m * arow + g);
+          } else if (MODE == 4) {
+            const uint32_t b = __ldg(aq + (int64_t)m * arow + g / 2);
+            v = (float)((g & 1) ? (b >> 4) : (b & 15u));
+          } else {
+            v = __ldg(alpha + (int64_t)m * ng + g) * mul;  // exact: a power-of-two scaling
+          }
+          const __half hi = __float2half_rn(v);
+          const __half lo = __float2half_rn(v - __half2float(hi));  // the remainder, exact in fp32
+          const uint32_t sgn = c == 3u ? 0x8000u : 0u;
+          v0[u] = (uint32_t)__half_as_ushort(hi) ^ sgn;
+          v1[u] = MODE == 0 ? ((uint32_t)__half_as_ushort(lo) ^ sgn) : 0u;
+        }
+      }
+      h0[e2] = v0[0] | (v0[1] << 16);
+      h1[e2] = v1[0] | (v1[1] << 16);
+    }
+    uint4* d0 = reinterpret_cast<uint4*>(a0 + ((int64_t)m * wrow + w) * 16);
+    d0[0] = make_uint4(h0[0], h0[1], h0[2], h0[3]);
+    d0[1] = make_uint4(h0[4], h0[5], h0[6], h0[7]);
+    if (MODE == 0) {
+      uint4* d1 = reinterpret_cast<uint4*>(a1 + ((int64_t)m * wrow + w) * 16);
+      d1[0] = make_uint4(h1[0], h1[1], h1[2], h1[3]);
+      d1[1] = make_uint4(h1[4], h1[5], h1[6], h1[7]);
+    }
+  }
+}
+
+template <int NA, bool SIGNED, bool TMAP>
+__global__ void __launch_bounds__(TD_THREADS, 1) dense_contract_kernel(const __grid_constant__ TDArgs a) {
+  using Cfg = DenseCfg<NA>;
+  constexpr int NAS = Cfg::NAS;
+  constexpr int NB = Cfg::NB;
+  extern __shared__ uint8_t smem_rawd[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_rawd) + 1023) & ~uintptr_t(1023));
+  uint8_t* abuf = smem;
+  uint8_t* bbuf = smem + Cfg::SMEM_A;
+  uint8_t* st = bbuf + Cfg::SMEM_B;
+  float* otile = reinterpret_cast<float*>(st + Cfg::SMEM_ST);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(st + Cfg::SMEM_ST + Cfg::SMEM_OUT);
+  uint64_t* a_full = bars;
+  uint64_t* a_empty = bars + NAS;
+  uint64_t* op_full = bars + 2 * NAS;
+  uint64_t* op_empty = op_full + NB;
+  uint64_t* st_full = op_empty + NB;
+  uint64_t* st_empty = st_full + TD_NS;
+  uint64_t* acc_full = st_empty + TD_NS;
+  uint64_t* acc_empty = acc_full + TD_NACC;
+  uint64_t* drain_bar = acc_empty + TD_NACC;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  volatile uint32_t* abort_flag = tmem_slot + 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const Geom& g = a.g;
+  const uint64_t tmo = a.timeout_ns;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < NAS; ++i) {
+      mbar_init(&a_full[i], 1);  // the A boxes' byte count
+      mbar_init(&a_empty[i], 1);
+    }
+    for (int i = 0; i < NB; ++i) {
+      mbar_init(&op_full[i], TD_LOADERS);  // B pieces
+      mbar_init(&op_empty[i], 1);
+    }
+    for (int i = 0; i < TD_NS; ++i) {
+      mbar_init(&st_full[i], TMAP ? 1 : TD_LOADERS);
+      mbar_init(&st_empty[i], TD_LOADERS);
+    }
+    for (int i = 0; i < TD_NACC; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], TD_EPI_WARPS);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == TD_MMA_WARP) {
+    tmem_alloc(tmem_slot, TD_TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+
+  auto fail = [&]() {
+    *abort_flag = 1;
+    record_error(a.err, FGQ_ERR_TIMEOUT);
+  };
+
+  // ------------------------------------------------------------------ loaders/converters
+  if (warp >= TD_LOAD_WARP0 && warp < TD_MMA_WARP) {
+    const int t = threadIdx.x - 32 * TD_LOAD_WARP0;  // tile positions t and t + 128
+    const int total = my_tiles * a.ktiles;
+    constexpr uint32_t TX_ACT = ST_STAGED;
+
+    int cur_tile = -1, gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0;
+    int64_t p0 = 0;
+    int pb[2] = {0, 0}, phb[2] = {0, 0}, pwb[2] = {0, 0};
+    bool pvalid[2] = {false, false};
+    int issued = 0;
+    // activation rows of K-tile j (of this CTA's sequence) into staging slot j % NS
+    auto issue = [&](int j) -> bool {
+      const int tl = j / a.ktiles;
+      if (tl != cur_tile) {
+        cur_tile = tl;
+        tile_coords_d(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+        tr = ts = tc0 = 0;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int64_t p = p0 + t + 128 * r;
+          pvalid[r] = p < g.P;
+          const int pp = pvalid[r] ? (int)p : 0;
+          const int wo = pp % g.Wo;
+          const int q = pp / g.Wo;
+          const int ho = q % g.Ho;
+          pb[r] = q / g.Ho;
+          phb[r] = ho * g.stride - g.pad;
+          pwb[r] = wo * g.stride - g.pad;
+        }
+      }
+      const int slot = j % TD_NS;
+      uint8_t* sa = st + slot * ST_STAGED;
+      if (TMAP) {
+        if (t == 0) {
+          if (j >= TD_NS && !mbar_wait_timed(&st_empty[slot], ((j / TD_NS) & 1) ^ 1, tmo, abort_flag, 64))
+            return false;
+          mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
+          tma_load_2d(smem_u32(sa), &a.act_map, gi * g.Cg + tc0, (int)p0, &st_full[slot]);
+          issued = j + 1;
+        }
+      } else {
+        if (j >= TD_NS && !mbar_wait_timed(&st_empty[slot], ((j / TD_NS) & 1) ^ 1, tmo, abort_flag, 64))
+          return false;
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const uint8_t* src = a.act;
+          bool inside = false;
+          if (pvalid[r]) {
+            const int hi = phb[r] + tr, wi = pwb[r] + ts;
+            if (hi >= 0 && hi < g.H && wi >= 0 && wi < g.W) {
+              src = a.act + (((int64_t)pb[r] * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + tc0;
+              inside = true;
+            }
+          }
+          const int row = t + 128 * r;
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            cp_async16(smem_u32(sa + st_off<8>(row, c)), inside ? (const void*)(src + 16 * c) : (const void*)a.act,
+                       inside ? 16u : 0u);
+        }
+        cp_async_mbar_arrive_noinc(&st_full[slot]);
+        issued = j + 1;
+      }
+      tc0 += TD_KT;
+      if (tc0 == g.Cg) {
+        tc0 = 0;
+        if (++ts == g.S) {
+          ts = 0;
+          ++tr;
+        }
+      }
+      return true;
+    };
+
+    bool ok = true;
+    for (int j = 0; j < TD_NS - 1 && j < total && ok; ++j) ok = issue(j);
+    int consumed = 0;
+    for (int j = 0; j < total && ok; ++j) {
+      if (j + TD_NS - 1 < total && !issue(j + TD_NS - 1)) {
+        ok = false;
+        break;
+      }
+      const int slot = j % TD_NS;
+      const int os = j % NB;
+      if (!mbar_wait_timed(&op_empty[os], ((j / NB) & 1) ^ 1, tmo, abort_flag, 64)) {
+        ok = false;
+        break;
+      }
+      uint8_t* Bt = bbuf + os * B_TILED;
+      if (!mbar_wait_timed(&st_full[slot], (j / TD_NS) & 1, tmo, abort_flag, 32)) {
+        ok = false;
+        break;
+      }
+      consumed = j + 1;
+      const uint8_t* sa = st + slot * ST_STAGED;
+      constexpr uint32_t bias2 = SIGNED ? 0x64806480u : 0x64006400u;
+      constexpr uint32_t flip = 0x80808080u;
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int row = t + 128 * r;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {  // staging chunk c: activations 16 c .. 16 c + 15
+          const uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<8>(row, c));
+          const uint32_t w[4] = {SIGNED ? v.x ^ flip : v.x, SIGNED ? v.y ^ flip : v.y, SIGNED ? v.z ^ flip : v.z,
+                                 SIGNED ? v.w ^ flip : v.w};
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint4 o = make_uint4(u8pair_to_h2(w[2 * h], 0x4140, bias2), u8pair_to_h2(w[2 * h], 0x4342, bias2),
+                                       u8pair_to_h2(w[2 * h + 1], 0x4140, bias2),
+                                       u8pair_to_h2(w[2 * h + 1], 0x4342, bias2));
+            *reinterpret_cast<uint4*>(Bt + sw128(row, 2 * c + h)) = o;
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(&op_full[os]);
+      mbar_arrive(&st_empty[slot]);
+    }
+    if (!ok && !*abort_flag) fail();
+    if (!TMAP) cp_async_wait_all();
+    if (TMAP && t == 0) {
+      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % TD_NS], (j / TD_NS) & 1, 1u << 16);
+    }
+  }
+
+  // ------------------------------------------------------------------ folded-weight boxes
+  if (warp == TD_A_WARP && lane == 0) {
+    const int total = my_tiles * a.ktiles;
+    int armed = 0;
+    bool ok = true;
+    for (int j = 0; j < total && ok; ++j) {
+      const int as = j % NAS;
+      if (!mbar_wait_timed(&a_empty[as], ((j / NAS) & 1) ^ 1, tmo, abort_flag, 64)) {
+        ok = false;
+        break;
+      }
+      const int tl = j / a.ktiles;
+      int gj, mj;
+      int64_t pj;
+      tile_coords_d(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
+      uint8_t* A = abuf + as * Cfg::A_STAGE;
+      mbar_arrive_expect_tx(&a_full[as], Cfg::A_STAGE);
+#pragma unroll
+      for (int part = 0; part < NA; ++part)
+        tma_load_2d(smem_u32(A + part * A_TILED), &a.a_map[part], (j - tl * a.ktiles) * TD_KT, mj, &a_full[as]);
+      armed = j + 1;
+    }
+    if (!ok && !*abort_flag) fail();
+    // boxes the MMA issuer did not consume may still be in flight
+    for (int j = armed - NAS < 0 ? 0 : armed - NAS; j < armed; ++j)
+      mbar_wait_bounded(&a_full[j % NAS], (j / NAS) & 1, 1u << 16);
+  }
+
+  // ------------------------------------------------------------------ MMA issuer
+  if (warp == TD_MMA_WARP && lane == 0) {
+    const uint32_t idesc = idesc_f16_f32(TD_BM, TD_BN);
+    const int total = my_tiles * a.ktiles;
+    bool ok = true;
+    for (int j = 0; j < total && ok; ++j) {
+      const int tl = j / a.ktiles;
+      const int kt = j - tl * a.ktiles;
+      const int b = tl & 1;
+      if (kt == 0 && !mbar_wait_timed(&acc_empty[b], ((tl >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
+        ok = false;
+        break;
+      }
+      const int os = j % NB;
+      const int as = j % NAS;
+      if (!mbar_wait_timed(&op_full[os], (j / NB) & 1, tmo, abort_flag, 0) ||
+          !mbar_wait_timed(&a_full[as], (j / NAS) & 1, tmo, abort_flag, 0)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t abase = smem_u32(abuf + as * Cfg::A_STAGE);
+      const uint64_t bd = sdesc_k_sw128(smem_u32(bbuf + os * B_TILED));
+#pragma unroll
+      for (int part = 0; part < NA; ++part) {
+        const uint64_t ad = sdesc_k_sw128(abase + part * A_TILED);
+#pragma unroll
+        for (int s = 0; s < 4; ++s)
+          mma_f16(tmem + (uint32_t)(b * 256), ad + 2 * s, bd + 2 * s, idesc, (kt | part | s) != 0 ? 1u : 0u);
+      }
+      mma_commit(&op_empty[os]);
+      mma_commit(&a_empty[as]);
+      if (kt == a.ktiles - 1) mma_commit(&acc_full[b]);
+    }
+    if (!ok && !*abort_flag) fail();
+    mma_commit(drain_bar);
+    mbar_wait_bounded(drain_bar, 0, 1u << 20);
+  }
+
+  // ------------------------------------------------------------------ epilogue
+  if (warp < TD_EPI_WARPS) {
+    const int quarter = warp & 3, half = warp >> 2;
+    const int t = 32 * quarter + lane;  // TMEM lane = filter row of the tile
+    const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(128 * half);
+    const float sx = __ldg(a.act_scale);
+    const bool leader = threadIdx.x == 0;
+    const bool out_tma = NA == 1 && a.out_tma;
+    for (int tl = 0; tl < my_tiles; ++tl) {
+      int gi, m0;
+      int64_t p0;
+      tile_coords_d(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+      const int m = m0 + t;
+      const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
+      const float sc = mok ? sx * __ldg(a.row_scale + m) : 0.0f;
+      const int b = tl & 1;
+      const bool ok = mbar_wait_timed(&acc_full[b], (tl >> 1) & 1, tmo, abort_flag, 0);
+      if (!ok && !*abort_flag) fail();
+      if (named_bar_or(BAR_EPID, 32 * TD_EPI_WARPS, !ok)) break;
+      tc_fence_after();
+      const uint32_t ta = tbase + (uint32_t)(b * 256);
+      const int64_t pw = p0 + 128 * half;  // this warp's first position
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {  // positions pw + 64 hh .. + 63
+        uint32_t r0[32], r1[32];
+        tmem_ld32(ta + 64 * hh, r0);
+        tmem_ld32(ta + 64 * hh + 32, r1);
+        tmem_ld_wait_regs(r0);
+        reg_fence(r1);
+        if (hh == 1) {  // every column of this accumulator is in registers: free it
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);
+        }
+        if (out_tma) {
+          // one staging box: positions p0 + 128 hb + 64 hh .. + 63 are written by the warps of
+          // half hb, then stored by one thread
+#pragma unroll 1
+          for (int hb = 0; hb < 2; ++hb) {
+            if (leader) bulk_wait_read_all();  // the previous box has been read out
+            named_bar_sync(BAR_EPID, 32 * TD_EPI_WARPS);
+            if (half == hb) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                otile[i * TD_BM + t] = sc * __uint_as_float(r0[i]);
+                otile[(32 + i) * TD_BM + t] = sc * __uint_as_float(r1[i]);
+              }
+            }
+            fence_proxy_async_smem();
+            named_bar_sync(BAR_EPID, 32 * TD_EPI_WARPS);
+            if (leader) {  // a box that starts inside the output (its tail past P is not written)
+              if (p0 + 128 * hb + 64 * hh < g.P) tma_store_2d(&a.out_map, m0, (int)(p0 + 128 * hb + 64 * hh), smem_u32(otile));
+              bulk_commit();
+            }
+          }
+        } else if (mok) {
+          if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
+            const RqMul rq = rq_mul(g.rq_scale, g.rq_signed);
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+              const int64_t p = pw + 64 * hh + i;
+              const uint32_t rv = i < 32 ? r0[i] : r1[i - 32];
+              if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sc * __uint_as_float(rv), rq);
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+              const int64_t p = pw + 64 * hh + i;
+              const uint32_t rv = i < 32 ? r0[i] : r1[i - 32];
+              if (p < g.P) a.out[p * g.M + m] = sc * __uint_as_float(rv);
+            }
+          }
+        }
+      }
+    }
+    if (leader) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == TD_MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TD_TMEM_COLS);
+  }
+}
+
+template <int NA, bool SIGNED, bool TMAP>
+fgq_status launch_dense(const TDArgs& args, int grid, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(dense_contract_kernel<NA, SIGNED, TMAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             DenseCfg<NA>::SMEM) != cudaSuccess)
+      return FGQ_ERR_CUDA;
+    attr_set = true;
+  }
+  dense_contract_kernel<NA, SIGNED, TMAP><<<grid, TD_THREADS, DenseCfg<NA>::SMEM, s>>>(args);
+  return after_launch();
+}
+
+template <int NA>
+fgq_status launch_dense_na(const TDArgs& args, bool sgn, bool tmap, int grid, cudaStream_t s) {
+  if (sgn) return tmap ? launch_dense<NA, true, true>(args, grid, s) : launch_dense<NA, true, false>(args, grid, s);
+  return tmap ? launch_dense<NA, false, true>(args, grid, s) : launch_dense<NA, false, false>(args, grid, s);
+}
+
+}  // namespace
+
+bool dense_supports(const Geom& g) {
+  if (g.act_type != FGQ_U8 && g.act_type != FGQ_S8) return false;
+  if (g.Cg % TD_KT != 0) return false;        // every K-tile inside one filter tap (conv) or row (GEMM)
+  if (g.C % 16 != 0) return false;            // 16-byte aligned activation rows
+  if (g.Kp % 16 != 0) return false;           // fp16 rows of the folded weights: 32-byte multiples
+  if (g.P >= (int64_t)1 << 31) return false;  // positions decoded in 32 bits
+  if (encode_tiled() == nullptr) return false;
+  return true;
+}
+
+fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
+                                 const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
+                                 unsigned int* err, cudaStream_t s) {
+  if (!dense_supports(g)) return FGQ_ERR_UNSUPPORTED;
+  if (aq ? (abits != 8 && abits != 4) || !ascale : !alpha) return FGQ_ERR_ARG;
+  const int NA = aq ? 1 : 2;
+  TDArgs a;
+  memset(&a, 0, sizeof a);
+  a.act = static_cast<const uint8_t*>(act);
+  a.act_scale = act_scale;
+  a.out = out;
+  a.err = err;
+  a.g = g;
+  a.mtiles = (g.Mg + TD_BM - 1) / TD_BM;
+  a.ptiles = (int)((g.P + TD_BN - 1) / TD_BN);
+  a.ntiles = g.groups * a.mtiles * a.ptiles;
+  a.ktiles = g.Kred / TD_KT;
+  a.timeout_ns = TD_TIMEOUT_NS;
+
+  // folded weights fp16 [NA][M][Kp] and row scales [M], in one temporary from the pool
+  cudaMemPool_t pool = scratch_pool();
+  if (!pool) return FGQ_ERR_CUDA;
+  const size_t part_bytes = (size_t)g.M * g.Kp * 2;
+  void* tmp = nullptr;
+  if (cudaMallocFromPoolAsync(&tmp, NA * part_bytes + (size_t)g.M * 4, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
+  __half* a0 = static_cast<__half*>(tmp);
+  __half* a1 = NA == 2 ? a0 + (size_t)g.M * g.Kp : nullptr;
+  float* rs = reinterpret_cast<float*>(static_cast<uint8_t*>(tmp) + NA * part_bytes);
+  a.row_scale = rs;
+  const unsigned fblocks = (unsigned)((g.M + 7) / 8);
+  if (!aq)
+    fold_weights_kernel<0><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, alpha, nullptr, nullptr, a0, a1, rs);
+  else if (abits == 8)
+    fold_weights_kernel<8><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1, rs);
+  else
+    fold_weights_kernel<4><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1, rs);
+  fgq_status st = after_launch();
+  for (int part = 0; part < NA && st == FGQ_OK; ++part)
+    if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, part ? (const void*)a1 : (const void*)a0,
+                     (uint64_t)g.Kp, (uint64_t)g.M, (uint64_t)g.Kp * 2, TD_KT, TD_BM, CU_TENSOR_MAP_SWIZZLE_128B))
+      st = FGQ_ERR_CUDA;
+  bool tmap = false;
+  if (st == FGQ_OK && g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0)
+    tmap = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, (uint64_t)g.C, (uint64_t)g.B * g.H * g.W,
+                       (uint64_t)g.C, TD_KT, TD_BN, CU_TENSOR_MAP_SWIZZLE_64B);
+  if (st == FGQ_OK && NA == 1 && g.groups == 1 && g.M % 4 == 0 && !g.rq_out)
+    a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
+                            (uint64_t)g.M * 4, TD_BM, 64, CU_TENSOR_MAP_SWIZZLE_NONE)
+                    ? 1
+                    : 0;
+  if (st == FGQ_OK) {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = a.ntiles < sms ? a.ntiles : sms;
+    const bool sgn = g.act_type == FGQ_S8;
+    st = NA == 1 ? launch_dense_na<1>(a, sgn, tmap, grid, s) : launch_dense_na<2>(a, sgn, tmap, grid, s);
+  }
+  // the temporary returns to the pool once the work queued on s before this point is done
+  if (cudaFreeAsync(tmp, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  return st;
+}
+
+}  // namespace fgq

@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "libfgq.so")
 
 FGQ_OK, FGQ_ERR_ARG, FGQ_ERR_ALIGN, FGQ_ERR_UNSUPPORTED, FGQ_ERR_NONFINITE, FGQ_ERR_TIMEOUT, FGQ_ERR_CUDA = range(7)
 U8, S8, U4, S4 = 0, 1, 2, 3
-PATH_AUTO, PATH_SIMT, PATH_TC, PATH_GEMV = 0, 1, 2, 3
+PATH_AUTO, PATH_SIMT, PATH_TC, PATH_GEMV, PATH_DENSE = 0, 1, 2, 3, 4
 ACT_TYPES = {"u8": U8, "s8": S8, "u4": U4, "s4": S4}
 
 _lib: Optional[ctypes.CDLL] = None

@@ -1,0 +1,161 @@
+"""GPU parity of the dense tensor-core path (alphas folded into fp16 weights), through the
+C ABI.
+
+* Fixed-point alphas (Section 4: 8/4-bit codes, one exponent per filter row): the folded
+  weights a * t are integers, so the contraction is exact and the output is the oracle's
+  exact value rounded once to fp32 wherever |sum a t q| < 2^24 (everywhere in these cases),
+  and within the contraction tolerance in any case.
+* fp32 alphas split into two fp16 parts (an ablation, only when forced): within the bound
+  its arithmetic gives, s_x sum_k |alpha t q| (2^-21 + steps 2^-23) with one rounding of
+  the accumulator per 16 reduction elements and per part, and most outputs inside the
+  spec tolerance as well."""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_1705_01462_gb300 import fgq
+from _gpu import TOL, check_within, dev, make_codes, quantize_oracle, random_acts, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _clean_status():
+    fgq.fgq_set_path(fgq.PATH_AUTO)
+    yield
+    fgq.fgq_set_path(fgq.PATH_AUTO)
+    assert fgq.fgq_stream_status() == fgq.FGQ_OK
+
+
+def _qa(al, bits):
+    a, asc, _ = O.quantize_alpha(al, bits)
+    aq = a.astype(np.uint8) if bits == 8 else O.pack_alpha4(a)
+    return O.dequantize_alpha(a, asc), aq, asc
+
+
+def _check_exact(got, y, ym, row_scale, sc, what):
+    """got == fp32(y) where the integer sum y / (s_x 2^E_m) is below 2^24; else within TOL."""
+    d = np.abs(y / (np.float64(sc) * row_scale.astype(np.float64)))
+    small = d < 2.0 ** 24
+    assert small.mean() > 0.99, what
+    exact = got == y.astype(np.float32)
+    assert np.all(exact | ~small), f"{what}: {np.sum(~exact & small)} outputs differ from the exact value"
+    check_within(got, y, ym, what)
+
+
+CONV_CASES = [
+    # B, H, W, C, M, R, S, stride, pad, groups, G, act
+    (2, 14, 14, 128, 128, 3, 3, 1, 1, 1, 4, "u8"),     # gather path, one full filter tile
+    (1, 19, 17, 64, 200, 3, 3, 2, 1, 1, 4, "u8"),      # stride 2, ragged M and P
+    (3, 10, 10, 256, 64, 1, 1, 1, 0, 1, 16, "s8"),     # 1x1: TMA activation boxes, M < 128
+    (2, 9, 9, 128, 130, 1, 1, 2, 0, 1, 64, "u8"),      # strided 1x1: gathered
+    (1, 12, 12, 128, 96, 3, 3, 1, 1, 2, 8, "u8"),      # conv groups (Mg = 48)
+    (1, 7, 7, 64, 256, 3, 3, 1, 1, 1, 128, "u8"),      # G = 128: Kred 576, Kp 640 (padding)
+]
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+@pytest.mark.parametrize("case", CONV_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_conv2d_qa_dense_exact(case, bits):
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr((case, bits)).encode()))
+    Kred = R * S * (C // groups)
+    w = (rng.standard_normal((M, Kred)) * np.sqrt(2.0 / Kred)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    ad, aq, asc = _qa(al, bits)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, ad, G)
+    got = fgq.fgq_conv2d_qa(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad,
+                            groups, to_dev(codes.view(np.int32)), to_dev(aq), bits, to_dev(asc), M, G)
+    assert fgq.fgq_last_path() == fgq.PATH_DENSE
+    _check_exact(got.cpu().numpy(), y, ym, asc.reshape(1, 1, 1, M), sc, f"conv2d_qa dense {case} bits={bits}")
+
+
+def test_gemm_qa_dense_many_tiles():
+    """470 tiles over 152 CTAs: every CTA cycles its two accumulators; sampled rows checked."""
+    P, K, M, G = 60000, 256, 256, 4
+    rng = np.random.default_rng(11)
+    w = rng.standard_normal((M, K)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((P, K), "u8", rng)
+    q, sc, packed = quantize_oracle(x, "u8")
+    ad, aq, asc = _qa(al, 8)
+    got = fgq.fgq_gemm_qa(to_dev(packed), "u8", to_dev(np.array([sc], np.float32)), P, K,
+                          to_dev(codes.view(np.int32)), to_dev(aq), 8, to_dev(asc), M, G).cpu().numpy()
+    assert fgq.fgq_last_path() == fgq.PATH_DENSE
+    rows = np.unique(np.concatenate([rng.integers(0, P, 600), np.arange(P - 300, P), np.arange(0, 300)]))
+    y, ym = O.gemm(q[rows], sc, t, ad, G)
+    _check_exact(got[rows], y, ym, asc.reshape(1, M), sc, "gemm_qa dense many tiles")
+
+
+def _split_bound(q, sc, t, al, G, conv_args=None):
+    """s_x sum_k |alpha t q| from the oracle on |t| and |q|."""
+    if conv_args is None:
+        s, _ = O.gemm(np.abs(q), sc, np.abs(t), al, G)
+    else:
+        s, _ = O.conv2d(np.abs(q), sc, *conv_args, np.abs(t), al, G)
+    return s
+
+
+@pytest.mark.parametrize("case", CONV_CASES[:4], ids=lambda c: "x".join(map(str, c)))
+def test_conv2d_split_fold_ablation(case):
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()) + 5)
+    Kred = R * S * (C // groups)
+    w = (rng.standard_normal((M, Kred)) * np.sqrt(2.0 / Kred)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    fgq.fgq_set_path(fgq.PATH_DENSE)
+    got = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad,
+                         groups, to_dev(codes.view(np.int32)), to_dev(al), M, G).cpu().numpy()
+    assert fgq.fgq_last_path() == fgq.PATH_DENSE
+    mag = _split_bound(q, sc, t, al, G, (R, S, stride, pad, groups))
+    steps = 2 * Kred // 16
+    err = np.abs(got.astype(np.float64) - y)
+    assert np.all(err <= mag * (2.0 ** -21 + steps * 2.0 ** -23) + 1e-30), f"split fold {case}"
+    assert np.mean(err <= TOL * ym) > 0.99, f"split fold {case}: {np.mean(err <= TOL * ym):.4f} within TOL"
+
+
+def test_conv2d_rq_dense_split():
+    """Requantizing epilogue on the dense path: the codes equal the quantizer applied to the
+    same path's fp32 output."""
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = CONV_CASES[0]
+    rng = np.random.default_rng(21)
+    Kred = R * S * C
+    w = (rng.standard_normal((M, Kred)) * np.sqrt(2.0 / Kred)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    args = (to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad, groups,
+            to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    fgq.fgq_set_path(fgq.PATH_DENSE)
+    y32 = fgq.fgq_conv2d(*args).cpu().numpy()
+    for out_type, ot in (("u8", O.U8), ("s8", O.S8)):
+        scale = np.float32(2.0 ** O.dfp_exponent(y32.reshape(-1), ot))
+        got = fgq.fgq_conv2d_rq(*args, out_type, to_dev(np.array([scale], np.float32))).cpu().numpy()
+        assert fgq.fgq_last_path() == fgq.PATH_DENSE
+        want, _, _, _ = O.quantize(y32.reshape(-1), ot, scale_in=scale)
+        g = got.reshape(-1).astype(np.int64)
+        if out_type == "s8":
+            g = np.where(g > 127, g - 256, g)
+        assert np.array_equal(g, want.astype(np.int64)), out_type
+
+
+def test_dense_unsupported_shapes():
+    fgq.fgq_set_path(fgq.PATH_DENSE)
+    codes = torch.zeros((8, 4), dtype=torch.int32, device=dev())
+    al = torch.zeros((8, 16), dtype=torch.float32, device=dev())
+    with pytest.raises(fgq.FGQError) as e:  # 4-bit activations
+        fgq.fgq_gemm(torch.zeros(32 * 32, dtype=torch.uint8, device=dev()), "u4", torch.ones(1, device=dev()), 32, 64,
+                     codes, al, 8, 4)
+    assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
+    with pytest.raises(fgq.FGQError) as e:  # Kred = 48: not a multiple of 64
+        fgq.fgq_gemm(torch.zeros(32 * 48, dtype=torch.uint8, device=dev()), "u8", torch.ones(1, device=dev()), 32, 48,
+                     codes[:, :3].contiguous(), al[:, :12].contiguous(), 8, 4)
+    assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
