@@ -345,7 +345,12 @@ fgq_status fgq_conv2d_qa(const void* act, fgq_act_type type, const float* act_sc
  * Dense 8-bit-weight convolution for the first layer (8w-8a, Section 4):
  *   out = act_scale[0] * wscale[m] * sum_j wq[m][j] * col[j]   (exact int32 dot product).
  *   wq int8 [M][Kred], wscale fp32 [M] (as from fgq_quantize_weights_w8).  Other arguments
- *   as fgq_conv2d.  Errors as fgq_conv2d.
+ *   as fgq_conv2d.  Errors as fgq_conv2d.  With 8-bit activations and groups == 1 (and unless
+ *   FGQ_PATH_SIMT is forced) it runs on the dense tensor-core path (FGQ_PATH_DENSE): an
+ *   explicit im2col of the activations into a stream-ordered pool temporary of P * Kc bytes
+ *   (Kc = Kred rounded up to 64, at most 4096), then one dense contraction on integer fp16
+ *   operands; the sums are exact while |sum_j wq col| < 2^24 (always for Kred <= 514).
+ *   Otherwise the dp4a path.
  */
 fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_scale, int B,
                          int H, int W, int C, int R, int S, int stride, int pad, int groups,

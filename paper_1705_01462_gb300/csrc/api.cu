@@ -390,6 +390,10 @@ fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_sc
   if (!act || !act_scale || !wq || !wscale || !out) return FGQ_ERR_ARG;
   if (!aligned(act, 16) || !aligned(wscale, 4) || !aligned(out, 16) || !aligned(act_scale, 4))
     return FGQ_ERR_ALIGN;
+  if (g_path.load() != FGQ_PATH_SIMT && dense_w8_supports(g)) {
+    t_last_path = FGQ_PATH_DENSE;
+    return launch_dense_w8(act, g, wq, wscale, act_scale, out, device_error_word(), stream);
+  }
   t_last_path = FGQ_PATH_SIMT;
   return launch_simt_contract(act, g, wq, wscale, 1, act_scale, out, nullptr, stream);
 }
@@ -409,6 +413,10 @@ fgq_status fgq_conv2d_w8_rq(const void* act, fgq_act_type type, const float* act
   g.rq_out = static_cast<uint8_t*>(out_q);
   g.rq_scale = out_scale;
   g.rq_signed = out_type == FGQ_S8;
+  if (g_path.load() != FGQ_PATH_SIMT && dense_w8_supports(g)) {
+    t_last_path = FGQ_PATH_DENSE;
+    return launch_dense_w8(act, g, wq, wscale, act_scale, nullptr, device_error_word(), stream);
+  }
   t_last_path = FGQ_PATH_SIMT;
   return launch_simt_contract(act, g, wq, wscale, 1, act_scale, nullptr, nullptr, stream);
 }

@@ -72,6 +72,11 @@ bool dense_supports(const Geom& g);
 fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                                  const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
                                  unsigned int* err, cudaStream_t s);
+// The 8-bit-weight convolution (dense weights wq, per-filter scales) on the same kernel, through
+// an explicit im2col of the activations in a pool temporary (any C, groups == 1); exact.
+bool dense_w8_supports(const Geom& g);
+fgq_status launch_dense_w8(const void* act, const Geom& g, const int8_t* wq, const float* wscale,
+                           const float* act_scale, float* out, unsigned int* err, cudaStream_t s);
 
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s);
 

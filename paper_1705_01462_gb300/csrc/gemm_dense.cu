@@ -554,15 +554,67 @@ bool dense_supports(const Geom& g) {
   return true;
 }
 
-fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
-                                 const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
-                                 unsigned int* err, cudaStream_t s) {
-  if (!dense_supports(g)) return FGQ_ERR_UNSUPPORTED;
-  if (aq ? (abits != 8 && abits != 4) || !ascale : !alpha) return FGQ_ERR_ARG;
-  const int NA = aq ? 1 : 2;
+namespace {
+
+// Explicit im2col of 8-bit activations for the dense path (any channel count): row p (an
+// output position, NHWC order) of col [P][Kc] holds act[b][ho stride - pad + r][wo stride - pad
+// + s][c] at k = (r S + s) C + c, 0 outside the image and for Kred <= k < Kc.  One thread per
+// position walks its row with running (r, s, c) counters and writes it in 16-byte pieces
+// (measured faster than one thread per piece, and than staging rows in shared memory for
+// contiguous warp stores).
+constexpr int IM2COL_MAX_KC = 4096;
+__global__ void __launch_bounds__(128) im2col_u8_kernel(const uint8_t* __restrict__ act, int B, int H, int W, int C,
+                                                        int R, int S, int stride, int pad, int Ho, int Wo, int Kred,
+                                                        int Kc, uint8_t* __restrict__ col) {
+  const int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= (int64_t)B * Ho * Wo) return;
+  const int wo = (int)(p % Wo);
+  const int64_t q = p / Wo;
+  const int ho = (int)(q % Ho);
+  const int b = (int)(q / Ho);
+  const int h0 = ho * stride - pad, w0 = wo * stride - pad;
+  uint4* dst = reinterpret_cast<uint4*>(col + p * Kc);
+  int r = 0, sx = 0, c = 0;
+  for (int k0 = 0; k0 < Kc; k0 += 16) {
+    uint32_t wv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      uint32_t byte = 0u;
+      if (k0 + e < Kred) {
+        const int h = h0 + r, w = w0 + sx;
+        if (h >= 0 && h < H && w >= 0 && w < W) byte = __ldg(act + (((int64_t)b * H + h) * W + w) * C + c);
+        if (++c == C) {
+          c = 0;
+          if (++sx == S) {
+            sx = 0;
+            ++r;
+          }
+        }
+      }
+      wv[e >> 2] |= byte << (8 * (e & 3));
+    }
+    dst[k0 / 16] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  }
+}
+
+// 8-bit weights wq [M][Kred] as fp16 [M][Kc] (zero-padded), rs = wscale: exact.
+__global__ void __launch_bounds__(256) fold_w8_kernel(const int8_t* __restrict__ wq, const float* __restrict__ wscale,
+                                                      int M, int Kred, int Kc, __half* __restrict__ a0,
+                                                      float* __restrict__ row_scale) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)M * Kc) return;
+  const int m = (int)(i / Kc), k = (int)(i % Kc);
+  a0[i] = __float2half_rn(k < Kred ? (float)__ldg(wq + (int64_t)m * Kred + k) : 0.0f);
+  if (k == 0) row_scale[m] = __ldg(wscale + m);
+}
+
+// Tensor maps and launch of the dense kernel for folded weights a0 (+ a1) and row scales rs.
+fgq_status run_dense(const void* act, const Geom& g, int NA, const __half* a0, const __half* a1, const float* rs,
+                     const float* act_scale, float* out, unsigned int* err, cudaStream_t s) {
   TDArgs a;
   memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
+  a.row_scale = rs;
   a.act_scale = act_scale;
   a.out = out;
   a.err = err;
@@ -572,7 +624,37 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
   a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.ktiles = g.Kred / TD_KT;
   a.timeout_ns = TD_TIMEOUT_NS;
+  for (int part = 0; part < NA; ++part)
+    if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, part ? (const void*)a1 : (const void*)a0,
+                     (uint64_t)g.Kp, (uint64_t)g.M, (uint64_t)g.Kp * 2, TD_KT, TD_BM, CU_TENSOR_MAP_SWIZZLE_128B))
+      return FGQ_ERR_CUDA;
+  bool tmap = false;
+  if (g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0)
+    tmap = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, (uint64_t)g.C, (uint64_t)g.B * g.H * g.W,
+                       (uint64_t)g.C, TD_KT, TD_BN, CU_TENSOR_MAP_SWIZZLE_64B);
+  if (NA == 1 && g.groups == 1 && g.M % 4 == 0 && !g.rq_out)
+    a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
+                            (uint64_t)g.M * 4, TD_BM, 64, CU_TENSOR_MAP_SWIZZLE_NONE)
+                    ? 1
+                    : 0;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = a.ntiles < sms ? a.ntiles : sms;
+  const bool sgn = g.act_type == FGQ_S8;
+  return NA == 1 ? launch_dense_na<1>(a, sgn, tmap, grid, s) : launch_dense_na<2>(a, sgn, tmap, grid, s);
+}
 
+constexpr int64_t DENSE_W8_MAX_COL_BYTES = (int64_t)8 << 30;  // the im2col temporary
+
+}  // namespace
+
+fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
+                                 const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
+                                 unsigned int* err, cudaStream_t s) {
+  if (!dense_supports(g)) return FGQ_ERR_UNSUPPORTED;
+  if (aq ? (abits != 8 && abits != 4) || !ascale : !alpha) return FGQ_ERR_ARG;
+  const int NA = aq ? 1 : 2;
   // folded weights fp16 [NA][M][Kp] and row scales [M], in one temporary from the pool
   cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
@@ -582,7 +664,6 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
   __half* a0 = static_cast<__half*>(tmp);
   __half* a1 = NA == 2 ? a0 + (size_t)g.M * g.Kp : nullptr;
   float* rs = reinterpret_cast<float*>(static_cast<uint8_t*>(tmp) + NA * part_bytes);
-  a.row_scale = rs;
   const unsigned fblocks = (unsigned)((g.M + 7) / 8);
   if (!aq)
     fold_weights_kernel<0><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, alpha, nullptr, nullptr, a0, a1, rs);
@@ -591,28 +672,55 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
   else
     fold_weights_kernel<4><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1, rs);
   fgq_status st = after_launch();
-  for (int part = 0; part < NA && st == FGQ_OK; ++part)
-    if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, part ? (const void*)a1 : (const void*)a0,
-                     (uint64_t)g.Kp, (uint64_t)g.M, (uint64_t)g.Kp * 2, TD_KT, TD_BM, CU_TENSOR_MAP_SWIZZLE_128B))
-      st = FGQ_ERR_CUDA;
-  bool tmap = false;
-  if (st == FGQ_OK && g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0)
-    tmap = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, (uint64_t)g.C, (uint64_t)g.B * g.H * g.W,
-                       (uint64_t)g.C, TD_KT, TD_BN, CU_TENSOR_MAP_SWIZZLE_64B);
-  if (st == FGQ_OK && NA == 1 && g.groups == 1 && g.M % 4 == 0 && !g.rq_out)
-    a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
-                            (uint64_t)g.M * 4, TD_BM, 64, CU_TENSOR_MAP_SWIZZLE_NONE)
-                    ? 1
-                    : 0;
-  if (st == FGQ_OK) {
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = a.ntiles < sms ? a.ntiles : sms;
-    const bool sgn = g.act_type == FGQ_S8;
-    st = NA == 1 ? launch_dense_na<1>(a, sgn, tmap, grid, s) : launch_dense_na<2>(a, sgn, tmap, grid, s);
-  }
+  if (st == FGQ_OK) st = run_dense(act, g, NA, a0, a1, rs, act_scale, out, err, s);
   // the temporary returns to the pool once the work queued on s before this point is done
+  if (cudaFreeAsync(tmp, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  return st;
+}
+
+bool dense_w8_supports(const Geom& g) {
+  if (g.act_type != FGQ_U8 && g.act_type != FGQ_S8) return false;
+  if (g.groups != 1 || g.P >= (int64_t)1 << 31) return false;
+  const int64_t Kc = (g.Kred + TD_KT - 1) / TD_KT * TD_KT;
+  if (Kc > IM2COL_MAX_KC || g.P * Kc > DENSE_W8_MAX_COL_BYTES) return false;
+  return encode_tiled() != nullptr;
+}
+
+fgq_status launch_dense_w8(const void* act, const Geom& g, const int8_t* wq, const float* wscale,
+                           const float* act_scale, float* out, unsigned int* err, cudaStream_t s) {
+  if (!dense_w8_supports(g)) return FGQ_ERR_UNSUPPORTED;
+  const int Kc = (g.Kred + TD_KT - 1) / TD_KT * TD_KT;
+  cudaMemPool_t pool = scratch_pool();
+  if (!pool) return FGQ_ERR_CUDA;
+  const size_t col_bytes = (size_t)g.P * Kc, a_bytes = (size_t)g.M * Kc * 2;
+  void* tmp = nullptr;
+  if (cudaMallocFromPoolAsync(&tmp, col_bytes + a_bytes + (size_t)g.M * 4, pool, s) != cudaSuccess)
+    return FGQ_ERR_CUDA;
+  uint8_t* col = static_cast<uint8_t*>(tmp);
+  __half* a0 = reinterpret_cast<__half*>(col + col_bytes);
+  float* rs = reinterpret_cast<float*>(col + col_bytes + a_bytes);
+  im2col_u8_kernel<<<(unsigned)((g.P + 127) / 128), 128, 0, s>>>(
+      static_cast<const uint8_t*>(act), g.B, g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
+  fgq_status st = after_launch();
+  if (st == FGQ_OK) {
+    fold_w8_kernel<<<(unsigned)(((int64_t)g.M * Kc + 255) / 256), 256, 0, s>>>(wq, wscale, g.M, g.Kred, Kc, a0, rs);
+    st = after_launch();
+  }
+  if (st == FGQ_OK) {
+    // the convolution as a GEMM over the im2col rows: P x Kc activations, M x Kc weights
+    Geom gg = g;
+    gg.B = (int)g.P;
+    gg.H = gg.W = gg.Ho = gg.Wo = 1;
+    gg.R = gg.S = gg.stride = 1;
+    gg.pad = 0;
+    gg.C = gg.Cg = gg.Kred = gg.Kp = Kc;
+    gg.G = TD_KT;
+    gg.ng = Kc / TD_KT;
+    gg.wrow = Kc / 16;
+    gg.Mg = g.M;
+    gg.is_conv = 0;
+    st = run_dense(col, gg, 1, a0, nullptr, rs, act_scale, out, err, s);
+  }
   if (cudaFreeAsync(tmp, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
   return st;
 }

@@ -159,3 +159,43 @@ def test_dense_unsupported_shapes():
         fgq.fgq_gemm(torch.zeros(32 * 48, dtype=torch.uint8, device=dev()), "u8", torch.ones(1, device=dev()), 32, 48,
                      codes[:, :3].contiguous(), al[:, :12].contiguous(), 8, 4)
     assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
+
+
+W8_CASES = [(2, 40, 36, 3, 64, 7, 2, 3, "u8"),   # the ResNet stem (7x7/2, C = 3) at a reduced image size
+            (1, 17, 15, 16, 70, 3, 1, 1, "s8"),  # ragged M (direct stores), signed activations
+            (3, 9, 9, 64, 128, 1, 1, 0, "u8")]   # 1x1, Kred = 64: one K-tile, no padding
+
+
+@pytest.mark.parametrize("case", W8_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_conv2d_w8_dense_exact(case):
+    """8-bit weights on the dense path (explicit im2col): integer products and sums below 2^24,
+    so the output is the exact value, equal to the dp4a path's, and the requantized codes are
+    the quantizer applied to the exact value."""
+    B, H, W, C, M, R, stride, pad, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()))
+    Kred = R * R * C
+    w = (rng.standard_normal((M, Kred)) * np.sqrt(2.0 / Kred)).astype(np.float32)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    owq, ows = O.quantize_weights_w8(w)
+    y, _ = O.conv2d_w8(q, sc, R, R, stride, pad, 1, owq, ows)
+    args = (to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, R, stride, pad, 1, to_dev(owq),
+            to_dev(ows), M)
+    got = fgq.fgq_conv2d_w8(*args).cpu().numpy()
+    assert fgq.fgq_last_path() == fgq.PATH_DENSE
+    assert np.array_equal(got, y.astype(np.float32))
+    fgq.fgq_set_path(fgq.PATH_SIMT)
+    simt = fgq.fgq_conv2d_w8(*args).cpu().numpy()
+    assert fgq.fgq_last_path() == fgq.PATH_SIMT
+    assert np.array_equal(got, simt)
+    fgq.fgq_set_path(fgq.PATH_AUTO)
+    y32 = y.astype(np.float32).reshape(-1)
+    for out_type, ot in (("u8", O.U8), ("s8", O.S8)):
+        scale = np.float32(2.0 ** O.dfp_exponent(y32, ot))
+        rq = fgq.fgq_conv2d_w8_rq(*args, out_type, to_dev(np.array([scale], np.float32))).cpu().numpy()
+        assert fgq.fgq_last_path() == fgq.PATH_DENSE
+        want, _, _, _ = O.quantize(y32, ot, scale_in=scale)
+        g = rq.reshape(-1).astype(np.int64)
+        if out_type == "s8":
+            g = np.where(g > 127, g - 256, g)
+        assert np.array_equal(g, want.astype(np.int64)), out_type
