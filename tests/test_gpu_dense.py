@@ -8,7 +8,7 @@ C ABI.
 * fp32 alphas split into two fp16 parts (an ablation, only when forced): within the bound
   its arithmetic gives, s_x sum_k |alpha t q| (2^-21 + steps 2^-23) with one rounding of
   the accumulator per 16 reduction elements and per part, and most outputs inside the
-  spec tolerance as well."""
+  contraction tolerance as well."""
 import zlib
 
 import numpy as np
