@@ -191,6 +191,16 @@ class Workload:
                     self.alpha[G].append(torch.empty((l.M, fgq.num_groups(l.Kred, G)), dtype=torch.float32,
                                                      device=dev))
                 self.out[G].append(torch.empty((B, l.Ho, l.Wo, l.M), dtype=torch.float32, device=dev))
+        # host tables of the ternary layers for fgq_ternarize_batch (one launch per G)
+        import ctypes
+        tl = list(range(1, len(layers)))
+        n = len(tl)
+        self.tern_n = n
+        self.tern_w = (ctypes.c_void_p * n)(*[self.w[i].data_ptr() for i in tl])
+        self.tern_M = (ctypes.c_int * n)(*[layers[i].M for i in tl])
+        self.tern_K = (ctypes.c_int * n)(*[layers[i].Kred for i in tl])
+        self.tern_codes = {G: (ctypes.c_void_p * n)(*[self.codes[G][i].data_ptr() for i in tl]) for G in GROUPS}
+        self.tern_alpha = {G: (ctypes.c_void_p * n)(*[self.alpha[G][i].data_ptr() for i in tl]) for G in GROUPS}
         torch.cuda.synchronize()
 
     def step(self, stream, timers=None, counts=None):
@@ -214,11 +224,10 @@ class Workload:
             calls.append(("quantize_weights_w8", lambda G=G, l=l: chk(L.fgq_quantize_weights_w8(
                 self.w[0].data_ptr(), l.M, l.Kred, self.codes[G][0].data_ptr(), self.alpha[G][0].data_ptr(), sh),
                 "w8")))
-        for G in GROUPS:
-            for i, l in enumerate(self.layers[1:], start=1):
-                calls.append((f"ternarize_g{G}", lambda G=G, i=i, l=l: chk(L.fgq_ternarize(
-                    self.w[i].data_ptr(), l.M, l.Kred, G, self.codes[G][i].data_ptr(), self.alpha[G][i].data_ptr(),
-                    sh), "ternarize")))
+        for G in GROUPS:  # all 52 ternary layers of the stack in one launch per G
+            calls.append((f"ternarize_g{G}", lambda G=G: chk(L.fgq_ternarize_batch(
+                self.tern_n, self.tern_w, self.tern_M, self.tern_K, G, self.tern_codes[G], self.tern_alpha[G], sh),
+                "ternarize_batch")))
         for i, l in enumerate(self.layers):
             calls.append(("quantize_act", lambda i=i: chk(L.fgq_quantize_act(
                 self.x[i].data_ptr(), self.x[i].numel(), fgq.U8, 0.0, self.q[i].data_ptr(), self.sc[i].data_ptr(),

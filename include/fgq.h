@@ -121,6 +121,24 @@ int64_t fgq_num_groups(int Kred, int G);
 fgq_status fgq_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
                          cudaStream_t stream);
 
+/* Largest number of weight sets one fgq_ternarize_batch call takes. */
+#define FGQ_TERNARIZE_BATCH_MAX 128
+
+/*
+ * fgq_ternarize for n weight sets of one group size G in one launch (the layers of a
+ * network): set i is w[i] fp32 [M[i]][Kred[i]] -> codes[i], alpha[i], with the layouts,
+ * results (bit for bit) and non-finite handling of fgq_ternarize.  w, M, Kred, codes,
+ * alpha are HOST arrays of n entries holding device pointers and sizes (read during the
+ * call, not kept); sets with M[i] * Kred[i] == 0 are skipped.  The sets must not overlap
+ * one another's outputs.  One kernel launch for all sets (work items numbered across them),
+ * so small layers do not each pay a launch and a partly idle grid.
+ * Errors: FGQ_ERR_ARG (n < 0 or n > FGQ_TERNARIZE_BATCH_MAX, a null array with n > 0, or
+ * any set that fgq_ternarize would reject for its arguments), FGQ_ERR_ALIGN (as
+ * fgq_ternarize, per set), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_ternarize_batch(int n, const float* const* w, const int* M, const int* Kred, int G,
+                               uint32_t* const* codes, float* const* alpha, cudaStream_t stream);
+
 /* Bytes of device workspace fgq_quantize_act needs for n elements (0 when n == 0). */
 size_t fgq_quantize_act_workspace_bytes(size_t n);
 

@@ -204,6 +204,20 @@ fgq_status fgq_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes
   return launch_ternarize(w, M, Kred, G, codes, alpha, device_error_word(), stream);
 }
 
+fgq_status fgq_ternarize_batch(int n, const float* const* w, const int* M, const int* Kred, int G,
+                               uint32_t* const* codes, float* const* alpha, cudaStream_t stream) {
+  if (n < 0 || n > FGQ_TERNARIZE_BATCH_MAX || !valid_G(G)) return FGQ_ERR_ARG;
+  if (n == 0) return FGQ_OK;
+  if (!w || !M || !Kred || !codes || !alpha) return FGQ_ERR_ARG;
+  for (int i = 0; i < n; ++i) {
+    if (M[i] < 0 || Kred[i] < 0 || (int64_t)Kred[i] + G > INT32_MAX) return FGQ_ERR_ARG;
+    if ((int64_t)M[i] * Kred[i] == 0) continue;
+    if (!w[i] || !codes[i] || !alpha[i]) return FGQ_ERR_ARG;
+    if (!aligned(w[i], 4) || !aligned(codes[i], 4) || !aligned(alpha[i], 4)) return FGQ_ERR_ALIGN;
+  }
+  return launch_ternarize_batch(n, w, M, Kred, G, codes, alpha, device_error_word(), stream);
+}
+
 size_t fgq_ternarize_threshold_workspace_bytes(void) { return threshold_workspace_bytes(); }
 
 fgq_status fgq_ternarize_threshold(const float* w, int M, int Kred, int G, int rule, int per_layer, uint32_t* codes,

@@ -35,6 +35,8 @@ fgq_status after_launch();
 // Kernel launchers (each returns FGQ_OK or FGQ_ERR_CUDA / FGQ_ERR_UNSUPPORTED).
 fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
                             unsigned int* err, cudaStream_t s);
+fgq_status launch_ternarize_batch(int n, const float* const* w, const int* M, const int* Kred, int G,
+                                  uint32_t* const* codes, float* const* alpha, unsigned int* err, cudaStream_t s);
 fgq_status launch_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
                                       unsigned int* err, cudaStream_t s);
 size_t quantize_workspace_bytes(size_t n);

@@ -13,6 +13,7 @@
 // candidates.  Equal magnitudes are kept or dropped together (a threshold rule), ties in
 // the objective go to the smaller kept set, and alpha is the fp32 nearest the exact mean.
 #include <cstdint>
+#include <cstring>
 
 #include "fgq_device.cuh"
 
@@ -145,6 +146,59 @@ __device__ __forceinline__ uint32_t solve_group_regs(const float (&v)[G], float&
   return bits;
 }
 
+// One unit of max(G, 4) consecutive weights of a row (one code byte for G <= 4): unit u of
+// the layer, units_per_row units per filter row.
+template <int G>
+__device__ __forceinline__ void small_unit(const float* __restrict__ w, int Kred, int ng, int wrow,
+                                           uint8_t* __restrict__ codes, float* __restrict__ alpha, unsigned int* err,
+                                           int vec4, int64_t units_per_row, int64_t u) {
+  constexpr int UNIT = G < 4 ? 4 : G;
+  constexpr int NSUB = UNIT / G;
+  const int m = (int)(u / units_per_row);
+  const int ui = (int)(u - (int64_t)m * units_per_row);
+  const int k0 = ui * UNIT;
+  const float* row = w + (int64_t)m * Kred;
+  float v[UNIT];
+  if (vec4 && k0 + UNIT <= Kred) {
+#pragma unroll
+    for (int i = 0; i < UNIT; i += 4) {
+      const float4 f = __ldg(reinterpret_cast<const float4*>(row + k0 + i));
+      v[i] = f.x; v[i + 1] = f.y; v[i + 2] = f.z; v[i + 3] = f.w;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < UNIT; ++i) v[i] = (k0 + i < Kred) ? __ldg(row + k0 + i) : 0.0f;
+  }
+  uint32_t bits = 0;
+#pragma unroll
+  for (int sub = 0; sub < NSUB; ++sub) {
+    const int g = ui * NSUB + sub;
+    if (g < ng) {
+      float gv[G];
+#pragma unroll
+      for (int i = 0; i < G; ++i) gv[i] = v[sub * G + i];
+      float a;
+      bool bad;
+      const uint32_t b = solve_group_regs<G>(gv, a, bad);
+      if (bad) record_error(err, FGQ_ERR_NONFINITE);
+      alpha[(int64_t)m * ng + g] = a;
+      bits |= b << (2 * sub * G);
+    }
+  }
+  uint8_t* crow = codes + (int64_t)m * wrow * 4;
+  const int byte0 = k0 / 4;
+  if (UNIT == 4) {
+    crow[byte0] = (uint8_t)bits;
+  } else if (UNIT == 8) {
+    *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)bits;
+  } else {
+    *reinterpret_cast<uint32_t*>(crow + byte0) = bits;
+  }
+  if (ui == units_per_row - 1) {  // zero the unused bytes of the row's last word
+    for (int b = byte0 + UNIT / 4; b < wrow * 4; ++b) crow[b] = 0;
+  }
+}
+
 // One thread per unit of max(G, 4) consecutive weights (one code byte for G <= 4).
 template <int G>
 __global__ void __launch_bounds__(256) ternarize_small_kernel(const float* __restrict__ w, int M, int Kred,
@@ -152,189 +206,200 @@ __global__ void __launch_bounds__(256) ternarize_small_kernel(const float* __res
                                                               float* __restrict__ alpha, unsigned int* err,
                                                               int vec4) {
   constexpr int UNIT = G < 4 ? 4 : G;
-  constexpr int NSUB = UNIT / G;
   const int Kp = ng * G;
   const int64_t units_per_row = (Kp + UNIT - 1) / UNIT;
   const int64_t total = (int64_t)M * units_per_row;
-  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total;
-       u += (int64_t)gridDim.x * blockDim.x) {
-    const int m = (int)(u / units_per_row);
-    const int ui = (int)(u - (int64_t)m * units_per_row);
-    const int k0 = ui * UNIT;
-    const float* row = w + (int64_t)m * Kred;
-    float v[UNIT];
-    if (vec4 && k0 + UNIT <= Kred) {
-#pragma unroll
-      for (int i = 0; i < UNIT; i += 4) {
-        const float4 f = __ldg(reinterpret_cast<const float4*>(row + k0 + i));
-        v[i] = f.x; v[i + 1] = f.y; v[i + 2] = f.z; v[i + 3] = f.w;
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < UNIT; ++i) v[i] = (k0 + i < Kred) ? __ldg(row + k0 + i) : 0.0f;
-    }
-    uint32_t bits = 0;
-#pragma unroll
-    for (int sub = 0; sub < NSUB; ++sub) {
-      const int g = ui * NSUB + sub;
-      if (g < ng) {
-        float gv[G];
-#pragma unroll
-        for (int i = 0; i < G; ++i) gv[i] = v[sub * G + i];
-        float a;
-        bool bad;
-        const uint32_t b = solve_group_regs<G>(gv, a, bad);
-        if (bad) record_error(err, FGQ_ERR_NONFINITE);
-        alpha[(int64_t)m * ng + g] = a;
-        bits |= b << (2 * sub * G);
-      }
-    }
-    uint8_t* crow = codes + (int64_t)m * wrow * 4;
-    const int byte0 = k0 / 4;
-    if (UNIT == 4) {
-      crow[byte0] = (uint8_t)bits;
-    } else if (UNIT == 8) {
-      *reinterpret_cast<uint16_t*>(crow + byte0) = (uint16_t)bits;
-    } else {
-      *reinterpret_cast<uint32_t*>(crow + byte0) = bits;
-    }
-    if (ui == units_per_row - 1) {  // zero the unused bytes of the row's last word
-      for (int b = byte0 + UNIT / 4; b < wrow * 4; ++b) crow[b] = 0;
-    }
-  }
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < total; u += (int64_t)gridDim.x * blockDim.x)
+    small_unit<G>(w, Kred, ng, wrow, codes, alpha, err, vec4, units_per_row, u);
 }
 
-// One warp per group for G in {32, 64, 128}: lane l holds elements l*E .. l*E+E-1.
+// One group of G in {32, 64, 128} weights (group grp = m ng + g of the layer) solved by one
+// warp: lane l holds elements l*E .. l*E+E-1.
+template <int G>
+__device__ __forceinline__ void warp_group(const float* __restrict__ w, int Kred, int ng, int wrow,
+                                           uint32_t* __restrict__ codes, float* __restrict__ alpha, unsigned int* err,
+                                           int64_t grp, int lane) {
+  constexpr int E = G / 32;
+  constexpr int L = 16 / E;  // lanes per code word
+  const int m = (int)(grp / ng);
+  const int g = (int)(grp - (int64_t)m * ng);
+  const float* row = w + (int64_t)m * Kred;
+  const int k0 = g * G + lane * E;
+  float v[E];
+  uint32_t mag[E], s[E];
+  bool bad = false;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    v[e] = (k0 + e < Kred) ? __ldg(row + k0 + e) : 0.0f;
+    mag[e] = __float_as_uint(v[e]) & 0x7fffffffu;
+    bad |= mag[e] >= 0x7f800000u;
+    s[e] = mag[e];
+  }
+  if (__any_sync(FULL_MASK, bad)) {
+    if (lane == 0) {
+      record_error(err, FGQ_ERR_NONFINITE);
+      alpha[grp] = 0.0f;
+    }
+    if (lane < G / 16) codes[(int64_t)m * wrow + g * (G / 16) + lane] = 0;
+    return;
+  }
+  // bitonic sort of the G magnitudes across the warp, descending
+#pragma unroll
+  for (int size = 2; size <= G; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      if (stride >= E) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int i = lane * E + e;
+          const uint32_t p = __shfl_xor_sync(FULL_MASK, s[e], stride / E);
+          const bool lower = (i & stride) == 0;
+          const bool desc = (i & size) == 0;
+          const uint32_t mx = s[e] > p ? s[e] : p, mn = s[e] > p ? p : s[e];
+          s[e] = (lower == desc) ? mx : mn;
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          if ((e & stride) == 0) {
+            const int i = lane * E + e;
+            const bool desc = (i & size) == 0;
+            const int e2 = (e + stride) < E ? e + stride : e;
+            const uint32_t a = s[e], b = s[e2];
+            const uint32_t mx = a > b ? a : b, mn = a > b ? b : a;
+            s[e] = desc ? mx : mn;
+            s[e2] = desc ? mn : mx;
+          }
+        }
+      }
+    }
+  }
+  const uint32_t mmax = __shfl_sync(FULL_MASK, s[0], 0);
+  uint32_t bk = 0, tau = 0;
+  uint64_t bS = 0;
+  int F = 1;
+  if (mmax != 0) {
+    F = max((int)(mmax >> 23), 1);
+    uint64_t pre[E];
+    uint64_t run = 0;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      run += fixed_of(s[e], F);
+      pre[e] = run;
+    }
+    uint64_t incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint64_t n = __shfl_up_sync(FULL_MASK, incl, o);
+      if (lane >= o) incl += n;
+    }
+    const uint64_t excl = incl - run;
+    const uint32_t next_first = __shfl_down_sync(FULL_MASK, s[0], 1);
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const int i = lane * E + e;
+      const uint32_t nxt = (e + 1 < E) ? s[(e + 1) < E ? e + 1 : e] : next_first;
+      const bool run_end = (i == G - 1) || (nxt < s[e]);
+      if (run_end && in_window(s[e], F)) {
+        const uint64_t S = excl + pre[e];
+        if (bk == 0 || j_greater(S, (uint32_t)(i + 1), bS, bk)) {
+          bS = S;
+          bk = (uint32_t)(i + 1);
+          tau = s[e];
+        }
+      }
+    }
+    // warp argmax of the objective; equal objectives keep the smaller kept count
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t oS = __shfl_xor_sync(FULL_MASK, bS, o);
+      const uint32_t ok = __shfl_xor_sync(FULL_MASK, bk, o);
+      const uint32_t ot = __shfl_xor_sync(FULL_MASK, tau, o);
+      bool take;
+      if (ok == 0) take = false;
+      else if (bk == 0) take = true;
+      else if (j_greater(oS, ok, bS, bk)) take = true;
+      else if (j_greater(bS, bk, oS, ok)) take = false;
+      else take = ok < bk;
+      if (take) {
+        bS = oS;
+        bk = ok;
+        tau = ot;
+      }
+    }
+  }
+  const float a = bk ? round_ratio_f32(bS, bk, F - 158) : 0.0f;
+  if (lane == 0) alpha[grp] = a;
+  uint32_t bits = 0;
+  if (bk) {
+#pragma unroll
+    for (int e = 0; e < E; ++e)
+      if (mag[e] >= tau) bits |= ((__float_as_uint(v[e]) >> 31) ? 3u : 1u) << (2 * e);
+  }
+  bits <<= 2 * E * (lane % L);
+#pragma unroll
+  for (int o = 1; o < L; o <<= 1) bits |= __shfl_xor_sync(FULL_MASK, bits, o);
+  if (lane % L == 0) codes[(int64_t)m * wrow + g * (G / 16) + lane / L] = bits;
+}
+
+// One warp per group for G in {32, 64, 128}.
 template <int G>
 __global__ void __launch_bounds__(256) ternarize_warp_kernel(const float* __restrict__ w, int M, int Kred,
                                                              int ng, int wrow, uint32_t* __restrict__ codes,
                                                              float* __restrict__ alpha, unsigned int* err) {
-  constexpr int E = G / 32;
-  constexpr int L = 16 / E;  // lanes per code word
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int64_t total = (int64_t)M * ng;
-  for (int64_t grp = warp0; grp < total; grp += nwarps) {
-    const int m = (int)(grp / ng);
-    const int g = (int)(grp - (int64_t)m * ng);
-    const float* row = w + (int64_t)m * Kred;
-    const int k0 = g * G + lane * E;
-    float v[E];
-    uint32_t mag[E], s[E];
-    bool bad = false;
-#pragma unroll
-    for (int e = 0; e < E; ++e) {
-      v[e] = (k0 + e < Kred) ? __ldg(row + k0 + e) : 0.0f;
-      mag[e] = __float_as_uint(v[e]) & 0x7fffffffu;
-      bad |= mag[e] >= 0x7f800000u;
-      s[e] = mag[e];
-    }
-    if (__any_sync(FULL_MASK, bad)) {
-      if (lane == 0) {
-        record_error(err, FGQ_ERR_NONFINITE);
-        alpha[grp] = 0.0f;
-      }
-      if (lane < G / 16) codes[(int64_t)m * wrow + g * (G / 16) + lane] = 0;
-      continue;
-    }
-    // bitonic sort of the G magnitudes across the warp, descending
-#pragma unroll
-    for (int size = 2; size <= G; size <<= 1) {
-#pragma unroll
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        if (stride >= E) {
-#pragma unroll
-          for (int e = 0; e < E; ++e) {
-            const int i = lane * E + e;
-            const uint32_t p = __shfl_xor_sync(FULL_MASK, s[e], stride / E);
-            const bool lower = (i & stride) == 0;
-            const bool desc = (i & size) == 0;
-            const uint32_t mx = s[e] > p ? s[e] : p, mn = s[e] > p ? p : s[e];
-            s[e] = (lower == desc) ? mx : mn;
-          }
-        } else {
-#pragma unroll
-          for (int e = 0; e < E; ++e) {
-            if ((e & stride) == 0) {
-              const int i = lane * E + e;
-              const bool desc = (i & size) == 0;
-              const int e2 = (e + stride) < E ? e + stride : e;
-              const uint32_t a = s[e], b = s[e2];
-              const uint32_t mx = a > b ? a : b, mn = a > b ? b : a;
-              s[e] = desc ? mx : mn;
-              s[e2] = desc ? mn : mx;
-            }
-          }
-        }
-      }
-    }
-    const uint32_t mmax = __shfl_sync(FULL_MASK, s[0], 0);
-    uint32_t bk = 0, tau = 0;
-    uint64_t bS = 0;
-    int F = 1;
-    if (mmax != 0) {
-      F = max((int)(mmax >> 23), 1);
-      uint64_t pre[E];
-      uint64_t run = 0;
-#pragma unroll
-      for (int e = 0; e < E; ++e) {
-        run += fixed_of(s[e], F);
-        pre[e] = run;
-      }
-      uint64_t incl = run;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint64_t n = __shfl_up_sync(FULL_MASK, incl, o);
-        if (lane >= o) incl += n;
-      }
-      const uint64_t excl = incl - run;
-      const uint32_t next_first = __shfl_down_sync(FULL_MASK, s[0], 1);
-#pragma unroll
-      for (int e = 0; e < E; ++e) {
-        const int i = lane * E + e;
-        const uint32_t nxt = (e + 1 < E) ? s[(e + 1) < E ? e + 1 : e] : next_first;
-        const bool run_end = (i == G - 1) || (nxt < s[e]);
-        if (run_end && in_window(s[e], F)) {
-          const uint64_t S = excl + pre[e];
-          if (bk == 0 || j_greater(S, (uint32_t)(i + 1), bS, bk)) {
-            bS = S;
-            bk = (uint32_t)(i + 1);
-            tau = s[e];
-          }
-        }
-      }
-      // warp argmax of the objective; equal objectives keep the smaller kept count
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const uint64_t oS = __shfl_xor_sync(FULL_MASK, bS, o);
-        const uint32_t ok = __shfl_xor_sync(FULL_MASK, bk, o);
-        const uint32_t ot = __shfl_xor_sync(FULL_MASK, tau, o);
-        bool take;
-        if (ok == 0) take = false;
-        else if (bk == 0) take = true;
-        else if (j_greater(oS, ok, bS, bk)) take = true;
-        else if (j_greater(bS, bk, oS, ok)) take = false;
-        else take = ok < bk;
-        if (take) {
-          bS = oS;
-          bk = ok;
-          tau = ot;
-        }
-      }
-    }
-    const float a = bk ? round_ratio_f32(bS, bk, F - 158) : 0.0f;
-    if (lane == 0) alpha[grp] = a;
-    uint32_t bits = 0;
-    if (bk) {
-#pragma unroll
-      for (int e = 0; e < E; ++e)
-        if (mag[e] >= tau) bits |= ((__float_as_uint(v[e]) >> 31) ? 3u : 1u) << (2 * e);
-    }
-    bits <<= 2 * E * (lane % L);
-#pragma unroll
-    for (int o = 1; o < L; o <<= 1) bits |= __shfl_xor_sync(FULL_MASK, bits, o);
-    if (lane % L == 0) codes[(int64_t)m * wrow + g * (G / 16) + lane / L] = bits;
+  for (int64_t grp = warp0; grp < total; grp += nwarps) warp_group<G>(w, Kred, ng, wrow, codes, alpha, err, grp, lane);
+}
+
+// Many layers of one group size in one launch (fgq_ternarize_batch): work items (units of
+// the thread-per-group kernel, groups of the warp-per-group kernel) are numbered across the
+// layers; item i belongs to the last layer whose first item is <= i.
+struct TernLayer {
+  const float* w;
+  uint32_t* codes;
+  float* alpha;
+  int64_t first;          // first work item of the layer
+  int64_t units_per_row;  // thread-per-group kernel only
+  int Kred, ng, wrow, vec4;
+};
+struct TernBatch {
+  TernLayer l[FGQ_TERNARIZE_BATCH_MAX];
+  int n;
+  int64_t total;
+};
+
+__device__ __forceinline__ int batch_layer(const TernBatch& b, int64_t i) {
+  int lo = 0, hi = b.n - 1;
+  while (lo < hi) {  // largest l with first <= i
+    const int mid = (lo + hi + 1) >> 1;
+    if (b.l[mid].first <= i) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <int G>
+__global__ void __launch_bounds__(256) ternarize_small_batch_kernel(const __grid_constant__ TernBatch b,
+                                                                    unsigned int* err) {
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < b.total; u += (int64_t)gridDim.x * blockDim.x) {
+    const TernLayer& L = b.l[batch_layer(b, u)];
+    small_unit<G>(L.w, L.Kred, L.ng, L.wrow, reinterpret_cast<uint8_t*>(L.codes), L.alpha, err, L.vec4,
+                  L.units_per_row, u - L.first);
+  }
+}
+
+template <int G>
+__global__ void __launch_bounds__(256) ternarize_warp_batch_kernel(const __grid_constant__ TernBatch b,
+                                                                   unsigned int* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t grp = warp0; grp < b.total; grp += nwarps) {
+    const TernLayer& L = b.l[batch_layer(b, grp)];
+    warp_group<G>(L.w, L.Kred, L.ng, L.wrow, L.codes, L.alpha, err, grp - L.first, lane);
   }
 }
 
@@ -411,6 +476,44 @@ fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* co
     case 32: ternarize_warp_kernel<32><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
     case 64: ternarize_warp_kernel<64><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
     case 128: ternarize_warp_kernel<128><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
+    default: return FGQ_ERR_ARG;
+  }
+  return after_launch();
+}
+
+fgq_status launch_ternarize_batch(int n, const float* const* w, const int* M, const int* Kred, int G,
+                                  uint32_t* const* codes, float* const* alpha, unsigned int* err, cudaStream_t s) {
+  if (n > FGQ_TERNARIZE_BATCH_MAX) return FGQ_ERR_ARG;
+  TernBatch b;
+  memset(&b, 0, sizeof b);
+  const int64_t unit = G < 4 ? 4 : G;
+  int64_t total = 0;
+  for (int i = 0; i < n; ++i) {
+    if ((int64_t)M[i] * Kred[i] == 0) continue;  // nothing to do for an empty layer
+    TernLayer& L = b.l[b.n++];
+    L.w = w[i];
+    L.codes = codes[i];
+    L.alpha = alpha[i];
+    L.Kred = Kred[i];
+    L.ng = (Kred[i] + G - 1) / G;
+    L.wrow = (L.ng * G + 15) / 16;
+    L.vec4 = (Kred[i] % 4 == 0) && ((reinterpret_cast<uintptr_t>(w[i]) & 15) == 0);
+    L.units_per_row = (L.ng * (int64_t)G + unit - 1) / unit;
+    L.first = total;
+    total += G >= 32 ? (int64_t)M[i] * L.ng : (int64_t)M[i] * L.units_per_row;
+  }
+  b.total = total;
+  if (total == 0) return FGQ_OK;
+  const int threads = 256;
+  switch (G) {
+    case 1: ternarize_small_batch_kernel<1><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
+    case 2: ternarize_small_batch_kernel<2><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
+    case 4: ternarize_small_batch_kernel<4><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
+    case 8: ternarize_small_batch_kernel<8><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
+    case 16: ternarize_small_batch_kernel<16><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
+    case 32: ternarize_warp_batch_kernel<32><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
+    case 64: ternarize_warp_batch_kernel<64><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
+    case 128: ternarize_warp_batch_kernel<128><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
     default: return FGQ_ERR_ARG;
   }
   return after_launch();

@@ -32,6 +32,7 @@ SIGNATURES = [
     ("fgq_codes_words_per_row", _i64, [_i, _i]),
     ("fgq_num_groups", _i64, [_i, _i]),
     ("fgq_ternarize", _i, [_vp, _i, _i, _i, _vp, _vp, _vp]),
+    ("fgq_ternarize_batch", _i, [_i, _vp, _vp, _vp, _i, _vp, _vp, _vp]),
     ("fgq_ternarize_threshold_workspace_bytes", _sz, []),
     ("fgq_ternarize_threshold", _i, [_vp, _i, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp, _vp]),
     ("fgq_ternary_error", _i, [_vp, _i, _i, _i, _vp, _vp, _vp, _vp]),
@@ -150,6 +151,27 @@ def fgq_ternarize(w: torch.Tensor, G: int, codes: Optional[torch.Tensor] = None,
 
 
 RULE_EXP, RULE_GAUSS = 0, 1
+
+
+def fgq_ternarize_batch(ws, G: int, stream=None):
+    """fgq_ternarize of every fp32 [M][Kred] tensor in ws (one group size, one launch) ->
+    list of (codes, alpha)."""
+    _require_cuda()
+    n = len(ws)
+    outs = []
+    for w in ws:
+        M, Kred = w.shape
+        codes = torch.empty((M, codes_words_per_row(Kred, G)), dtype=torch.int32, device=w.device)
+        alpha = torch.empty((M, num_groups(Kred, G)), dtype=torch.float32, device=w.device)
+        outs.append((codes, alpha))
+    VP, I = ctypes.c_void_p * max(n, 1), ctypes.c_int * max(n, 1)
+    tw = VP(*[_dev(w, torch.float32, "w") for w in ws])
+    tm = I(*[int(w.shape[0]) for w in ws])
+    tk = I(*[int(w.shape[1]) for w in ws])
+    tc = VP(*[c.data_ptr() for c, _ in outs])
+    ta = VP(*[a.data_ptr() for _, a in outs])
+    _check(lib().fgq_ternarize_batch(n, tw, tm, tk, G, tc, ta, _stream(stream)), "fgq_ternarize_batch")
+    return outs
 
 
 def fgq_ternarize_threshold(w: torch.Tensor, G: int, rule: int, per_layer: bool = False, stream=None):

@@ -62,6 +62,34 @@ def test_ternarize_resnet50_weight_set(G):
         assert np.array_equal(ga.cpu().numpy(), al), layer.name
 
 
+@pytest.mark.parametrize("G", [1, 2, 4, 8, 16, 32, 64, 128])
+def test_ternarize_batch_bit_exact(G):
+    """fgq_ternarize_batch over several layers in one launch: every set bit-exact against the
+    oracle (ResNet-50 layers, a row length not a multiple of 4, an empty set, one filter)."""
+    rng = np.random.default_rng(G)
+    ws = [synth.weights(l, synth.layer_seed(i)) for i, l in enumerate(synth.resnet50_convs()[1:6], start=1)]
+    ws += [rng.standard_normal((3, 7)).astype(np.float32), np.zeros((0, 10), np.float32),
+           rng.standard_normal((1, 1001)).astype(np.float32), rng.standard_normal((40, 130)).astype(np.float32)]
+    outs = fgq.fgq_ternarize_batch([to_dev(w) for w in ws], G)
+    for w, (codes, alpha) in zip(ws, outs):
+        if w.size == 0:
+            continue
+        t, al, _ = O.ternarize(w, G)
+        assert np.array_equal(codes.cpu().numpy().view(np.uint32), O.pack_codes(t)), (G, w.shape)
+        assert np.array_equal(alpha.cpu().numpy(), al), (G, w.shape)
+
+
+def test_ternarize_batch_args():
+    w = torch.zeros((4, 16), dtype=torch.float32, device=dev())
+    with pytest.raises(fgq.FGQError) as e:  # more sets than one call takes
+        fgq.fgq_ternarize_batch([w] * 129, 4)
+    assert e.value.code == fgq.FGQ_ERR_ARG
+    with pytest.raises(fgq.FGQError) as e:  # bad group size
+        fgq.fgq_ternarize_batch([w], 5)
+    assert e.value.code == fgq.FGQ_ERR_ARG
+    assert fgq.fgq_ternarize_batch([], 4) == []
+
+
 def test_ternarize_nonfinite_status():
     w = np.ones((4, 64), np.float32)
     w[1, 5] = np.nan
