@@ -17,8 +17,9 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfgq.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-SOURCES = ["api.cu", "ternarize.cu", "ternarize_threshold.cu", "quantize.cu", "gemm_simt.cu", "gemm_tc.cu",
-           "gemm_tc4.cu", "gemm_dense.cu", "gemv.cu", "elementwise.cu"]
+SOURCES = ["api.cu", "ternarize.cu", "ternarize_threshold.cu", "quantize.cu", "gemm_simt.cu", "gemm_simt_g4.cu",
+           "gemm_simt_g8.cu", "gemm_simt_g32.cu", "gemm_simt_g128.cu", "gemm_tc.cu", "gemm_tc4.cu", "gemm_dense.cu",
+           "gemv.cu", "elementwise.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
               "--expt-relaxed-constexpr", "-I" + INCLUDE]
