@@ -328,7 +328,7 @@ def _oracle_inputs(layers):
     """Seeded inputs for the CPU sample, prepared once outside the timed oracle work: each
     conv layer's weights ternarized by the oracle at G = 4 and G = 64, and one input image
     quantized by the oracle (ternarization is an offline step in the paper, Section 4; in the
-    GPU step it is under 1% of the work)."""
+    GPU step it is about 5% of the work)."""
     import oracle as O
     from paper_1705_01462_gb300 import synth
     if not _ORACLE_INPUTS:
