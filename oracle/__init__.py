@@ -73,6 +73,8 @@ def lib() -> ctypes.CDLL:
         L.oracle_quantize_alpha.argtypes = [_P(c_f), c_i, c_i, c_i, _P(ctypes.c_int32), _P(c_f)]
         L.oracle_group_sums.argtypes = [_P(ctypes.c_int32), c_i, c_i, _P(ctypes.c_int8), c_i, c_i,
                                         _P(ctypes.c_int64)]
+        L.oracle_conv2d_group_sums.argtypes = [_P(ctypes.c_int32)] + [c_i] * 9 + [_P(ctypes.c_int8), c_i, c_i,
+                                                                               _P(c_i64), c_i64, _P(c_i64)]
         _lib = L
     return _lib
 
@@ -312,6 +314,25 @@ def group_sums(q, t, G):
     s = np.zeros((M, ng, P), dtype=np.int64)
     _check(lib().oracle_group_sums(_ptr(q, ctypes.c_int32), P, Kred, _ptr(t, ctypes.c_int8), M, G,
                                    _ptr(s, ctypes.c_int64)), "group_sums")
+    return s
+
+
+def conv2d_group_sums(q, R, S, stride, pad, groups, t, G, positions=None):
+    """Group sums of a convolution: q int32 NHWC codes [B][H][W][C]; t [M][Kp]; positions
+    (flat output indices, default all) -> int64 [M][ng][npos]."""
+    q = np.ascontiguousarray(q, dtype=np.int32)
+    t = np.ascontiguousarray(t, dtype=np.int8)
+    B, H, W, C = q.shape
+    M = t.shape[0]
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    if positions is None:
+        positions = np.arange(B * Ho * Wo)
+    pos = np.ascontiguousarray(positions, dtype=np.int64)
+    ng = num_groups(R * S * (C // groups), G)
+    s = np.zeros((M, ng, pos.size), dtype=np.int64)
+    _check(lib().oracle_conv2d_group_sums(_ptr(q, ctypes.c_int32), B, H, W, C, R, S, stride, pad, groups,
+                                          _ptr(t, ctypes.c_int8), M, G, _ptr(pos, ctypes.c_int64), pos.size,
+                                          _ptr(s, ctypes.c_int64)), "conv2d_group_sums")
     return s
 
 

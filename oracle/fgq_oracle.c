@@ -23,6 +23,7 @@
  *   oracle_conv2d_at            the same at a list of output positions
  *   oracle_gemm                 grouped contraction for a [P][Kred] activation matrix
  *   oracle_group_sums           the int32-accumulator group sums s[m][g][p]
+ *   oracle_conv2d_group_sums    the same sums of a convolution, at listed output positions
  *   oracle_conv2d_w8            dense 8-bit-weight convolution (first layer, Section 4)
  *   oracle_ternarize_threshold  ternarization at an analytical threshold (Section 3, Lemma 1),
  *                               per group or with one threshold and one alpha per layer
@@ -525,6 +526,46 @@ int oracle_group_sums(const int32_t* q, int P, int Kred, const int8_t* t, int M,
           acc += (int64_t)t[(size_t)m * Kp + j] * q[(size_t)p * Kred + j];
         s[((size_t)m * ng + g) * P + p] = acc;
       }
+  return ORACLE_OK;
+}
+
+/*
+ * Group sums of a convolution (the 32-bit accumulators of Section 4 inside Eq. 2) at npos
+ * listed flat output positions p = (b*Ho + ho)*Wo + wo: for filter m of conv group gi and
+ * group g of its reduction vector, s[m][g][i] = sum_{j in g} t[m][j] * col[j] with col the
+ * im2col column of position pos[i] for conv group gi.  q NHWC codes [B][H][W][C]; t
+ * [M][Kp]; s int64 [M][ng][npos].
+ */
+int oracle_conv2d_group_sums(const int32_t* q, int B, int H, int W, int C, int R, int S,
+                             int stride, int pad, int groups, const int8_t* t, int M, int G,
+                             const int64_t* pos, int64_t npos, int64_t* s) {
+  int Ho, Wo, Cg, Kred, Kp, ng, gi, m, g, j;
+  int64_t i;
+  int64_t* col;
+  int st = conv_geometry(H, W, C, R, S, stride, pad, groups, M, G, &Ho, &Wo, &Cg, &Kred,
+                         &Kp, &ng);
+  if (st != ORACLE_OK || B <= 0 || npos < 0) return ORACLE_ERR_ARG;
+  col = (int64_t*)malloc(sizeof(int64_t) * (size_t)Kp);
+  if (!col) return ORACLE_ERR_ARG;
+  for (i = 0; i < npos; i++) {
+    int64_t p = pos[i];
+    int wo = (int)(p % Wo), ho = (int)((p / Wo) % Ho), b = (int)(p / ((int64_t)Wo * Ho));
+    int Mg = M / groups;
+    if (p < 0 || b >= B) {
+      free(col);
+      return ORACLE_ERR_ARG;
+    }
+    for (gi = 0; gi < groups; gi++) {
+      im2col_column(q, H, W, C, R, S, stride, pad, Cg, gi, b, ho, wo, Kp, col);
+      for (m = gi * Mg; m < (gi + 1) * Mg; m++)
+        for (g = 0; g < ng; g++) {
+          int64_t acc = 0;
+          for (j = g * G; j < (g + 1) * G; j++) acc += (int64_t)t[(size_t)m * Kp + j] * col[j];
+          s[((size_t)m * ng + g) * (size_t)npos + (size_t)i] = acc;
+        }
+    }
+  }
+  free(col);
   return ORACLE_OK;
 }
 

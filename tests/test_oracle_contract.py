@@ -122,3 +122,42 @@ def test_codes_worked_examples():
     for ts, ws, why in read_golden("codes_worked.txt", 3):
         t = np.array([parse_ints(ts)], np.int8)
         assert list(O.pack_codes(t)[0]) == parse_ints(ws), why
+
+
+@pytest.mark.parametrize("B,H,W,C,M,R,stride,pad,groups,G", [
+    (2, 6, 5, 8, 6, 3, 1, 1, 1, 4),     # groups of 4 channels at one tap
+    (1, 7, 7, 3, 4, 3, 2, 1, 1, 4),     # C = 3: groups straddle taps
+    (2, 9, 8, 16, 6, 3, 2, 0, 2, 8),    # two conv groups, stride 2, no padding
+    (1, 5, 5, 64, 3, 3, 1, 1, 1, 64),   # G = 64: one group per tap
+    (1, 4, 4, 6, 2, 1, 1, 0, 1, 128),   # one group longer than Kred (zero padding)
+])
+def test_conv_group_sums_match_torch_conv(B, H, W, C, M, R, stride, pad, groups, G):
+    """oracle.conv2d_group_sums[m][g] equals a float64 torch convolution whose weights keep
+    only group g's codes of filter m (every other code zeroed): the group decomposition of
+    Eq. 2 read off a library convolution, including the (r, s, c) order, padding, stride and
+    conv groups."""
+    rng = np.random.default_rng(11)
+    Cg = C // groups
+    Kred = R * R * Cg
+    ng = O.num_groups(Kred, G)
+    Kp = ng * G
+    t = rng.integers(-1, 2, (M, Kp)).astype(np.int8)
+    t[:, Kred:] = 0
+    q = rng.integers(0, 256, (B, H, W, C)).astype(np.int32)
+    s = O.conv2d_group_sums(q, R, R, stride, pad, groups, t, G)
+    Ho, Wo = O.conv_out_hw(H, W, R, R, stride, pad)
+    x = torch.from_numpy(q.transpose(0, 3, 1, 2).astype(np.float64))
+    for g in range(ng):
+        tm = np.zeros_like(t)
+        tm[:, g * G:(g + 1) * G] = t[:, g * G:(g + 1) * G]
+        wt = tm[:, :Kred].astype(np.float64).reshape(M, R, R, Cg).transpose(0, 3, 1, 2)
+        ref = torch.nn.functional.conv2d(x, torch.from_numpy(np.ascontiguousarray(wt)), stride=stride,
+                                         padding=pad, groups=groups).numpy()
+        ref = ref.transpose(1, 0, 2, 3).reshape(M, B * Ho * Wo)
+        assert np.array_equal(s[:, g, :], ref.astype(np.int64)), f"group {g}"
+    # listed positions return the same columns
+    pos = rng.choice(B * Ho * Wo, size=min(5, B * Ho * Wo), replace=False)
+    assert np.array_equal(O.conv2d_group_sums(q, R, R, stride, pad, groups, t, G, positions=pos), s[:, :, pos])
+    # a 1x1 stride-1 convolution is the GEMM of the group sums
+    if R == 1 and stride == 1 and pad == 0 and groups == 1:
+        assert np.array_equal(s, O.group_sums(q.reshape(-1, C), t, G))
