@@ -63,33 +63,6 @@ typedef enum {
 
 typedef enum { FGQ_U8 = 0, FGQ_S8 = 1, FGQ_U4 = 2, FGQ_S4 = 3 } fgq_act_type;
 
-/* Contraction kernel families (see fgq_set_path / fgq_last_path). */
-typedef enum {
-  FGQ_PATH_AUTO = 0,   /* choose per shape: the few-row path for small GEMMs; with
-                          fixed-point alphas the dense tensor-core path where it applies;
-                          else the tensor cores where the shape is covered (G = 4 only with
-                          at least 128 filters per conv group), else the CUDA cores */
-  FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
-  FGQ_PATH_TC = 2,     /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
-                          the group; G = 4 with a block-diagonal activation operand
-                          (Cg a multiple of 64) */
-  FGQ_PATH_GEMV = 3,   /* few-row path for GEMMs with P <= 8 (8-bit activations, Kred a
-                          multiple of 16, G >= 4): one warp per filter row streams the
-                          weights once; the automatic choice for such calls */
-  FGQ_PATH_DENSE = 4   /* dense tensor-core path (tcgen05, any G, 8-bit activations, Cg a
-                          multiple of 64): the alphas are folded into fp16 weights
-                          alpha(m, k / G) * t[m][k] built per call, and one dense
-                          contraction replaces the per-group multiplies.  Fixed-point alphas
-                          fold exactly (integer weights |a t| <= 255; the result is the exact
-                          value rounded once while |sum a t q| < 2^24): the automatic choice
-                          for fgq_gemm_qa / fgq_conv2d_qa.  fp32 alphas (only when forced)
-                          are split per filter row into two fp16 parts after scaling the
-                          row's largest alpha into [2^14, 2^15), about 22 bits of alpha, and
-                          the fp32 accumulator rounds once per 16 reduction elements: a
-                          numerical ablation of folding, outside the fgq_gemm tolerance
-                          guarantee. */
-} fgq_path;
-
 /* ABI version of this header (incremented on any signature change). */
 int fgq_version(void);
 
@@ -380,29 +353,66 @@ fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_sc
                          cudaStream_t stream);
 
 /*
+ * One convolution layer end to end from HOST buffers (the inference pipeline of Section 4:
+ * fp32 weights are ternarized per group of G (Eq. 5), the fp32 input is quantized to
+ * dynamic fixed point, the grouped contraction runs, the fp32 output comes back):
+ *   h_w    host fp32 weights [M][Kred] (Kred in (r, s, c) order).
+ *   h_x    host fp32 activations NHWC [B][H][W][C].
+ *   type   activation type of the quantized input (scale derived as fgq_quantize_act does).
+ *   G      group size as fgq_ternarize; G = 0 selects the 8-bit-weight first layer instead
+ *          (fgq_quantize_weights_w8 + fgq_conv2d_w8; 8-bit activation types only).
+ *   h_out  host fp32 output NHWC [B][Ho][Wo][M].
+ *   workspace  device buffer of fgq_conv2d_host_workspace_bytes(...) bytes, 256-byte
+ *          aligned, owned by the caller (it holds the device copies, codes, alphas,
+ *          quantized input and output).
+ * Issues, in order on `stream`: one cudaMemcpyAsync per input buffer (weights, then
+ * activations), the kernels of fgq_ternarize (or fgq_quantize_weights_w8), fgq_quantize_act
+ * and fgq_conv2d (or fgq_conv2d_w8), and one cudaMemcpyAsync of the output back.  The call
+ * is asynchronous: h_out is valid once the stream has completed; host buffers should be
+ * page-locked (cudaHostAlloc) for the copies to overlap other work.  Calls on different
+ * streams need workspaces of their own.  The contraction tolerance is fgq_conv2d's.
+ * Errors: those of the calls it makes; FGQ_ERR_ARG (null pointer, workspace too small),
+ * FGQ_ERR_ALIGN (workspace), FGQ_ERR_CUDA (a copy could not be issued).
+ */
+size_t fgq_conv2d_host_workspace_bytes(fgq_act_type type, int B, int H, int W, int C, int R, int S,
+                                       int stride, int pad, int groups, int M, int G);
+fgq_status fgq_conv2d_host(const float* h_w, const float* h_x, fgq_act_type type, int B, int H, int W,
+                           int C, int R, int S, int stride, int pad, int groups, int M, int G,
+                           float* h_out, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * The 32-bit group accumulators themselves (Section 4), for verification:
  *   s[m][g][p] = sum_{j in g, j < Kred} t[m][j] * q[p][j],  int32 [M][ng][P].
- * q as in fgq_gemm.  Always computed by the CUDA-core (dp4a) kernel family, whatever
- * fgq_set_path selects.  Errors as fgq_gemm.
+ * q as in fgq_gemm.  Computed by the kernel family the fp32-output call of the same shape
+ * uses (the automatic choice, or the family fgq_set_path forces, see fgq_debug.h): the
+ * tensor-core kernels store each group's TMEM accumulator (an exact integer in fp32) as
+ * int32, the CUDA-core kernel its dp4a sums.  The dense and few-row paths form no group
+ * sums; where the automatic choice would take one of them the dp4a kernel runs, and
+ * forcing either returns FGQ_ERR_UNSUPPORTED.  Errors as fgq_gemm.
  */
 fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred,
                           const uint32_t* codes, int M, int G, int32_t* s, cudaStream_t stream);
 
 /*
- * Synchronizes the stream, then returns (and clears) the first error a kernel recorded
- * since the last call (FGQ_OK if none), or FGQ_ERR_CUDA if the synchronization failed.
+ * The group sums of a convolution (Section 3.2 grouping, Eq. 2, Section 4 accumulators):
+ *   s[m][g][p] = sum_{j in g, j < Kred} t[m][j] * col_p[j],  int32 [M][ng][P],
+ * col_p the im2col column of output position p = (b * Ho + ho) * Wo + wo for filter m's
+ * conv group, as in fgq_conv2d.  Kernel family and errors as fgq_group_sums and
+ * fgq_conv2d.
  */
-fgq_status fgq_stream_status(cudaStream_t stream);
+fgq_status fgq_conv2d_group_sums(const void* act, fgq_act_type type, int B, int H, int W, int C, int R,
+                                 int S, int stride, int pad, int groups, const uint32_t* codes, int M,
+                                 int G, int32_t* s, cudaStream_t stream);
 
 /*
- * Restricts contraction calls to one kernel family (FGQ_PATH_AUTO restores the default
- * per-shape choice).  A forced path that cannot run a shape makes the call return
- * FGQ_ERR_UNSUPPORTED.  Process-wide; returns the previous setting.
+ * Returns (and clears) the first error a kernel recorded on the current device since the
+ * last call (FGQ_OK if none), or FGQ_ERR_CUDA if a CUDA call failed.  The error word is one
+ * per device and shared by every stream: the call reads and clears it in one atomic step,
+ * in order on `stream`, and synchronizes `stream` before it returns, so it covers every
+ * kernel on `stream` and any kernel on another stream that recorded its error before the
+ * read.  Synchronize the device first to cover the kernels of all streams.
  */
-int fgq_set_path(int path);
-
-/* The kernel family (fgq_path) the most recent contraction call on this host thread used. */
-int fgq_last_path(void);
+fgq_status fgq_stream_status(cudaStream_t stream);
 
 /* Number of kernels this library has launched in this process (all calls, all threads). */
 uint64_t fgq_launch_count(void);

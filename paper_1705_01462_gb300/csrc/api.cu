@@ -11,13 +11,19 @@ namespace fgq {
 namespace {
 
 __device__ unsigned int g_error_word;
+constexpr int kReadSlots = 64;
+__device__ unsigned int g_error_read[kReadSlots];  // the word's value at a read-and-clear, per call
+std::atomic<unsigned int> g_read_slot{0};
 
 constexpr int kMaxDevices = 64;
 unsigned int* g_err_ptr[kMaxDevices];
 std::mutex g_err_mu;
 std::atomic<uint64_t> g_launches{0};
-std::atomic<int> g_path{FGQ_PATH_AUTO};
+// test and benchmark controls (fgq_debug.h), each per host thread
+thread_local int t_path = FGQ_PATH_AUTO;
 thread_local int t_last_path = FGQ_PATH_AUTO;
+thread_local int64_t t_wait_limit_us = -1;
+thread_local int t_split_fold = 0;
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
@@ -62,12 +68,22 @@ bool tc_any(const Geom& g) { return g.G == 4 ? tc4_supports(g) : tc_supports(g);
 bool gemv_any(const Geom& g) { return !g.is_conv && gemv_supports((int)g.P, g.Kred, g.G, g.act_type); }
 
 int choose_path(const Geom& g, bool sums, bool qa) {
-  const int forced = g_path.load();
-  if (sums) return FGQ_PATH_SIMT;  // the int32 group sums are read from the CUDA-core kernel
+  const int forced = t_path;
+  if (sums) {
+    // the group sums come from the kernel family the output call of this shape would use;
+    // the dense and few-row paths form no group sums
+    if (forced == FGQ_PATH_GEMV || forced == FGQ_PATH_DENSE) return -1;
+    if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
+    if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
+    if (g.G == 4 && g.Mg < 128) return FGQ_PATH_SIMT;
+    return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
+  }
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
   if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
   if (forced == FGQ_PATH_GEMV) return gemv_any(g) ? FGQ_PATH_GEMV : -1;
-  if (forced == FGQ_PATH_DENSE) return dense_supports(g) ? FGQ_PATH_DENSE : -1;
+  // fp32 alphas fold only approximately (split into two fp16 parts): an ablation outside the
+  // tolerance guarantee, run only when a test or benchmark asked for it
+  if (forced == FGQ_PATH_DENSE) return dense_supports(g) && (qa || t_split_fold) ? FGQ_PATH_DENSE : -1;
   if (gemv_any(g)) return FGQ_PATH_GEMV;  // a few activation rows: stream the weights once
   // fixed-point alphas fold exactly into fp16 weights: one dense tensor-core contraction
   if (qa && dense_supports(g)) return FGQ_PATH_DENSE;
@@ -114,7 +130,7 @@ fgq_status contract(const void* act, const Geom& g, const uint32_t* codes, const
   }
   fgq_status st;
   if (path == FGQ_PATH_TC)
-    st = g.G == 4 ? launch_tc4_contract(act, g, codes, alpha, act_scale, out, err, s)
+    st = g.G == 4 ? launch_tc4_contract(act, g, codes, alpha, act_scale, out, sums, err, s)
                   : launch_tc_contract(act, g, codes, alpha, act_scale, out, sums, err, s);
   else
     st = launch_simt_contract(act, g, codes, alpha, 0, act_scale, out, sums, s);
@@ -162,6 +178,63 @@ fgq_status after_launch() {
   return cudaGetLastError() == cudaSuccess ? FGQ_OK : FGQ_ERR_CUDA;
 }
 
+int64_t debug_wait_limit_us() { return t_wait_limit_us; }
+
+namespace {
+
+// Reads and clears the error word in one atomic step, so that an error a kernel on another
+// stream records concurrently is either returned now or kept for the next read.
+__global__ void error_read_clear_kernel(unsigned int slot) { g_error_read[slot] = atomicExch(&g_error_word, 0u); }
+
+}  // namespace
+
+}  // namespace fgq
+
+namespace fgq {
+namespace {
+
+// Byte offsets of the regions of fgq_conv2d_host's workspace (each 256-byte aligned).
+struct HostLayout {
+  size_t w, x, codes, alpha, q, scale, qws, out, total, qws_bytes;
+};
+
+size_t up256(size_t v) { return (v + 255) & ~size_t(255); }
+
+HostLayout host_layout(const Geom& g) {
+  HostLayout L;
+  const size_t n = (size_t)g.B * g.H * g.W * g.C;
+  const bool w8 = g.G == 0;
+  size_t o = 0;
+  L.w = o;     o = up256(o + sizeof(float) * (size_t)g.M * g.Kred);
+  L.x = o;     o = up256(o + sizeof(float) * n);
+  L.codes = o; o = up256(o + (w8 ? (size_t)g.M * g.Kred : sizeof(uint32_t) * (size_t)g.M * g.wrow));
+  L.alpha = o; o = up256(o + sizeof(float) * (size_t)g.M * (w8 ? 1 : g.ng));
+  L.q = o;     o = up256(o + (is4(g.act_type) ? (n + 1) / 2 : n));
+  L.scale = o; o = up256(o + sizeof(float));
+  L.qws_bytes = quantize_workspace_bytes(n);
+  L.qws = o;   o = up256(o + L.qws_bytes);
+  L.out = o;   o = up256(o + sizeof(float) * (size_t)g.P * g.M);
+  L.total = o;
+  return L;
+}
+
+// Geometry of a host call (G == 0: the 8-bit-weight layer, 8-bit activations only).
+fgq_status host_geom(fgq_act_type type, int B, int H, int W, int C, int R, int S, int stride, int pad, int groups,
+                     int M, int G, Geom& g) {
+  if (G != 0 && !valid_G(G)) return FGQ_ERR_ARG;
+  if (G == 0 && type != FGQ_U8 && type != FGQ_S8) return FGQ_ERR_ARG;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G == 0 ? 1 : G, 1, g);
+  if (st != FGQ_OK) return st;
+  if (G == 0) {  // dense 8-bit weights: no groups
+    g.G = 0;
+    g.ng = 1;
+    g.Kp = g.Kred;
+    g.wrow = 0;
+  }
+  return FGQ_OK;
+}
+
+}  // namespace
 }  // namespace fgq
 
 using namespace fgq;
@@ -404,7 +477,7 @@ fgq_status fgq_conv2d_w8(const void* act, fgq_act_type type, const float* act_sc
   if (!act || !act_scale || !wq || !wscale || !out) return FGQ_ERR_ARG;
   if (!aligned(act, 16) || !aligned(wscale, 4) || !aligned(out, 16) || !aligned(act_scale, 4))
     return FGQ_ERR_ALIGN;
-  if (g_path.load() != FGQ_PATH_SIMT && dense_w8_supports(g)) {
+  if (t_path != FGQ_PATH_SIMT && dense_w8_supports(g)) {
     t_last_path = FGQ_PATH_DENSE;
     return launch_dense_w8(act, g, wq, wscale, act_scale, out, device_error_word(), stream);
   }
@@ -427,7 +500,7 @@ fgq_status fgq_conv2d_w8_rq(const void* act, fgq_act_type type, const float* act
   g.rq_out = static_cast<uint8_t*>(out_q);
   g.rq_scale = out_scale;
   g.rq_signed = out_type == FGQ_S8;
-  if (g_path.load() != FGQ_PATH_SIMT && dense_w8_supports(g)) {
+  if (t_path != FGQ_PATH_SIMT && dense_w8_supports(g)) {
     t_last_path = FGQ_PATH_DENSE;
     return launch_dense_w8(act, g, wq, wscale, act_scale, nullptr, device_error_word(), stream);
   }
@@ -474,16 +547,78 @@ fgq_status fgq_group_sums(const void* q, fgq_act_type type, int P, int Kred, con
   return contract(q, g, codes, nullptr, nullptr, nullptr, s, stream);
 }
 
+fgq_status fgq_conv2d_group_sums(const void* act, fgq_act_type type, int B, int H, int W, int C, int R, int S,
+                                 int stride, int pad, int groups, const uint32_t* codes, int M, int G, int32_t* s,
+                                 cudaStream_t stream) {
+  if (!valid_G(G)) return FGQ_ERR_ARG;
+  Geom g;
+  fgq_status st = make_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, 1, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!act || !codes || !s) return FGQ_ERR_ARG;
+  if (!aligned(act, 16) || !aligned(codes, 16) || !aligned(s, 4)) return FGQ_ERR_ALIGN;
+  return contract(act, g, codes, nullptr, nullptr, nullptr, s, stream);
+}
+
+size_t fgq_conv2d_host_workspace_bytes(fgq_act_type type, int B, int H, int W, int C, int R, int S, int stride,
+                                       int pad, int groups, int M, int G) {
+  Geom g;
+  if (host_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, g) != FGQ_OK) return 0;
+  return host_layout(g).total;
+}
+
+fgq_status fgq_conv2d_host(const float* h_w, const float* h_x, fgq_act_type type, int B, int H, int W, int C, int R,
+                           int S, int stride, int pad, int groups, int M, int G, float* h_out, void* workspace,
+                           size_t workspace_bytes, cudaStream_t stream) {
+  Geom g;
+  fgq_status st = host_geom(type, B, H, W, C, R, S, stride, pad, groups, M, G, g);
+  if (st != FGQ_OK) return st;
+  if (g.P == 0 || g.M == 0) return FGQ_OK;
+  if (!h_w || !h_x || !h_out || !workspace) return FGQ_ERR_ARG;
+  if (!aligned(workspace, 256)) return FGQ_ERR_ALIGN;
+  const HostLayout L = host_layout(g);
+  if (workspace_bytes < L.total) return FGQ_ERR_ARG;
+  uint8_t* base = static_cast<uint8_t*>(workspace);
+  float* w = reinterpret_cast<float*>(base + L.w);
+  float* x = reinterpret_cast<float*>(base + L.x);
+  float* alpha = reinterpret_cast<float*>(base + L.alpha);
+  float* scale = reinterpret_cast<float*>(base + L.scale);
+  float* out = reinterpret_cast<float*>(base + L.out);
+  const size_t n = (size_t)g.B * g.H * g.W * g.C;
+  // one copy per input buffer, in order on the stream
+  if (cudaMemcpyAsync(w, h_w, sizeof(float) * (size_t)g.M * g.Kred, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaMemcpyAsync(x, h_x, sizeof(float) * n, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+    return FGQ_ERR_CUDA;
+  if (G == 0)
+    st = fgq_quantize_weights_w8(w, g.M, g.Kred, reinterpret_cast<int8_t*>(base + L.codes), alpha, stream);
+  else
+    st = fgq_ternarize(w, g.M, g.Kred, G, reinterpret_cast<uint32_t*>(base + L.codes), alpha, stream);
+  if (st != FGQ_OK) return st;
+  st = fgq_quantize_act(x, n, type, 0.0f, base + L.q, scale, base + L.qws, L.qws_bytes, stream);
+  if (st != FGQ_OK) return st;
+  if (G == 0)
+    st = fgq_conv2d_w8(base + L.q, type, scale, B, H, W, C, R, S, stride, pad, groups,
+                       reinterpret_cast<const int8_t*>(base + L.codes), alpha, M, out, stream);
+  else
+    st = fgq_conv2d(base + L.q, type, scale, B, H, W, C, R, S, stride, pad, groups,
+                    reinterpret_cast<const uint32_t*>(base + L.codes), alpha, M, G, out, stream);
+  if (st != FGQ_OK) return st;
+  if (cudaMemcpyAsync(h_out, out, sizeof(float) * (size_t)g.P * g.M, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    return FGQ_ERR_CUDA;
+  return FGQ_OK;
+}
+
 fgq_status fgq_stream_status(cudaStream_t stream) {
-  if (cudaStreamSynchronize(stream) != cudaSuccess) return FGQ_ERR_CUDA;
-  unsigned int* e = device_error_word();
-  if (!e) return FGQ_ERR_CUDA;
+  if (!device_error_word()) return FGQ_ERR_CUDA;
+  // a slot of its own for each concurrent call (up to kReadSlots of them)
+  const unsigned int slot = g_read_slot.fetch_add(1u) % kReadSlots;
+  error_read_clear_kernel<<<1, 1, 0, stream>>>(slot);
+  if (cudaGetLastError() != cudaSuccess) return FGQ_ERR_CUDA;
   unsigned int v = 0;
-  if (cudaMemcpy(&v, e, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return FGQ_ERR_CUDA;
-  if (v != 0) {
-    const unsigned int zero = 0;
-    if (cudaMemcpy(e, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return FGQ_ERR_CUDA;
-  }
+  if (cudaMemcpyFromSymbolAsync(&v, g_error_read, sizeof v, sizeof v * slot, cudaMemcpyDeviceToHost, stream) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess)
+    return FGQ_ERR_CUDA;
   return (fgq_status)v;
 }
 
@@ -491,7 +626,21 @@ int fgq_set_path(int path) {
   if (path != FGQ_PATH_AUTO && path != FGQ_PATH_SIMT && path != FGQ_PATH_TC && path != FGQ_PATH_GEMV &&
       path != FGQ_PATH_DENSE)
     return -1;
-  return g_path.exchange(path);
+  const int prev = t_path;
+  t_path = path;
+  return prev;
+}
+
+int64_t fgq_debug_set_wait_limit_us(int64_t us) {
+  const int64_t prev = t_wait_limit_us;
+  t_wait_limit_us = us < 0 ? -1 : us;
+  return prev;
+}
+
+int fgq_debug_allow_split_fold(int allow) {
+  const int prev = t_split_fold;
+  t_split_fold = allow ? 1 : 0;
+  return prev;
 }
 
 int fgq_last_path(void) { return t_last_path; }

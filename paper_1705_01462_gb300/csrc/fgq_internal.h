@@ -7,6 +7,7 @@
 #include <cuda_runtime_api.h>
 
 #include "../../include/fgq.h"
+#include "../../include/fgq_debug.h"
 
 namespace fgq {
 
@@ -32,6 +33,10 @@ unsigned int* device_error_word();
 // Counts one kernel launch (for fgq_launch_count) and converts a launch error.
 fgq_status after_launch();
 
+// Wait limit, in microseconds, that a test set on this host thread for the tensor-core
+// kernels' mbarrier waits (fgq_debug_set_wait_limit_us), or -1 for the kernels' own limits.
+int64_t debug_wait_limit_us();
+
 // Kernel launchers (each returns FGQ_OK or FGQ_ERR_CUDA / FGQ_ERR_UNSUPPORTED).
 fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,
                             unsigned int* err, cudaStream_t s);
@@ -56,7 +61,8 @@ fgq_status launch_simt_contract(const void* act, const Geom& g, const void* weig
                                 const float* scales, int dense, const float* act_scale, float* out,
                                 int32_t* sums, cudaStream_t s);
 // Tensor-core contraction (tcgen05), G in {64, 128}; returns FGQ_ERR_UNSUPPORTED for shapes
-// it does not cover.
+// it does not cover.  sums != nullptr writes the int32 group sums [M][ng][P] (drained from
+// TMEM) instead of the output.
 bool tc_supports(const Geom& g);
 fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* codes,
                               const float* alpha, const float* act_scale, float* out,
@@ -64,8 +70,10 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
 
 // Tensor-core contraction for G = 4 (block-diagonal activation operand).
 bool tc4_supports(const Geom& g);
+// sums != nullptr writes the int32 group sums [M][ng][P] instead of the output.
 fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
-                               const float* act_scale, float* out, unsigned int* err, cudaStream_t s);
+                               const float* act_scale, float* out, int32_t* sums, unsigned int* err,
+                               cudaStream_t s);
 
 // Dense tensor-core contraction with the alphas folded into fp16 weights: fixed-point alphas
 // (aq, abits 8 or 4, ascale) exactly, or fp32 alphas (aq == nullptr) split into two fp16

@@ -525,13 +525,7 @@ __global__ void __launch_bounds__(TD_THREADS, 1) dense_contract_kernel(const __g
 
 template <int NA, bool SIGNED, bool TMAP>
 fgq_status launch_dense(const TDArgs& args, int grid, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(dense_contract_kernel<NA, SIGNED, TMAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             DenseCfg<NA>::SMEM) != cudaSuccess)
-      return FGQ_ERR_CUDA;
-    attr_set = true;
-  }
+  if (!tc::smem_attr_once<dense_contract_kernel<NA, SIGNED, TMAP>>(DenseCfg<NA>::SMEM)) return FGQ_ERR_CUDA;
   dense_contract_kernel<NA, SIGNED, TMAP><<<grid, TD_THREADS, DenseCfg<NA>::SMEM, s>>>(args);
   return after_launch();
 }
@@ -623,7 +617,9 @@ fgq_status run_dense(const void* act, const Geom& g, int NA, const __half* a0, c
   a.ptiles = (int)((g.P + TD_BN - 1) / TD_BN);
   a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.ktiles = g.Kred / TD_KT;
-  a.timeout_ns = TD_TIMEOUT_NS;
+  // a test may shorten the waits (debug_wait_limit_us), never the final drains
+  const int64_t lim_us = debug_wait_limit_us();
+  a.timeout_ns = lim_us < 0 ? TD_TIMEOUT_NS : (uint64_t)lim_us * 1000u;
   for (int part = 0; part < NA; ++part)
     if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, part ? (const void*)a1 : (const void*)a0,
                      (uint64_t)g.Kp, (uint64_t)g.M, (uint64_t)g.Kp * 2, TD_KT, TD_BM, CU_TENSOR_MAP_SWIZZLE_128B))

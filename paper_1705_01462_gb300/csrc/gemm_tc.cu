@@ -11,6 +11,8 @@
 // holds exactly s[m][g][p] for a 128-filter x 128-position tile; the epilogue multiplies
 // it by alpha[m][g] and adds it into an fp32 register accumulator (one multiply per group,
 // Section 4.1).  Four TMEM buffers let the MMAs of later groups run while a group drains.
+// The group-sums variant (SUMS) stores each drained accumulator as the int32 s[m][g][p]
+// instead (the exact integers themselves, for verification).
 //
 // Warp roles (416 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
@@ -63,6 +65,8 @@ constexpr int TC_MMA_WARP = TC_EPI_WARPS + TC_LOAD_WARPS;  // warp 16
 constexpr int TC_THREADS = 32 * (TC_MMA_WARP + 1);
 constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
 constexpr uint32_t TC_WAIT_LIMIT = 50000;        // polls of up to 20 us: about 1 s per wait
+constexpr uint32_t TC_WAIT_SLEEP_NS = 20000;     // suspend hint of one poll
+constexpr uint32_t TC_DRAIN_LIMIT = 1u << 20;    // polls of the final drains (never shortened)
 constexpr uint32_t BAR_EPI = 2;                  // named barrier of the 256 epilogue threads
 
 constexpr int OP_TILE = TC_BM * TC_KT * 2;            // 16 KB: one fp16 operand tile
@@ -89,6 +93,7 @@ struct TcArgs {
   const float* alpha;
   const float* act_scale;
   float* out;
+  int32_t* sums;    // SUMS: int32 group sums [M][ng][P]
   unsigned int* err;
   Geom g;
   int mtiles;       // filter tiles per conv group
@@ -98,7 +103,8 @@ struct TcArgs {
   int kt_per_group; // G / 64
   int act_tma;      // activation rows by TMA (im2col rows are consecutive input rows)
   int out_tma;      // output tile by TMA store (one conv group, M % 4 == 0)
-  uint32_t wait_limit;
+  uint32_t wait_limit;     // polls per wait (each up to wait_sleep_ns)
+  uint32_t wait_sleep_ns;
 };
 
 __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, int& m0, int64_t& p0) {
@@ -113,7 +119,7 @@ __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, 
 
 // TMAP: the layer's im2col rows are contiguous input rows (TMA loads, TMA-store epilogue);
 // otherwise rows are gathered with cp.async.
-template <int ABITS, bool SIGNED, bool TMAP>
+template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
 __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid_constant__ TcArgs a) {
   constexpr int TC_NS = TMAP ? TC_NS_TMA : TC_NS_GATHER;
   extern __shared__ uint8_t smem_raw[];
@@ -212,7 +218,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         // the slot's previous contents (K-tile j - TC_NS) have been released by every thread
         bool free_ok = true;
         if (j >= TC_NS)
-          free_ok = mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag);
+          free_ok = mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns);
         if (free_ok) {
           mbar_arrive_expect_tx(&st_full[slot], TX_CODES + (TMAP ? TX_ACT : 0u));
           tma_load_2d(smem_u32(sa + ST_ACT), &a.codes_map, kk * (TC_KT / 16), m0, &st_full[slot]);
@@ -270,11 +276,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       if (!TMAP) cp_async_wait<TC_NS - 1>();  // this thread's copies for K-tile j have landed
       const int slot = j % TC_NS;
       const int os = j % TC_NO;
-      if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag)) ||
+      if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) ||
           !(a.kt_per_group > 1
-                ? mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag)
+                ? mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)
                 : (j < TC_NO || mbar_wait_or_abort(&acc_full[(j - TC_NO) % TC_NACC], ((j - TC_NO) / TC_NACC) & 1,
-                                                   a.wait_limit, abort_flag)))) {
+                                                   a.wait_limit, abort_flag, a.wait_sleep_ns)))) {
         if (!*abort_flag) fail();
         break;
       }
@@ -350,7 +356,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     // TMA loads issued but not consumed (only after a failure): wait, bounded, for their
     // bytes to land so that no copy into this CTA's shared memory outlives it
     if (tid == 0) {
-      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % TC_NS], (j / TC_NS) & 1, 1u << 16);
+      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % TC_NS], (j / TC_NS) & 1, TC_DRAIN_LIMIT);
     }
   }
 
@@ -363,7 +369,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
       for (int grp = 0; grp < g.ng && ok; ++grp, ++gc) {
         const int b = gc % TC_NACC;
-        if (!mbar_wait_or_abort(&acc_empty[b], ((gc / TC_NACC) & 1) ^ 1, a.wait_limit, abort_flag)) {
+        if (!mbar_wait_or_abort(&acc_empty[b], ((gc / TC_NACC) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
           if (!*abort_flag) fail();
           ok = false;
           break;
@@ -372,7 +378,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         const uint32_t d = tmem + (uint32_t)(b * TC_BN);
         for (int sub = 0; sub < a.kt_per_group; ++sub, ++kt) {
           const int os = kt % TC_NO;
-          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag)) {
+          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
             if (!*abort_flag) fail();
             ok = false;
             break;
@@ -395,7 +401,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     }
     // all MMAs issued by this thread are complete once the drain barrier flips
     mma_commit(drain_bar);
-    mbar_wait_bounded(drain_bar, 0, a.wait_limit);
+    mbar_wait_bounded(drain_bar, 0, TC_DRAIN_LIMIT);
   }
 
   // ------------------------------------------------------------------ epilogue
@@ -423,13 +429,36 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         const int b = gc % TC_NACC;
         const float al = al_next;  // alpha of this group, loaded one group ahead
         if (mok && grp + 1 < g.ng) al_next = __ldg(arow + grp + 1);
-        if (!mbar_wait_or_abort(&acc_full[b], (gc / TC_NACC) & 1, a.wait_limit, abort_flag)) {
+        if (!mbar_wait_or_abort(&acc_full[b], (gc / TC_NACC) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
           if (!*abort_flag) fail();
           ok = false;
           continue;
         }
         tc_fence_after();
         uint32_t r[32];
+        if (SUMS) {
+          // the exact group sums of positions p0 + 64 half + j, filter m: s[m][grp][p]
+          int32_t* srow = a.sums + ((int64_t)(mok ? m : 0) * g.ng + grp) * g.P;
+          const int64_t pbase = p0 + 64 * half;
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            tmem_ld32(tbase + (uint32_t)(b * TC_BN + 32 * hh), r);
+            tmem_ld_wait();
+            if (hh == 1) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&acc_empty[b]);
+            }
+            if (mok) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                const int64_t p = pbase + 32 * hh + j;
+                if (p < g.P) srow[p] = __float2int_rn(__uint_as_float(r[j]));
+              }
+            }
+          }
+          continue;
+        }
         tmem_ld32(tbase + (uint32_t)(b * TC_BN), r);
         tmem_ld_wait();
 #pragma unroll
@@ -443,6 +472,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         for (int j = 0; j < 32; ++j) acc[32 + j] = fmaf(al, __uint_as_float(r[j]), acc[32 + j]);
       }
       if (named_bar_or(BAR_EPI, 32 * TC_EPI_WARPS, !ok)) break;  // leave together
+      if (SUMS) continue;  // the group sums are stored already
       if (TMAP && a.out_tma) {
         // the previous tile's store has finished reading the staging tile
         if (leader) bulk_wait_read_all();
@@ -485,22 +515,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
   }
 }
 
-template <int ABITS, bool SIGNED, bool TMAP>
+template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
 fgq_status launch_tc(const TcArgs& args, int grid, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(tc_contract_kernel<ABITS, SIGNED, TMAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             TC_SMEM) != cudaSuccess)
-      return FGQ_ERR_CUDA;
-    attr_set = true;
-  }
-  tc_contract_kernel<ABITS, SIGNED, TMAP><<<grid, TC_THREADS, TC_SMEM, s>>>(args);
+  if (!tc::smem_attr_once<tc_contract_kernel<ABITS, SIGNED, TMAP, SUMS>>(TC_SMEM)) return FGQ_ERR_CUDA;
+  tc_contract_kernel<ABITS, SIGNED, TMAP, SUMS><<<grid, TC_THREADS, TC_SMEM, s>>>(args);
   return after_launch();
 }
 
 template <int ABITS, bool SIGNED>
 fgq_status launch_tc_path(const TcArgs& args, int grid, cudaStream_t s) {
-  return args.act_tma ? launch_tc<ABITS, SIGNED, true>(args, grid, s) : launch_tc<ABITS, SIGNED, false>(args, grid, s);
+  if (args.sums)
+    return args.act_tma ? launch_tc<ABITS, SIGNED, true, true>(args, grid, s)
+                        : launch_tc<ABITS, SIGNED, false, true>(args, grid, s);
+  return args.act_tma ? launch_tc<ABITS, SIGNED, true, false>(args, grid, s)
+                      : launch_tc<ABITS, SIGNED, false, false>(args, grid, s);
 }
 
 // One block waits on an mbarrier that nothing arrives on; every wait is bounded, so the
@@ -530,7 +558,7 @@ bool tc_supports(const Geom& g) {
 fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                               const float* act_scale, float* out, int32_t* sums, unsigned int* err,
                               cudaStream_t s) {
-  if (sums != nullptr || !tc_supports(g)) return FGQ_ERR_UNSUPPORTED;
+  if (!tc_supports(g)) return FGQ_ERR_UNSUPPORTED;
   TcArgs a;
   memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
@@ -538,6 +566,7 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   a.alpha = alpha;
   a.act_scale = act_scale;
   a.out = out;
+  a.sums = sums;
   a.err = err;
   a.g = g;
   a.mtiles = (g.Mg + TC_BM - 1) / TC_BM;
@@ -545,7 +574,10 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.kt_per_group = g.G / TC_KT;
   a.ktiles = g.ng * a.kt_per_group;
-  a.wait_limit = TC_WAIT_LIMIT;
+  // a test may shorten the waits (debug_wait_limit_us), never the final drains
+  const int64_t lim_us = debug_wait_limit_us();
+  a.wait_limit = lim_us < 0 ? TC_WAIT_LIMIT : (uint32_t)(lim_us / 20 + 1);
+  a.wait_sleep_ns = lim_us < 0 ? TC_WAIT_SLEEP_NS : (uint32_t)(lim_us < 20 ? lim_us * 1000 : 20000);
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
   if (!make_map_2d(&a.codes_map, CU_TENSOR_MAP_DATA_TYPE_UINT32, codes, (uint64_t)g.wrow, (uint64_t)g.M,
                    (uint64_t)g.wrow * 4, TC_KT / 16, TC_BM, CU_TENSOR_MAP_SWIZZLE_NONE))
@@ -559,7 +591,7 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                     ? 1
                     : 0;
   }
-  if (a.act_tma && g.groups == 1 && g.M % 4 == 0 && !g.rq_out) {
+  if (a.act_tma && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, TC_BM, TC_BN, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1

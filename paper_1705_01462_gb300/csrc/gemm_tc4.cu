@@ -8,7 +8,8 @@
 // N = 256, K = 16) into its own 256-column TMEM buffer: D[m][64 j + P] = s[m][group
 // 4 step + j][P] exactly (fp16 operands on exact integers, |s| <= 4 * 255), and the
 // epilogue applies alpha once per group-output on the CUDA cores (Section 4.1) with packed
-// fp32 FMAs.  The zeros of B' never change, so they are written once per CTA; each K-tile
+// fp32 FMAs; the group-sums variant (SUMS) stores the drained integers as int32 s[m][g][p]
+// instead (for verification).  The zeros of B' never change, so they are written once per CTA; each K-tile
 // writes only the diagonal 8-byte pieces.
 //
 // The ternary operand A is expanded once per call from the 2-bit codes to fp16 {0, +1, -1}
@@ -61,6 +62,7 @@ constexpr int T4_MMA_WARP = 12;
 constexpr int T4_THREADS = 32 * (T4_MMA_WARP + 1);
 constexpr int T4_TMEM_COLS = T4_NACC * 256;
 constexpr uint64_t T4_TIMEOUT_NS = 1000000000ull;  // 1 s per wait
+constexpr uint32_t T4_DRAIN_LIMIT = 1u << 20;      // polls of the final drains (never shortened)
 constexpr uint32_t BAR_EPI4 = 2;
 
 constexpr int A_TILE4 = 128 * T4_KT * 2;   // 16 KB fp16 codes [128 filters][64 K]
@@ -83,6 +85,7 @@ struct T4Args {
   const float* alpha;
   const float* act_scale;
   float* out;
+  int32_t* sums;  // SUMS: int32 group sums [M][ng][P]
   unsigned int* err;
   Geom g;
   int mtiles, ptiles, ntiles, ktiles;
@@ -127,7 +130,7 @@ __global__ void __launch_bounds__(256) expand_codes_kernel(const uint32_t* __res
   a16[2 * i + 1] = make_uint4(h[4], h[5], h[6], h[7]);
 }
 
-template <int ABITS, bool SIGNED, bool TMAP>
+template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
 __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __grid_constant__ T4Args a) {
   extern __shared__ uint8_t smem_raw4[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw4) + 1023) & ~uintptr_t(1023));
@@ -342,11 +345,13 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     if (!ok && !*abort_flag) fail();
     if (!TMAP) cp_async_wait_all();
     if (TMAP && t == 0) {
-      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % T4_NS], (j / T4_NS) & 1, 1u << 16);
+      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % T4_NS], (j / T4_NS) & 1, T4_DRAIN_LIMIT);
     }
-    if (t == 0 && !ok && a_armed > 0) {  // the last A box may still be in flight
-      const int j = a_armed - 1;
-      mbar_wait_bounded(&a_full[j % T4_NO], (j / T4_NO) & 1, 1u << 16);
+    if (t == 0 && !ok) {
+      // A boxes the MMA issuer may not have consumed: the last T4_NO armed ones, one per
+      // stage, each the latest phase of its stage's barrier
+      for (int j = a_armed - T4_NO < 0 ? 0 : a_armed - T4_NO; j < a_armed; ++j)
+        mbar_wait_bounded(&a_full[j % T4_NO], (j / T4_NO) & 1, T4_DRAIN_LIMIT);
     }
   }
 
@@ -382,7 +387,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     }
     if (!ok && !*abort_flag) fail();
     mma_commit(drain_bar);
-    mbar_wait_bounded(drain_bar, 0, 1u << 20);
+    mbar_wait_bounded(drain_bar, 0, T4_DRAIN_LIMIT);
   }
 
   // ------------------------------------------------------------------ epilogue
@@ -420,6 +425,34 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         // slot j at columns 64 j .. 64 j + 63; this warp's 32 positions at + 32 hsub
         const uint32_t ta = tbase + (uint32_t)(b * 256);
         uint32_t r0[32], r1[32];
+        if (SUMS) {
+          // exact sums of groups 4 gs + j, filter m, positions p0 + 32 hsub + i
+          const int64_t pw = p0 + 32 * hsub;
+          int32_t* s0 = a.sums + ((int64_t)(mok ? m : 0) * g.ng + 4 * gs) * g.P;
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            tmem_ld32(ta + 128 * hh, r0);
+            tmem_ld32(ta + 128 * hh + 64, r1);
+            tmem_ld_wait_regs(r0);
+            reg_fence(r1);
+            if (hh == 1) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&acc_empty[b]);
+            }
+            if (mok) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const int64_t p = pw + i;
+                if (p < g.P) {
+                  s0[(2 * hh) * g.P + p] = __float2int_rn(__uint_as_float(r0[i]));
+                  s0[(2 * hh + 1) * g.P + p] = __float2int_rn(__uint_as_float(r1[i]));
+                }
+              }
+            }
+          }
+          continue;
+        }
         tmem_ld32(ta, r0);
         tmem_ld32(ta + 64, r1);
         tmem_ld_wait_regs(r0);
@@ -438,6 +471,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       }
       if (!ok && !*abort_flag) fail();
       if (named_bar_or(BAR_EPI4, 32 * T4_EPI_WARPS, !ok)) break;
+      if (SUMS) continue;  // the group sums are stored already
       if (a.out_tma) {
         if (leader) bulk_wait_read_all();  // the previous tile's store has read the buffer
         named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
@@ -477,22 +511,20 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   }
 }
 
-template <int ABITS, bool SIGNED, bool TMAP>
+template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
 fgq_status launch_tc4(const T4Args& args, int grid, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(tc4_contract_kernel<ABITS, SIGNED, TMAP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             T4_SMEM) != cudaSuccess)
-      return FGQ_ERR_CUDA;
-    attr_set = true;
-  }
-  tc4_contract_kernel<ABITS, SIGNED, TMAP><<<grid, T4_THREADS, T4_SMEM, s>>>(args);
+  if (!tc::smem_attr_once<tc4_contract_kernel<ABITS, SIGNED, TMAP, SUMS>>(T4_SMEM)) return FGQ_ERR_CUDA;
+  tc4_contract_kernel<ABITS, SIGNED, TMAP, SUMS><<<grid, T4_THREADS, T4_SMEM, s>>>(args);
   return after_launch();
 }
 
 template <int ABITS, bool SIGNED>
 fgq_status launch_tc4_path(const T4Args& args, int grid, cudaStream_t s) {
-  return args.act_tma ? launch_tc4<ABITS, SIGNED, true>(args, grid, s) : launch_tc4<ABITS, SIGNED, false>(args, grid, s);
+  if (args.sums)
+    return args.act_tma ? launch_tc4<ABITS, SIGNED, true, true>(args, grid, s)
+                        : launch_tc4<ABITS, SIGNED, false, true>(args, grid, s);
+  return args.act_tma ? launch_tc4<ABITS, SIGNED, true, false>(args, grid, s)
+                      : launch_tc4<ABITS, SIGNED, false, false>(args, grid, s);
 }
 
 }  // namespace
@@ -507,7 +539,8 @@ bool tc4_supports(const Geom& g) {
 }
 
 fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
-                               const float* act_scale, float* out, unsigned int* err, cudaStream_t s) {
+                               const float* act_scale, float* out, int32_t* sums, unsigned int* err,
+                               cudaStream_t s) {
   if (!tc4_supports(g)) return FGQ_ERR_UNSUPPORTED;
   T4Args a;
   memset(&a, 0, sizeof a);
@@ -515,13 +548,16 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   a.alpha = alpha;
   a.act_scale = act_scale;
   a.out = out;
+  a.sums = sums;
   a.err = err;
   a.g = g;
   a.mtiles = (g.Mg + T4_BM - 1) / T4_BM;
   a.ptiles = (int)((g.P + T4_BP - 1) / T4_BP);
   a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.ktiles = g.Kp / T4_KT;
-  a.timeout_ns = T4_TIMEOUT_NS;
+  // a test may shorten the waits (debug_wait_limit_us), never the final drains
+  const int64_t lim_us = debug_wait_limit_us();
+  a.timeout_ns = lim_us < 0 ? T4_TIMEOUT_NS : (uint64_t)lim_us * 1000u;
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
 
   // expanded codes: fp16 [M][Kp] (Kp = 16 wrow), in a temporary from the stream-ordered pool
@@ -544,7 +580,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
                     ? 1
                     : 0;
   }
-  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out) {
+  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, T4_BM, T4_BP, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1

@@ -59,14 +59,14 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
   return false;
 }
 
-// Waits (sleeping in the hardware for up to 20 us per poll) for the phase with the given
+// Waits (sleeping in the hardware for up to sleep_ns per poll) for the phase with the given
 // parity; gives up after max_iter polls or once *abort becomes non-zero, so that one
 // role's timeout releases the roles waiting on it.  max_iter polls bound the wait by
-// max_iter * 20 us.
+// max_iter * sleep_ns (plus the hardware's own short limit per poll).
 __device__ __forceinline__ bool mbar_wait_or_abort(uint64_t* bar, uint32_t parity, uint32_t max_iter,
-                                                   volatile uint32_t* abort) {
+                                                   volatile uint32_t* abort, uint32_t sleep_ns = 20000u) {
   for (uint32_t i = 0; i < max_iter; ++i) {
-    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (mbar_try_wait_sleep(bar, parity, sleep_ns)) return true;
     if (*abort) return false;
   }
   return false;

@@ -79,6 +79,21 @@ __device__ __forceinline__ void codes_half_row_to_fp16(const uint8_t* codes16, i
   }
 }
 
+// Raises a kernel's dynamic shared-memory limit to `bytes`, once per device (the attribute
+// belongs to the device's context); thread-safe.  Returns false if the call failed.
+template <auto Kernel>
+bool smem_attr_once(int bytes) {
+  constexpr int kDev = 64;
+  static std::once_flag once[kDev];
+  static bool ok[kDev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDev) return false;
+  std::call_once(once[dev], [&] {
+    ok[dev] = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess;
+  });
+  return ok[dev];
+}
+
 // cuTensorMapEncodeTiled from the driver, looked up once through the runtime.
 inline PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;

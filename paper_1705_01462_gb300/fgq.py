@@ -23,7 +23,7 @@ ACT_TYPES = {"u8": U8, "s8": S8, "u4": U4, "s4": S4}
 
 _lib: Optional[ctypes.CDLL] = None
 
-# (name, restype, argtypes) of every exported symbol of include/fgq.h
+# (name, restype, argtypes) of every exported symbol of include/fgq.h and include/fgq_debug.h
 _vp, _i, _i64, _u32, _u64, _f, _sz = (ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_uint32,
                                       ctypes.c_uint64, ctypes.c_float, ctypes.c_size_t)
 SIGNATURES = [
@@ -52,11 +52,16 @@ SIGNATURES = [
     ("fgq_gemm_qa", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d_qa", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _vp, _i, _i, _vp, _vp]),
     ("fgq_group_sums", _i, [_vp, _i, _i, _i, _vp, _i, _i, _vp, _vp]),
+    ("fgq_conv2d_group_sums", _i, [_vp, _i] + [_i] * 9 + [_vp, _i, _i, _vp, _vp]),
+    ("fgq_conv2d_host_workspace_bytes", _sz, [_i] * 12),
+    ("fgq_conv2d_host", _i, [_vp, _vp, _i] + [_i] * 11 + [_vp, _vp, _sz, _vp]),
     ("fgq_stream_status", _i, [_vp]),
     ("fgq_set_path", _i, [_i]),
     ("fgq_last_path", _i, []),
     ("fgq_launch_count", _u64, []),
     ("fgq_selftest_wait_timeout", _i, [_u32, _vp]),
+    ("fgq_debug_set_wait_limit_us", _i64, [_i64]),
+    ("fgq_debug_allow_split_fold", _i, [_i]),
 ]
 
 
@@ -415,12 +420,55 @@ def fgq_group_sums(q: torch.Tensor, act_type, P: int, Kred: int, codes: torch.Te
     return s
 
 
+def fgq_conv2d_group_sums(act: torch.Tensor, act_type, B: int, H: int, W: int, C: int, R: int, S: int, stride: int,
+                          pad: int, groups: int, codes: torch.Tensor, M: int, G: int, stream=None) -> torch.Tensor:
+    _require_cuda()
+    Ho, Wo = conv_out_hw(H, W, R, S, stride, pad)
+    s = torch.empty((M, num_groups(R * S * (C // groups), G), B * Ho * Wo), dtype=torch.int32, device=act.device)
+    _check(lib().fgq_conv2d_group_sums(_dev(act, torch.uint8, "act"), _act_type(act_type), B, H, W, C, R, S, stride,
+                                       pad, groups, _dev(codes, torch.int32, "codes"), M, G, s.data_ptr(),
+                                       _stream(stream)), "fgq_conv2d_group_sums")
+    return s
+
+
+def conv2d_host_workspace_bytes(act_type, B: int, H: int, W: int, C: int, R: int, S: int, stride: int, pad: int,
+                                groups: int, M: int, G: int) -> int:
+    return int(lib().fgq_conv2d_host_workspace_bytes(_act_type(act_type), B, H, W, C, R, S, stride, pad, groups, M, G))
+
+
+def fgq_conv2d_host(h_w: torch.Tensor, h_x: torch.Tensor, act_type, B: int, H: int, W: int, C: int, R: int, S: int,
+                    stride: int, pad: int, groups: int, M: int, G: int, h_out: torch.Tensor, workspace: torch.Tensor,
+                    stream=None) -> None:
+    """One layer end to end from host fp32 tensors (h_w [M][Kred], h_x NHWC) into host fp32
+    h_out, through the C ABI; asynchronous on the stream (synchronize before reading h_out)."""
+    _require_cuda()
+    for t, name in ((h_w, "h_w"), (h_x, "h_x"), (h_out, "h_out")):
+        if t.device.type != "cpu" or t.dtype != torch.float32 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous float32 host tensor")
+    if not workspace.is_cuda or not workspace.is_contiguous():
+        raise ValueError("workspace must be a contiguous device tensor")
+    _check(lib().fgq_conv2d_host(h_w.data_ptr(), h_x.data_ptr(), _act_type(act_type), B, H, W, C, R, S, stride, pad,
+                                 groups, M, G, h_out.data_ptr(), workspace.data_ptr(),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)), "fgq_conv2d_host")
+
+
 def fgq_stream_status(stream=None) -> int:
     return int(lib().fgq_stream_status(_stream(stream)))
 
 
 def fgq_set_path(path: int) -> int:
+    """Kernel family of this thread's contraction calls (test and benchmark control)."""
     return int(lib().fgq_set_path(path))
+
+
+def fgq_debug_set_wait_limit_us(us: int) -> int:
+    """Wait limit of this thread's tensor-core kernel launches (test control; -1 restores)."""
+    return int(lib().fgq_debug_set_wait_limit_us(us))
+
+
+def fgq_debug_allow_split_fold(allow: bool) -> int:
+    """Lets FGQ_PATH_DENSE run fp32 alphas as the split-fp16 ablation on this thread."""
+    return int(lib().fgq_debug_allow_split_fold(1 if allow else 0))
 
 
 def fgq_last_path() -> int:

@@ -9,13 +9,18 @@ import pytest
 
 from conftest import ROOT
 
-HEADER = os.path.join(ROOT, "include", "fgq.h")
+INCLUDE = os.path.join(ROOT, "include")
 
 
 def header_functions():
-    src = open(HEADER).read()
-    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(fgq_[a-z0-9_]+)\s*\(", src, flags=re.M)
+    """Every function declared in include/*.h."""
+    names = []
+    for fn in sorted(os.listdir(INCLUDE)):
+        if not fn.endswith(".h"):
+            continue
+        src = open(os.path.join(INCLUDE, fn)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(fgq_[a-z0-9_]+)\s*\(", src, flags=re.M)
     return sorted(set(names))
 
 
@@ -39,7 +44,7 @@ def test_every_declared_symbol_is_exported(L):
     from paper_1705_01462_gb300 import fgq
     bound = {n for n, _, _ in fgq.SIGNATURES}
     for name in header_functions():
-        assert hasattr(L, name), f"{name} declared in fgq.h but not exported"
+        assert hasattr(L, name), f"{name} declared in include/*.h but not exported"
         assert name in bound, f"{name} has no Python binding"
 
 
@@ -75,3 +80,42 @@ def test_host_argument_errors(L):
     assert L.fgq_set_path(9) == -1
     prev = L.fgq_set_path(fgq.PATH_SIMT)
     assert L.fgq_set_path(prev) == fgq.PATH_SIMT
+    # conv group sums: bad G, groups not dividing C; forced dense / few-row paths form no sums
+    assert L.fgq_conv2d_group_sums(p, 0, 1, 8, 8, 8, 3, 3, 1, 1, 1, p, 8, 3, p, None) == fgq.FGQ_ERR_ARG
+    assert L.fgq_conv2d_group_sums(p, 0, 1, 8, 8, 6, 3, 3, 1, 1, 4, p, 8, 4, p, None) == fgq.FGQ_ERR_ARG
+    assert L.fgq_conv2d_group_sums(p, 0, 0, 8, 8, 8, 3, 3, 1, 1, 1, p, 8, 4, p, None) == fgq.FGQ_OK  # B = 0
+    for path in (fgq.PATH_DENSE, fgq.PATH_GEMV):
+        prev = L.fgq_set_path(path)
+        try:
+            assert L.fgq_group_sums(p, 0, 8, 64, p, 8, 4, p, None) == fgq.FGQ_ERR_UNSUPPORTED
+        finally:
+            L.fgq_set_path(prev)
+
+
+def test_debug_controls_are_per_thread(L):
+    """The test controls of fgq_debug.h set on one host thread leave another's alone."""
+    import threading
+    from paper_1705_01462_gb300 import fgq
+    prev = L.fgq_set_path(fgq.PATH_TC)
+    prev_w = L.fgq_debug_set_wait_limit_us(5)
+    prev_s = L.fgq_debug_allow_split_fold(1)
+    seen = {}
+
+    def other():
+        seen["path"] = L.fgq_set_path(fgq.PATH_AUTO)
+        seen["wait"] = L.fgq_debug_set_wait_limit_us(-1)
+        seen["split"] = L.fgq_debug_allow_split_fold(0)
+
+    th = threading.Thread(target=other)
+    th.start()
+    th.join()
+    try:
+        assert seen == {"path": fgq.PATH_AUTO, "wait": -1, "split": 0}
+        assert L.fgq_set_path(prev) == fgq.PATH_TC
+        assert L.fgq_debug_set_wait_limit_us(prev_w) == 5
+        assert L.fgq_debug_allow_split_fold(prev_s) == 1
+    finally:
+        L.fgq_set_path(prev)
+        L.fgq_debug_set_wait_limit_us(prev_w)
+        L.fgq_debug_allow_split_fold(prev_s)
+

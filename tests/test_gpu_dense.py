@@ -5,7 +5,8 @@ C ABI.
   weights a * t are integers, so the contraction is exact and the output is the oracle's
   exact value rounded once to fp32 wherever |sum a t q| < 2^24 (everywhere in these cases),
   and within the contraction tolerance in any case.
-* fp32 alphas split into two fp16 parts (an ablation, only when forced): within the bound
+* fp32 alphas split into two fp16 parts (an ablation, only when forced and allowed by the
+  test switch fgq_debug_allow_split_fold; refused otherwise): within the bound
   its arithmetic gives, s_x sum_k |alpha t q| (2^-21 + steps 2^-23) with one rounding of
   the accumulator per 16 reduction elements and per part, and most outputs inside the
   contraction tolerance as well."""
@@ -25,8 +26,10 @@ pytestmark = pytest.mark.gpu
 @pytest.fixture(autouse=True)
 def _clean_status():
     fgq.fgq_set_path(fgq.PATH_AUTO)
+    fgq.fgq_debug_allow_split_fold(False)
     yield
     fgq.fgq_set_path(fgq.PATH_AUTO)
+    fgq.fgq_debug_allow_split_fold(False)
     assert fgq.fgq_stream_status() == fgq.FGQ_OK
 
 
@@ -111,9 +114,14 @@ def test_conv2d_split_fold_ablation(case):
     x = random_acts((B, H, W, C), act, rng)
     q, sc, packed = quantize_oracle(x, act)
     y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    args = (to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad, groups,
+            to_dev(codes.view(np.int32)), to_dev(al), M, G)
     fgq.fgq_set_path(fgq.PATH_DENSE)
-    got = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad,
-                         groups, to_dev(codes.view(np.int32)), to_dev(al), M, G).cpu().numpy()
+    with pytest.raises(fgq.FGQError) as e:  # fp32 alphas: refused without the ablation switch
+        fgq.fgq_conv2d(*args)
+    assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
+    fgq.fgq_debug_allow_split_fold(True)
+    got = fgq.fgq_conv2d(*args).cpu().numpy()
     assert fgq.fgq_last_path() == fgq.PATH_DENSE
     mag = _split_bound(q, sc, t, al, G, (R, S, stride, pad, groups))
     steps = 2 * Kred // 16
@@ -135,6 +143,7 @@ def test_conv2d_rq_dense_split():
     args = (to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad, groups,
             to_dev(codes.view(np.int32)), to_dev(al), M, G)
     fgq.fgq_set_path(fgq.PATH_DENSE)
+    fgq.fgq_debug_allow_split_fold(True)
     y32 = fgq.fgq_conv2d(*args).cpu().numpy()
     for out_type, ot in (("u8", O.U8), ("s8", O.S8)):
         scale = np.float32(2.0 ** O.dfp_exponent(y32.reshape(-1), ot))
