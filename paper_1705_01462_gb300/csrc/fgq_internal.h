@@ -82,6 +82,12 @@ bool dense_supports(const Geom& g);
 fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
                                  const uint8_t* aq, int abits, const float* ascale, const float* act_scale, float* out,
                                  unsigned int* err, cudaStream_t s);
+// fp32 alphas folded into the codes as two fp16 parts: a0[m][k] + a1[m][k] = alpha(m, k / G) *
+// t[m][k] * 2^e_m to about 22 bits (a0 the fp16 nearest, a1 the fp16 nearest the remainder),
+// with e_m putting row m's largest alpha in [2^14, 2^15), and rs[m] = 2^-e_m.  a0, a1 fp16
+// [M][16 wrow]; codes 00 and padding give 0.
+fgq_status launch_fold_alpha_split(const uint32_t* codes, int M, int wrow, int G, int ng, const float* alpha,
+                                   void* a0, void* a1, float* rs, cudaStream_t s);
 // The 8-bit-weight convolution (dense weights wq, per-filter scales) on the same kernel, through
 // an explicit im2col of the activations in a pool temporary (any C, groups == 1); exact.
 bool dense_w8_supports(const Geom& g);

@@ -674,6 +674,13 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
   return st;
 }
 
+fgq_status launch_fold_alpha_split(const uint32_t* codes, int M, int wrow, int G, int ng, const float* alpha,
+                                   void* a0, void* a1, float* rs, cudaStream_t s) {
+  fold_weights_kernel<0><<<(unsigned)((M + 7) / 8), 256, 0, s>>>(codes, M, wrow, G, ng, alpha, nullptr, nullptr,
+                                                                static_cast<__half*>(a0), static_cast<__half*>(a1), rs);
+  return after_launch();
+}
+
 bool dense_w8_supports(const Geom& g) {
   if (g.act_type != FGQ_U8 && g.act_type != FGQ_S8) return false;
   if (g.groups != 1 || g.P >= (int64_t)1 << 31) return false;

@@ -4,29 +4,41 @@
 // * s[m][g][p] with s an exact integer sum over a group of 4 reduction elements.  A dense
 // MMA would sum across groups, so each K = 16 MMA step (4 groups) uses a block-diagonal
 // activation operand B' of 256 rows: row 64 j + P holds the activations of tile position P
-// only in the 4 columns of group slot j (zeros elsewhere).  Each step is one MMA (M = 128,
-// N = 256, K = 16) into its own 256-column TMEM buffer: D[m][64 j + P] = s[m][group
-// 4 step + j][P] exactly (fp16 operands on exact integers, |s| <= 4 * 255), and the
-// epilogue applies alpha once per group-output on the CUDA cores (Section 4.1) with packed
-// fp32 FMAs; the group-sums variant (SUMS) stores the drained integers as int32 s[m][g][p]
-// instead (for verification).  The zeros of B' never change, so they are written once per CTA; each K-tile
-// writes only the diagonal 8-byte pieces.
+// only in the 4 columns of group slot j (zeros elsewhere), and D[m][64 j + P] of one MMA
+// (M = 128, N = 256, K = 16) receives the products of group 4 step + j alone.  The zeros of
+// B' never change, so they are written once per CTA; each K-tile writes only the diagonal
+// 8-byte pieces.  Two variants share the loaders:
 //
-// The ternary operand A is expanded once per call from the 2-bit codes to fp16 {0, +1, -1}
-// in a stream-ordered temporary (expand_codes_kernel) and reaches shared memory by TMA box
-// loads in the MMA's swizzled layout.
+//   output (FOLD): the group's scale multiplies inside the MMA (one multiply per group,
+//     Section 4.1): the ternary operand is the fp32 alpha folded into the codes as two fp16
+//     parts, alpha(m, g) t[m][k] 2^e_m = hi + lo to about 22 bits (hi the fp16 nearest, lo the
+//     fp16 nearest the remainder; e_m puts row m's largest alpha in [2^14, 2^15)).  Every
+//     product hi t q and lo t q is exact in fp32 and so is each part's group sum hi s_g (11
+//     significant bits times |s_g| <= 1020), so one step adds (hi + lo) s_g to the element
+//     its slot owns.  The 8 MMAs of a K-tile (4 steps x 2 parts) accumulate in TMEM, and the
+//     epilogue adds the K-tile's four slot partials into fp32 registers with round-to-nearest
+//     adds: every rounding is bounded by a K-tile's share of sum_g |alpha_g s_g|, far inside
+//     the 1e-5 sum_g |alpha_g s_g| tolerance, and the accumulator is drained (and committed)
+//     once per K-tile instead of once per step.  y = s_x 2^-e_m acc.
+//   group sums (!FOLD): the ternary operand is the codes in fp16 {0, +1, -1}; each step's
+//     D is exactly s[m][g][p] (fp16 operands on exact integers), stored as int32 (for
+//     verification of the integer accumulators).
+//
+// The ternary operand reaches shared memory by TMA box loads in the MMA's swizzled layout,
+// from a per-call stream-ordered temporary (folded: launch_fold_alpha_split; codes:
+// expand_codes_kernel).
 //
 // Tile: 128 filters x 64 positions; K-tile 64 (16 groups, 4 steps).  TMEM: two 256-column
-// buffers; the MMA of step s + 1 runs while the epilogue drains step s.  N = 256 keeps the
-// tensor pipe at its full rate, and one commit per step keeps the commits (each of which
-// drains the pipe) to four per K-tile.
+// buffers.  Output: one buffer per K-tile, so the MMAs of K-tile j + 1 run while the
+// epilogue drains K-tile j.  Group sums: one buffer per step.
 // Warp roles (416 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w owns TMEM lanes 32 (w % 4) .. (filters) and the 32
-//              positions of half w / 4; per step it loads its four 32-column slices (two
-//              at a time, each later load overlapped with the FMAs of an earlier one), frees
-//              the buffer, and adds alpha * s into 32 position accumulators; at tile end it
-//              scales by s_x and writes its 32 x 32 block (through shared memory and a TMA
-//              box store when the output allows).
+//              positions of half w / 4; it loads its 32-column slices of the four slots
+//              (two at a time), frees the buffer once they are in registers, and adds them
+//              into 32 position accumulators (output), or stores them as int32 (group
+//              sums).  At tile end the output is scaled by s_x 2^-e_m and written through
+//              shared memory with TMA box stores (two 32-position boxes) when the output
+//              allows, else directly (or requantized).
 //   warps 8-11 loaders/converters: thread t builds, for position t % 64, MMA steps
 //              2 (t / 64), 2 (t / 64) + 1 of B'; activations come by TMA boxes (1x1
 //              stride-1 layers and GEMMs) or by per-thread cp.async gathers whose completion
@@ -53,8 +65,7 @@ constexpr int T4_BM = 128;      // filters per tile (MMA M, TMEM lanes)
 constexpr int T4_BP = 64;       // positions per tile
 constexpr int T4_KT = 64;       // reduction elements per K-tile: 16 groups, 4 MMA steps
 constexpr int T4_NO = 3;        // operand ring depth
-constexpr int T4_NS = 6;        // staging ring depth
-constexpr int T4_NACC = 2;      // TMEM buffers of 256 columns (one step each)
+constexpr int T4_NACC = 2;      // TMEM buffers of 256 columns
 constexpr int T4_EPI_WARPS = 8;
 constexpr int T4_LOAD_WARP0 = 8;  // loaders: warps 8-11
 constexpr int T4_LOADERS = 128;
@@ -65,27 +76,36 @@ constexpr uint64_t T4_TIMEOUT_NS = 1000000000ull;  // 1 s per wait
 constexpr uint32_t T4_DRAIN_LIMIT = 1u << 20;      // polls of the final drains (never shortened)
 constexpr uint32_t BAR_EPI4 = 2;
 
-constexpr int A_TILE4 = 128 * T4_KT * 2;   // 16 KB fp16 codes [128 filters][64 K]
-constexpr int B_TILE4 = 256 * T4_KT * 2;   // 32 KB fp16 block-diagonal activations
-constexpr int OP_STAGE4 = A_TILE4 + B_TILE4;
-constexpr int ST_STAGE4 = T4_BP * T4_KT;   // 4 KB: 64 raw activation rows (8-bit: 64 B each)
-constexpr int OUT_TILE4 = T4_BP * T4_BM * 4;  // 32 KB fp32 [64 positions][128 filters]
-constexpr int SMEM_OP4 = T4_NO * OP_STAGE4;
-constexpr int SMEM_ST4 = T4_NS * ST_STAGE4;
-constexpr int SMEM_BAR4 = 8 * (3 * T4_NO + 2 * T4_NS + 2 * T4_NACC + 1) + 16;
-constexpr int T4_SMEM = 1024 + SMEM_OP4 + SMEM_ST4 + OUT_TILE4 + SMEM_BAR4;
-static_assert(T4_SMEM <= 232448, "shared memory budget");
-static_assert(ST_STAGE4 % 1024 == 0 && OP_STAGE4 % 1024 == 0, "stage alignment");
+constexpr int A_TILE4 = 128 * T4_KT * 2;      // 16 KB fp16 ternary operand [128 filters][64 K], per part
+constexpr int B_TILE4 = 256 * T4_KT * 2;      // 32 KB fp16 block-diagonal activations
+constexpr int ST_STAGE4 = T4_BP * T4_KT;      // 4 KB: 64 raw activation rows (8-bit: 64 B each)
+constexpr int OUT_BOX4 = 32 * T4_BM * 4;      // 16 KB fp32 [32 positions][128 filters]
+
+// Shared-memory plan of a variant: operand stages (A parts + B'), staging ring, output box.
+template <bool FOLD>
+struct T4Cfg {
+  static constexpr int NPART = FOLD ? 2 : 1;
+  static constexpr int A_STAGE = NPART * A_TILE4;
+  static constexpr int OP_STAGE = A_STAGE + B_TILE4;
+  static constexpr int NS = FOLD ? 4 : 6;  // staging ring depth
+  static constexpr int OUT = FOLD ? OUT_BOX4 : 0;
+  static constexpr int BAR = 8 * (3 * T4_NO + 2 * NS + 2 * T4_NACC + 1) + 16;
+  static constexpr int SMEM = 1024 + T4_NO * OP_STAGE + NS * ST_STAGE4 + OUT + BAR;
+};
+static_assert(T4Cfg<true>::SMEM <= 232448 && T4Cfg<false>::SMEM <= 232448, "shared memory budget");
+static_assert(ST_STAGE4 % 1024 == 0 && T4Cfg<true>::OP_STAGE % 1024 == 0 && T4Cfg<false>::OP_STAGE % 1024 == 0,
+              "stage alignment");
 
 struct T4Args {
-  CUtensorMap a16_map;    // fp16 [M][Kp] expanded codes, box {64, 128 rows}, 128-byte swizzle
+  CUtensorMap a_map[2];   // fp16 [M][Kp] ternary operand parts (folded hi, lo; or codes), box {64, 128 rows},
+                          // 128-byte swizzle
   CUtensorMap act_map;    // uint8 [pixels][row bytes], box {64 (or 32) bytes, 64 rows}; TMA path
-  CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 64 positions}; if out_tma
+  CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 32 positions}; if out_tma
   const uint8_t* act;
-  const float* alpha;
+  const float* row_scale;  // FOLD: 2^-e_m [M]
   const float* act_scale;
   float* out;
-  int32_t* sums;  // SUMS: int32 group sums [M][ng][P]
+  int32_t* sums;  // !FOLD: int32 group sums [M][ng][P]
   unsigned int* err;
   Geom g;
   int mtiles, ptiles, ntiles, ktiles;
@@ -104,11 +124,9 @@ __device__ __forceinline__ void tile_coords4(const T4Args& a, int tile, int& gi,
   p0 = (int64_t)pt * T4_BP;
 }
 
-// acc[2i..2i+1] += al * r[2i..2i+1]
-__device__ __forceinline__ void scale_add(float (&acc)[32], const uint32_t (&r)[32], float al) {
+__device__ __forceinline__ void add32(float (&acc)[32], const uint32_t (&r)[32]) {
 #pragma unroll
-  for (int i = 0; i < 16; ++i)
-    ffma2(acc[2 * i], acc[2 * i + 1], __uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]), al);
+  for (int i = 0; i < 32; ++i) acc[i] += __uint_as_float(r[i]);
 }
 
 // Expands 2-bit codes (00 = 0, 01 = +1, 11 = -1; element k in word k / 16, bits 2 (k % 16))
@@ -130,20 +148,22 @@ __global__ void __launch_bounds__(256) expand_codes_kernel(const uint32_t* __res
   a16[2 * i + 1] = make_uint4(h[4], h[5], h[6], h[7]);
 }
 
-template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
+template <int ABITS, bool SIGNED, bool TMAP, bool FOLD>
 __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __grid_constant__ T4Args a) {
+  using Cfg = T4Cfg<FOLD>;
+  constexpr int NS = Cfg::NS;
   extern __shared__ uint8_t smem_raw4[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw4) + 1023) & ~uintptr_t(1023));
   uint8_t* op = smem;
-  uint8_t* st = smem + SMEM_OP4;
-  float* otile = reinterpret_cast<float*>(smem + SMEM_OP4 + SMEM_ST4);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP4 + SMEM_ST4 + OUT_TILE4);
+  uint8_t* st = smem + T4_NO * Cfg::OP_STAGE;
+  float* otile = reinterpret_cast<float*>(st + NS * ST_STAGE4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(st + NS * ST_STAGE4 + Cfg::OUT);
   uint64_t* op_full = bars;
   uint64_t* op_empty = bars + T4_NO;
   uint64_t* a_full = bars + 2 * T4_NO;
   uint64_t* st_full = bars + 3 * T4_NO;
-  uint64_t* st_empty = st_full + T4_NS;
-  uint64_t* acc_full = st_empty + T4_NS;
+  uint64_t* st_empty = st_full + NS;
+  uint64_t* acc_full = st_empty + NS;
   uint64_t* acc_empty = acc_full + T4_NACC;
   uint64_t* drain_bar = acc_empty + T4_NACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
@@ -158,9 +178,9 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     for (int i = 0; i < T4_NO; ++i) {
       mbar_init(&op_full[i], T4_LOADERS);  // B' pieces
       mbar_init(&op_empty[i], 1);
-      mbar_init(&a_full[i], 1);            // the A box's byte count
+      mbar_init(&a_full[i], 1);            // the A boxes' byte count
     }
-    for (int i = 0; i < T4_NS; ++i) {
+    for (int i = 0; i < NS; ++i) {
       mbar_init(&st_full[i], TMAP ? 1 : T4_LOADERS);
       mbar_init(&st_empty[i], T4_LOADERS);
     }
@@ -174,7 +194,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   }
   // the off-diagonal zeros of every B' tile, written once
   for (int s = 0; s < T4_NO; ++s) {
-    uint4* bt = reinterpret_cast<uint4*>(op + s * OP_STAGE4 + A_TILE4);
+    uint4* bt = reinterpret_cast<uint4*>(op + s * Cfg::OP_STAGE + Cfg::A_STAGE);
     for (int i = threadIdx.x; i < B_TILE4 / 16; i += blockDim.x) bt[i] = make_uint4(0u, 0u, 0u, 0u);
   }
   fence_proxy_async_smem();
@@ -226,18 +246,18 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         phb = ho * g.stride - g.pad;
         pwb = wo * g.stride - g.pad;
       }
-      const int slot = j % T4_NS;
+      const int slot = j % NS;
       uint8_t* sa = st + slot * ST_STAGE4;
       if (TMAP) {
         if (t == 0) {
-          if (j >= T4_NS && !mbar_wait_timed(&st_empty[slot], ((j / T4_NS) & 1) ^ 1, tmo, abort_flag, 64))
+          if (j >= NS && !mbar_wait_timed(&st_empty[slot], ((j / NS) & 1) ^ 1, tmo, abort_flag, 64))
             return false;
           mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
           tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
           issued = j + 1;
         }
       } else {
-        if (j >= T4_NS && !mbar_wait_timed(&st_empty[slot], ((j / T4_NS) & 1) ^ 1, tmo, abort_flag, 64))
+        if (j >= NS && !mbar_wait_timed(&st_empty[slot], ((j / NS) & 1) ^ 1, tmo, abort_flag, 64))
           return false;
         const uint8_t* src = a.act;
         bool inside = false;
@@ -270,31 +290,33 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     };
 
     bool ok = true;
-    for (int j = 0; j < T4_NS - 1 && j < total && ok; ++j) ok = issue(j);
+    for (int j = 0; j < NS - 1 && j < total && ok; ++j) ok = issue(j);
     int consumed = 0;
     for (int j = 0; j < total && ok; ++j) {
-      if (j + T4_NS - 1 < total && !issue(j + T4_NS - 1)) {
+      if (j + NS - 1 < total && !issue(j + NS - 1)) {
         ok = false;
         break;
       }
-      const int slot = j % T4_NS;
+      const int slot = j % NS;
       const int os = j % T4_NO;
       if (!mbar_wait_timed(&op_empty[os], ((j / T4_NO) & 1) ^ 1, tmo, abort_flag, 64)) {
         ok = false;
         break;
       }
-      uint8_t* A = op + os * OP_STAGE4;
-      uint8_t* Bt = A + A_TILE4;
-      if (t == 0) {  // the A box of K-tile j: expanded codes of the tile's 128 filters
+      uint8_t* A = op + os * Cfg::OP_STAGE;
+      uint8_t* Bt = A + Cfg::A_STAGE;
+      if (t == 0) {  // the A boxes of K-tile j: the tile's 128 filter rows, per part
         const int tl = j / a.ktiles;
         int gj, mj;
         int64_t pj;
         tile_coords4(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
-        mbar_arrive_expect_tx(&a_full[os], A_TILE4);
-        tma_load_2d(smem_u32(A), &a.a16_map, (j - tl * a.ktiles) * T4_KT, mj, &a_full[os]);
+        mbar_arrive_expect_tx(&a_full[os], Cfg::A_STAGE);
+#pragma unroll
+        for (int part = 0; part < Cfg::NPART; ++part)
+          tma_load_2d(smem_u32(A + part * A_TILE4), &a.a_map[part], (j - tl * a.ktiles) * T4_KT, mj, &a_full[os]);
         a_armed = j + 1;
       }
-      if (!mbar_wait_timed(&st_full[slot], (j / T4_NS) & 1, tmo, abort_flag, 32)) {
+      if (!mbar_wait_timed(&st_full[slot], (j / NS) & 1, tmo, abort_flag, 32)) {
         ok = false;
         break;
       }
@@ -345,7 +367,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     if (!ok && !*abort_flag) fail();
     if (!TMAP) cp_async_wait_all();
     if (TMAP && t == 0) {
-      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % T4_NS], (j / T4_NS) & 1, T4_DRAIN_LIMIT);
+      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % NS], (j / NS) & 1, T4_DRAIN_LIMIT);
     }
     if (t == 0 && !ok) {
       // A boxes the MMA issuer may not have consumed: the last T4_NO armed ones, one per
@@ -360,7 +382,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     const uint32_t idesc = idesc_f16_f32(128, 256);
     const uint32_t op_base = smem_u32(op);
     const int total = my_tiles * a.ktiles;
-    int sc = 0;
+    int sc = 0;  // group sums: steps issued
     bool ok = true;
     for (int j = 0; j < total && ok; ++j) {
       const int os = j % T4_NO;
@@ -370,18 +392,35 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         break;
       }
       tc_fence_after();
-      const uint32_t abase = op_base + os * OP_STAGE4;
-      const uint64_t ad = sdesc_k_sw128(abase);
-      const uint64_t bd = sdesc_k_sw128(abase + A_TILE4);
-      for (int s = 0; s < 4; ++s, ++sc) {
-        const int b = sc & 1;
-        if (!mbar_wait_timed(&acc_empty[b], ((sc >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
+      const uint32_t abase = op_base + os * Cfg::OP_STAGE;
+      const uint64_t bd = sdesc_k_sw128(abase + Cfg::A_STAGE);
+      if (FOLD) {
+        // the K-tile's 8 MMAs (4 steps x 2 parts) accumulate into buffer j % 2
+        const int b = j & 1;
+        if (!mbar_wait_timed(&acc_empty[b], ((j >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        mma_f16(tmem + (uint32_t)(b * 256), ad + 2 * s, bd + 2 * s, idesc, 0u);
+#pragma unroll
+        for (int s = 0; s < 4; ++s)
+#pragma unroll
+          for (int part = 0; part < Cfg::NPART; ++part)
+            mma_f16(tmem + (uint32_t)(b * 256), sdesc_k_sw128(abase + part * A_TILE4) + 2 * s, bd + 2 * s, idesc,
+                    (s | part) != 0 ? 1u : 0u);
         mma_commit(&acc_full[b]);
+      } else {
+        const uint64_t ad = sdesc_k_sw128(abase);
+        for (int s = 0; s < 4; ++s, ++sc) {
+          const int b = sc & 1;
+          if (!mbar_wait_timed(&acc_empty[b], ((sc >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          mma_f16(tmem + (uint32_t)(b * 256), ad + 2 * s, bd + 2 * s, idesc, 0u);
+          mma_commit(&acc_full[b]);
+        }
       }
       mma_commit(&op_empty[os]);
     }
@@ -397,8 +436,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(32 * hsub);
     const float sx = __ldg(a.act_scale);
     const bool leader = threadIdx.x == 0;
-    const int nsteps = a.ktiles * 4;
-    int sc = 0;
+    int sc = 0;  // buffer uses drained so far (K-tiles when folded, steps otherwise)
     bool ok = true;
     for (int tl = 0; tl < my_tiles; ++tl) {
       int gi, m0;
@@ -406,16 +444,13 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       tile_coords4(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
       const int m = m0 + t;
       const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
-      // alphas of step gs: groups 4 gs .. 4 gs + 3 (16-byte aligned: ng is a multiple of 16)
-      const float4* arow = reinterpret_cast<const float4*>(a.alpha + (int64_t)(mok ? m : 0) * g.ng);
+      const int64_t pw = p0 + 32 * hsub;  // this warp's first position
       float acc[32];
 #pragma unroll
       for (int i = 0; i < 32; ++i) acc[i] = 0.0f;
-      float4 al_next = mok ? __ldg(arow) : make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int gs = 0; gs < nsteps; ++gs, ++sc) {
+      const int ndrain = FOLD ? a.ktiles : a.ktiles * 4;
+      for (int u = 0; u < ndrain; ++u, ++sc) {
         if (!ok) continue;
-        const float4 al = al_next;
-        if (mok && gs + 1 < nsteps) al_next = __ldg(arow + gs + 1);
         const int b = sc & 1;
         if (!mbar_wait_timed(&acc_full[b], (sc >> 1) & 1, tmo, abort_flag, 0)) {
           ok = false;
@@ -425,10 +460,25 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         // slot j at columns 64 j .. 64 j + 63; this warp's 32 positions at + 32 hsub
         const uint32_t ta = tbase + (uint32_t)(b * 256);
         uint32_t r0[32], r1[32];
-        if (SUMS) {
-          // exact sums of groups 4 gs + j, filter m, positions p0 + 32 hsub + i
-          const int64_t pw = p0 + 32 * hsub;
-          int32_t* s0 = a.sums + ((int64_t)(mok ? m : 0) * g.ng + 4 * gs) * g.P;
+        if (FOLD) {
+          tmem_ld32(ta, r0);
+          tmem_ld32(ta + 64, r1);
+          tmem_ld_wait_regs(r0);
+          reg_fence(r1);
+          add32(acc, r0);
+          tmem_ld32(ta + 128, r0);
+          add32(acc, r1);
+          tmem_ld32(ta + 192, r1);
+          tmem_ld_wait_regs(r0);
+          reg_fence(r1);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);  // every column of the K-tile is in registers
+          add32(acc, r0);
+          add32(acc, r1);
+        } else {
+          // exact sums of groups 4 u + j, filter m, positions pw + i
+          int32_t* s0 = a.sums + ((int64_t)(mok ? m : 0) * g.ng + 4 * u) * g.P;
 #pragma unroll
           for (int hh = 0; hh < 2; ++hh) {
             tmem_ld32(ta + 128 * hh, r0);
@@ -451,51 +501,42 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
               }
             }
           }
-          continue;
         }
-        tmem_ld32(ta, r0);
-        tmem_ld32(ta + 64, r1);
-        tmem_ld_wait_regs(r0);
-        reg_fence(r1);
-        scale_add(acc, r0, al.x);
-        tmem_ld32(ta + 128, r0);
-        scale_add(acc, r1, al.y);
-        tmem_ld32(ta + 192, r1);
-        tmem_ld_wait_regs(r0);
-        reg_fence(r1);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&acc_empty[b]);
-        scale_add(acc, r0, al.z);
-        scale_add(acc, r1, al.w);
       }
       if (!ok && !*abort_flag) fail();
       if (named_bar_or(BAR_EPI4, 32 * T4_EPI_WARPS, !ok)) break;
-      if (SUMS) continue;  // the group sums are stored already
+      if (!FOLD) continue;  // the group sums are stored already
+      const float sc_m = mok ? sx * __ldg(a.row_scale + m) : 0.0f;
       if (a.out_tma) {
-        if (leader) bulk_wait_read_all();  // the previous tile's store has read the buffer
-        named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
+        // two boxes of 32 positions, each written by the warps of its half, stored by one thread
+#pragma unroll 1
+        for (int hb = 0; hb < 2; ++hb) {
+          if (leader) bulk_wait_read_all();  // the previous box has been read out
+          named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
+          if (hsub == hb) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) otile[(32 * hsub + i) * T4_BM + t] = sx * acc[i];
-        fence_proxy_async_smem();
-        named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
-        if (leader) {
-          tma_store_2d(&a.out_map, m0, (int)p0, smem_u32(otile));
-          bulk_commit();
+            for (int i = 0; i < 32; ++i) otile[i * T4_BM + t] = sc_m * acc[i];
+          }
+          fence_proxy_async_smem();
+          named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
+          if (leader) {  // a box that starts inside the output (its tail past P is not written)
+            if (p0 + 32 * hb < g.P) tma_store_2d(&a.out_map, m0, (int)(p0 + 32 * hb), smem_u32(otile));
+            bulk_commit();
+          }
         }
       } else if (mok) {
         if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
           const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const int64_t p = p0 + 32 * hsub + i;
-            if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sx * acc[i], r);
+            const int64_t p = pw + i;
+            if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sc_m * acc[i], r);
           }
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const int64_t p = p0 + 32 * hsub + i;
-            if (p < g.P) a.out[p * g.M + m] = sx * acc[i];
+            const int64_t p = pw + i;
+            if (p < g.P) a.out[p * g.M + m] = sc_m * acc[i];
           }
         }
       }
@@ -511,20 +552,21 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   }
 }
 
-template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
+template <int ABITS, bool SIGNED, bool TMAP, bool FOLD>
 fgq_status launch_tc4(const T4Args& args, int grid, cudaStream_t s) {
-  if (!tc::smem_attr_once<tc4_contract_kernel<ABITS, SIGNED, TMAP, SUMS>>(T4_SMEM)) return FGQ_ERR_CUDA;
-  tc4_contract_kernel<ABITS, SIGNED, TMAP, SUMS><<<grid, T4_THREADS, T4_SMEM, s>>>(args);
+  constexpr int smem = T4Cfg<FOLD>::SMEM;
+  if (!tc::smem_attr_once<tc4_contract_kernel<ABITS, SIGNED, TMAP, FOLD>>(smem)) return FGQ_ERR_CUDA;
+  tc4_contract_kernel<ABITS, SIGNED, TMAP, FOLD><<<grid, T4_THREADS, smem, s>>>(args);
   return after_launch();
 }
 
 template <int ABITS, bool SIGNED>
 fgq_status launch_tc4_path(const T4Args& args, int grid, cudaStream_t s) {
   if (args.sums)
-    return args.act_tma ? launch_tc4<ABITS, SIGNED, true, true>(args, grid, s)
-                        : launch_tc4<ABITS, SIGNED, false, true>(args, grid, s);
-  return args.act_tma ? launch_tc4<ABITS, SIGNED, true, false>(args, grid, s)
-                      : launch_tc4<ABITS, SIGNED, false, false>(args, grid, s);
+    return args.act_tma ? launch_tc4<ABITS, SIGNED, true, false>(args, grid, s)
+                        : launch_tc4<ABITS, SIGNED, false, false>(args, grid, s);
+  return args.act_tma ? launch_tc4<ABITS, SIGNED, true, true>(args, grid, s)
+                      : launch_tc4<ABITS, SIGNED, false, true>(args, grid, s);
 }
 
 }  // namespace
@@ -545,7 +587,6 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   T4Args a;
   memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
-  a.alpha = alpha;
   a.act_scale = act_scale;
   a.out = out;
   a.sums = sums;
@@ -559,19 +600,33 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   const int64_t lim_us = debug_wait_limit_us();
   a.timeout_ns = lim_us < 0 ? T4_TIMEOUT_NS : (uint64_t)lim_us * 1000u;
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
+  const bool fold = sums == nullptr;
 
-  // expanded codes: fp16 [M][Kp] (Kp = 16 wrow), in a temporary from the stream-ordered pool
+  // the ternary operand, fp16 [M][Kp] (Kp = 16 wrow) per part, and (folded) the row scales,
+  // in one temporary from the stream-ordered pool
   cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
-  const int64_t nwords = (int64_t)g.M * g.wrow;
-  void* a16 = nullptr;
-  if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 32, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
-  expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
-  fgq_status st = after_launch();
-  if (st == FGQ_OK &&
-      !make_map_2d(&a.a16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a16, (uint64_t)g.wrow * 16, (uint64_t)g.M,
-                   (uint64_t)g.wrow * 32, T4_KT, T4_BM, CU_TENSOR_MAP_SWIZZLE_128B))
-    st = FGQ_ERR_CUDA;
+  const size_t part_bytes = (size_t)g.M * g.wrow * 32;
+  const int nparts = fold ? 2 : 1;
+  void* tmp = nullptr;
+  if (cudaMallocFromPoolAsync(&tmp, nparts * part_bytes + (fold ? (size_t)g.M * 4 : 0), pool, s) != cudaSuccess)
+    return FGQ_ERR_CUDA;
+  uint8_t* parts = static_cast<uint8_t*>(tmp);
+  fgq_status st;
+  if (fold) {
+    float* rs = reinterpret_cast<float*>(parts + 2 * part_bytes);
+    a.row_scale = rs;
+    st = launch_fold_alpha_split(codes, g.M, g.wrow, g.G, g.ng, alpha, parts, parts + part_bytes, rs, s);
+  } else {
+    const int64_t nwords = (int64_t)g.M * g.wrow;
+    expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, reinterpret_cast<uint4*>(parts));
+    st = after_launch();
+  }
+  for (int part = 0; st == FGQ_OK && part < nparts; ++part)
+    if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, parts + part * part_bytes,
+                     (uint64_t)g.wrow * 16, (uint64_t)g.M, (uint64_t)g.wrow * 32, T4_KT, T4_BM,
+                     CU_TENSOR_MAP_SWIZZLE_128B))
+      st = FGQ_ERR_CUDA;
   if (st == FGQ_OK && g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
     const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
     a.act_tma = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, row_bytes, (uint64_t)g.B * g.H * g.W,
@@ -580,9 +635,9 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
                     ? 1
                     : 0;
   }
-  if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums) {
+  if (st == FGQ_OK && fold && g.groups == 1 && g.M % 4 == 0 && !g.rq_out) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
-                            (uint64_t)g.M * 4, T4_BM, T4_BP, CU_TENSOR_MAP_SWIZZLE_NONE)
+                            (uint64_t)g.M * 4, T4_BM, 32, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1
                     : 0;
   }
@@ -598,7 +653,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
       st = sgn ? launch_tc4_path<8, true>(a, grid, s) : launch_tc4_path<8, false>(a, grid, s);
   }
   // the temporary returns to the pool once the work queued on s before this point is done
-  if (cudaFreeAsync(a16, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  if (cudaFreeAsync(tmp, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
   return st;
 }
 

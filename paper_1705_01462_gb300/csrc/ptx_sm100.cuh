@@ -80,15 +80,22 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 }
 
 // Waits for the phase with the given parity for at most timeout_ns of global time (and at
-// most 2^26 polls), sleeping sleep_ns between polls (0: poll back to back); returns false
-// on expiry or once *abort becomes non-zero.
+// most 2^26 polls), sleeping sleep_ns between polls (0: each poll instead suspends the thread
+// in hardware until the phase completes or about 1 us passes, so a waiting warp takes no
+// issue slots); returns false on expiry or once *abort becomes non-zero.  timeout_ns = 0
+// (a test's forced expiry) passes only a phase already complete at the first test.
 __device__ __forceinline__ bool mbar_wait_timed(uint64_t* bar, uint32_t parity, uint64_t timeout_ns,
                                                 volatile uint32_t* abort, uint32_t sleep_ns) {
   if (mbar_try_wait(bar, parity)) return true;
+  if (timeout_ns == 0) return false;  // a zero limit passes only a phase already complete
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1; i < (1u << 26); ++i) {
-    if (sleep_ns) __nanosleep(sleep_ns);
-    if (mbar_try_wait(bar, parity)) return true;
+    if (sleep_ns) {
+      __nanosleep(sleep_ns);
+      if (mbar_try_wait(bar, parity)) return true;
+    } else if (mbar_try_wait_sleep(bar, parity, 1000u)) {
+      return true;
+    }
     if ((i & 7u) == 0) {
       if (*abort) return false;
       if (globaltimer_ns() - t0 > timeout_ns) return false;
@@ -159,7 +166,36 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : "r"(taddr)
       : "memory");
 }
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// Waits for this thread's TMEM loads, with r as in/out operands so that no use of r is
+// placed before the wait (16-register form).
+__device__ __forceinline__ void tmem_ld_wait_regs16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15])
+               :
+               : "memory");
+}
+// Orders every later use of r after this point (no instruction), 16-register form.
+__device__ __forceinline__ void reg_fence16(uint32_t (&r)[16]) {
+  asm volatile(""
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15])
+               :
+               : "memory");
+}
 // Waits for this thread's TMEM loads, with r as in/out operands so that no use of r is
 // placed before the wait.
 __device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
