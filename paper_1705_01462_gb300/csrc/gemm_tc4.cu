@@ -64,13 +64,15 @@ using tc::u8pair_to_h2;
 constexpr int T4_BM = 128;      // filters per tile (MMA M, TMEM lanes)
 constexpr int T4_BP = 64;       // positions per tile
 constexpr int T4_KT = 64;       // reduction elements per K-tile: 16 groups, 4 MMA steps
-constexpr int T4_NO = 3;        // operand ring depth
+constexpr int T4_NB = 2;        // B' (activation operand) ring depth
+constexpr int T4_NAS = 4;       // A (ternary operand) ring depth
 constexpr int T4_NACC = 2;      // TMEM buffers of 256 columns
 constexpr int T4_EPI_WARPS = 8;
 constexpr int T4_LOAD_WARP0 = 8;  // loaders: warps 8-11
 constexpr int T4_LOADERS = 128;
 constexpr int T4_MMA_WARP = 12;
-constexpr int T4_THREADS = 32 * (T4_MMA_WARP + 1);
+constexpr int T4_A_WARP = 13;     // lane 0 streams the A boxes
+constexpr int T4_THREADS = 32 * (T4_A_WARP + 1);
 constexpr int T4_TMEM_COLS = T4_NACC * 256;
 constexpr uint64_t T4_TIMEOUT_NS = 1000000000ull;  // 1 s per wait
 constexpr uint32_t T4_DRAIN_LIMIT = 1u << 20;      // polls of the final drains (never shortened)
@@ -81,20 +83,21 @@ constexpr int B_TILE4 = 256 * T4_KT * 2;      // 32 KB fp16 block-diagonal activ
 constexpr int ST_STAGE4 = T4_BP * T4_KT;      // 4 KB: 64 raw activation rows (8-bit: 64 B each)
 constexpr int OUT_BOX4 = 32 * T4_BM * 4;      // 16 KB fp32 [32 positions][128 filters]
 
-// Shared-memory plan of a variant: operand stages (A parts + B'), staging ring, output box.
+// Shared-memory plan of a variant: A ring (the ternary operand's parts), B' ring, staging
+// ring, output box, barriers.
 template <bool FOLD>
 struct T4Cfg {
   static constexpr int NPART = FOLD ? 2 : 1;
   static constexpr int A_STAGE = NPART * A_TILE4;
-  static constexpr int OP_STAGE = A_STAGE + B_TILE4;
   static constexpr int NS = FOLD ? 4 : 6;  // staging ring depth
   static constexpr int OUT = FOLD ? OUT_BOX4 : 0;
-  static constexpr int BAR = 8 * (3 * T4_NO + 2 * NS + 2 * T4_NACC + 1) + 16;
-  static constexpr int SMEM = 1024 + T4_NO * OP_STAGE + NS * ST_STAGE4 + OUT + BAR;
+  static constexpr int SMEM_A = T4_NAS * A_STAGE;
+  static constexpr int SMEM_B = T4_NB * B_TILE4;
+  static constexpr int BAR = 8 * (2 * T4_NAS + 2 * T4_NB + 2 * NS + 2 * T4_NACC + 1) + 16;
+  static constexpr int SMEM = 1024 + SMEM_A + SMEM_B + NS * ST_STAGE4 + OUT + BAR;
 };
 static_assert(T4Cfg<true>::SMEM <= 232448 && T4Cfg<false>::SMEM <= 232448, "shared memory budget");
-static_assert(ST_STAGE4 % 1024 == 0 && T4Cfg<true>::OP_STAGE % 1024 == 0 && T4Cfg<false>::OP_STAGE % 1024 == 0,
-              "stage alignment");
+static_assert(ST_STAGE4 % 1024 == 0 && A_TILE4 % 1024 == 0 && B_TILE4 % 1024 == 0, "stage alignment");
 
 struct T4Args {
   CUtensorMap a_map[2];   // fp16 [M][Kp] ternary operand parts (folded hi, lo; or codes), box {64, 128 rows},
@@ -154,14 +157,16 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   constexpr int NS = Cfg::NS;
   extern __shared__ uint8_t smem_raw4[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw4) + 1023) & ~uintptr_t(1023));
-  uint8_t* op = smem;
-  uint8_t* st = smem + T4_NO * Cfg::OP_STAGE;
+  uint8_t* abuf = smem;
+  uint8_t* bbuf = smem + Cfg::SMEM_A;
+  uint8_t* st = bbuf + Cfg::SMEM_B;
   float* otile = reinterpret_cast<float*>(st + NS * ST_STAGE4);
   uint64_t* bars = reinterpret_cast<uint64_t*>(st + NS * ST_STAGE4 + Cfg::OUT);
-  uint64_t* op_full = bars;
-  uint64_t* op_empty = bars + T4_NO;
-  uint64_t* a_full = bars + 2 * T4_NO;
-  uint64_t* st_full = bars + 3 * T4_NO;
+  uint64_t* a_full = bars;
+  uint64_t* a_empty = bars + T4_NAS;
+  uint64_t* op_full = bars + 2 * T4_NAS;
+  uint64_t* op_empty = op_full + T4_NB;
+  uint64_t* st_full = op_empty + T4_NB;
   uint64_t* st_empty = st_full + NS;
   uint64_t* acc_full = st_empty + NS;
   uint64_t* acc_empty = acc_full + T4_NACC;
@@ -175,10 +180,13 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   const uint64_t tmo = a.timeout_ns;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < T4_NO; ++i) {
+    for (int i = 0; i < T4_NAS; ++i) {
+      mbar_init(&a_full[i], 1);   // the A boxes' byte count
+      mbar_init(&a_empty[i], 1);  // released by the epilogue once the K-tile's MMAs completed
+    }
+    for (int i = 0; i < T4_NB; ++i) {
       mbar_init(&op_full[i], T4_LOADERS);  // B' pieces
-      mbar_init(&op_empty[i], 1);
-      mbar_init(&a_full[i], 1);            // the A boxes' byte count
+      mbar_init(&op_empty[i], 1);          // released like a_empty
     }
     for (int i = 0; i < NS; ++i) {
       mbar_init(&st_full[i], TMAP ? 1 : T4_LOADERS);
@@ -193,8 +201,8 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     fence_mbar_init();
   }
   // the off-diagonal zeros of every B' tile, written once
-  for (int s = 0; s < T4_NO; ++s) {
-    uint4* bt = reinterpret_cast<uint4*>(op + s * Cfg::OP_STAGE + Cfg::A_STAGE);
+  for (int s = 0; s < T4_NB; ++s) {
+    uint4* bt = reinterpret_cast<uint4*>(bbuf + s * B_TILE4);
     for (int i = threadIdx.x; i < B_TILE4 / 16; i += blockDim.x) bt[i] = make_uint4(0u, 0u, 0u, 0u);
   }
   fence_proxy_async_smem();
@@ -228,7 +236,7 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     int64_t p0 = 0;
     int pb = 0, phb = 0, pwb = 0;
     bool pvalid = false;
-    int issued = 0, a_armed = 0;
+    int issued = 0;
     // activation copies of K-tile j (of this CTA's sequence) into staging slot j % NS
     auto issue = [&](int j) -> bool {
       const int tl = j / a.ktiles;
@@ -298,24 +306,12 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         break;
       }
       const int slot = j % NS;
-      const int os = j % T4_NO;
-      if (!mbar_wait_timed(&op_empty[os], ((j / T4_NO) & 1) ^ 1, tmo, abort_flag, 64)) {
+      const int os = j % T4_NB;
+      if (!mbar_wait_timed(&op_empty[os], ((j / T4_NB) & 1) ^ 1, tmo, abort_flag, 64)) {
         ok = false;
         break;
       }
-      uint8_t* A = op + os * Cfg::OP_STAGE;
-      uint8_t* Bt = A + Cfg::A_STAGE;
-      if (t == 0) {  // the A boxes of K-tile j: the tile's 128 filter rows, per part
-        const int tl = j / a.ktiles;
-        int gj, mj;
-        int64_t pj;
-        tile_coords4(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
-        mbar_arrive_expect_tx(&a_full[os], Cfg::A_STAGE);
-#pragma unroll
-        for (int part = 0; part < Cfg::NPART; ++part)
-          tma_load_2d(smem_u32(A + part * A_TILE4), &a.a_map[part], (j - tl * a.ktiles) * T4_KT, mj, &a_full[os]);
-        a_armed = j + 1;
-      }
+      uint8_t* Bt = bbuf + os * B_TILE4;
       if (!mbar_wait_timed(&st_full[slot], (j / NS) & 1, tmo, abort_flag, 32)) {
         ok = false;
         break;
@@ -369,31 +365,53 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     if (TMAP && t == 0) {
       for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % NS], (j / NS) & 1, T4_DRAIN_LIMIT);
     }
-    if (t == 0 && !ok) {
-      // A boxes the MMA issuer may not have consumed: the last T4_NO armed ones, one per
-      // stage, each the latest phase of its stage's barrier
-      for (int j = a_armed - T4_NO < 0 ? 0 : a_armed - T4_NO; j < a_armed; ++j)
-        mbar_wait_bounded(&a_full[j % T4_NO], (j / T4_NO) & 1, T4_DRAIN_LIMIT);
+  }
+
+  // ------------------------------------------------------------------ A boxes
+  if (warp == T4_A_WARP && lane == 0) {
+    const int total = my_tiles * a.ktiles;
+    int armed = 0;
+    bool ok = true;
+    for (int j = 0; j < total; ++j) {
+      const int as = j % T4_NAS;
+      if (!mbar_wait_timed(&a_empty[as], ((j / T4_NAS) & 1) ^ 1, tmo, abort_flag, 64)) {
+        ok = false;
+        break;
+      }
+      const int tl = j / a.ktiles;
+      int gj, mj;
+      int64_t pj;
+      tile_coords4(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
+      uint8_t* A = abuf + as * Cfg::A_STAGE;
+      mbar_arrive_expect_tx(&a_full[as], Cfg::A_STAGE);
+#pragma unroll
+      for (int part = 0; part < Cfg::NPART; ++part)
+        tma_load_2d(smem_u32(A + part * A_TILE4), &a.a_map[part], (j - tl * a.ktiles) * T4_KT, mj, &a_full[as]);
+      armed = j + 1;
     }
+    if (!ok && !*abort_flag) fail();
+    // boxes the MMA issuer may not have consumed: the last T4_NAS armed ones, one per stage,
+    // each the latest phase of its stage's barrier
+    for (int j = armed - T4_NAS < 0 ? 0 : armed - T4_NAS; j < armed; ++j)
+      mbar_wait_bounded(&a_full[j % T4_NAS], (j / T4_NAS) & 1, T4_DRAIN_LIMIT);
   }
 
   // ------------------------------------------------------------------ MMA issuer
   if (warp == T4_MMA_WARP && lane == 0) {
     const uint32_t idesc = idesc_f16_f32(128, 256);
-    const uint32_t op_base = smem_u32(op);
     const int total = my_tiles * a.ktiles;
     int sc = 0;  // group sums: steps issued
     bool ok = true;
     for (int j = 0; j < total && ok; ++j) {
-      const int os = j % T4_NO;
-      if (!mbar_wait_timed(&op_full[os], (j / T4_NO) & 1, tmo, abort_flag, 0) ||
-          !mbar_wait_timed(&a_full[os], (j / T4_NO) & 1, tmo, abort_flag, 0)) {
+      const int os = j % T4_NB, as = j % T4_NAS;
+      if (!mbar_wait_timed(&op_full[os], (j / T4_NB) & 1, tmo, abort_flag, 0) ||
+          !mbar_wait_timed(&a_full[as], (j / T4_NAS) & 1, tmo, abort_flag, 0)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t abase = op_base + os * Cfg::OP_STAGE;
-      const uint64_t bd = sdesc_k_sw128(abase + Cfg::A_STAGE);
+      const uint32_t abase = smem_u32(abuf + as * Cfg::A_STAGE);
+      const uint64_t bd = sdesc_k_sw128(smem_u32(bbuf + os * B_TILE4));
       if (FOLD) {
         // the K-tile's 8 MMAs (4 steps x 2 parts) accumulate into buffer j % 2
         const int b = j & 1;
@@ -422,7 +440,8 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
           mma_commit(&acc_full[b]);
         }
       }
-      mma_commit(&op_empty[os]);
+      // the operand stages are released by the epilogue, which sees the K-tile's last
+      // accumulator commit (one commit per buffer use, none spent on the stages)
     }
     if (!ok && !*abort_flag) fail();
     mma_commit(drain_bar);
@@ -455,6 +474,12 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
         if (!mbar_wait_timed(&acc_full[b], (sc >> 1) & 1, tmo, abort_flag, 0)) {
           ok = false;
           continue;
+        }
+        if (leader && (FOLD || (u & 3) == 3)) {
+          // the K-tile's MMAs have completed: its A and B' stages may be refilled
+          const int kt = FOLD ? sc : sc >> 2;
+          mbar_arrive(&a_empty[kt % T4_NAS]);
+          mbar_arrive(&op_empty[kt % T4_NB]);
         }
         tc_fence_after();
         // slot j at columns 64 j .. 64 j + 63; this warp's 32 positions at + 32 hsub
