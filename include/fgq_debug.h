@@ -21,7 +21,7 @@ typedef enum {
   FGQ_PATH_AUTO = 0,   /* choose per shape: the few-row path for small GEMMs; with
                           fixed-point alphas the dense tensor-core path where it applies;
                           else the tensor cores where the shape is covered (G = 4 only with
-                          at least 128 filters per conv group), else the CUDA cores */
+                          at least 64 filters per conv group), else the CUDA cores */
   FGQ_PATH_SIMT = 1,   /* CUDA-core path: dp4a group sums, one FMA per group */
   FGQ_PATH_TC = 2,     /* tensor-core path (tcgen05): G in {64, 128} with K-tiles aligned to
                           the group; G = 4 with a block-diagonal activation operand

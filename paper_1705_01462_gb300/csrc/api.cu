@@ -67,6 +67,11 @@ bool tc_any(const Geom& g) { return g.G == 4 ? tc4_supports(g) : tc_supports(g);
 
 bool gemv_any(const Geom& g) { return !g.is_conv && gemv_supports((int)g.P, g.Kred, g.G, g.act_type); }
 
+// Fewest filters per conv group for which the automatic choice sends a G = 4 layer to the
+// tensor cores (a 64-filter layer fills half of the 128-row tile and still runs at about
+// twice the dp4a kernel's rate).
+constexpr int T4_MIN_FILTERS = 64;
+
 int choose_path(const Geom& g, bool sums, bool qa) {
   const int forced = t_path;
   if (sums) {
@@ -75,7 +80,7 @@ int choose_path(const Geom& g, bool sums, bool qa) {
     if (forced == FGQ_PATH_GEMV || forced == FGQ_PATH_DENSE) return -1;
     if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
     if (forced == FGQ_PATH_TC) return tc_any(g) ? FGQ_PATH_TC : -1;
-    if (g.G == 4 && g.Mg < 128) return FGQ_PATH_SIMT;
+    if (g.G == 4 && g.Mg < T4_MIN_FILTERS) return FGQ_PATH_SIMT;
     return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
   }
   if (forced == FGQ_PATH_SIMT) return FGQ_PATH_SIMT;
@@ -88,9 +93,9 @@ int choose_path(const Geom& g, bool sums, bool qa) {
   // fixed-point alphas fold exactly into fp16 weights: one dense tensor-core contraction
   if (qa && dense_supports(g)) return FGQ_PATH_DENSE;
   // automatic choice: the tensor cores where the shape is covered, except G = 4 layers with
-  // fewer than 128 filters per conv group, where the 128-row MMA tile would leave half its
-  // rows idle and the dp4a kernel is faster
-  if (g.G == 4 && g.Mg < 128) return FGQ_PATH_SIMT;
+  // fewer than T4_MIN_FILTERS filters per conv group, where most rows of the 128-row MMA
+  // tile would sit idle and the dp4a kernel is faster
+  if (g.G == 4 && g.Mg < T4_MIN_FILTERS) return FGQ_PATH_SIMT;
   return tc_any(g) ? FGQ_PATH_TC : FGQ_PATH_SIMT;
 }
 

@@ -50,7 +50,7 @@ def _paths(G, Mg, Kg):
     tc_ok = G in (4, 64, 128) and Kg % 64 == 0
     if tc_ok:
         out.append((fgq.PATH_TC, fgq.PATH_TC))
-    auto = fgq.PATH_TC if tc_ok and not (G == 4 and Mg < 128) else fgq.PATH_SIMT
+    auto = fgq.PATH_TC if tc_ok and not (G == 4 and Mg < 64) else fgq.PATH_SIMT
     out.append((fgq.PATH_AUTO, auto))
     return out
 
