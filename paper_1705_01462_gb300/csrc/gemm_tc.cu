@@ -21,16 +21,21 @@
 //              fp32 registers.  At tile end the fp32 tile goes to shared memory and one
 //              thread writes it to HBM with a TMA box store (direct stores when the
 //              output has several conv groups or M % 4 != 0).
-//   warps 8-11 loaders/converters: per K-tile one thread issues a TMA box load of the
-//              tile's 128 code rows (16 bytes each) and, for layers whose im2col rows are
-//              contiguous input rows (1x1 stride-1 convolutions, GEMMs), one TMA box load
-//              of the 128 activation rows; for other layers each thread copies its own
-//              activation row and code row with 16-byte cp.async.  Thread t converts row t of both
-//              tiles to fp16 in the 128-byte-swizzled K-major layout the MMA reads; a
-//              staging slot is refilled by TMA only after every loader has released it
-//              (st_empty), so the loader warps never wait for each other otherwise.
+//   warps 8-11 loaders/converters: for layers whose im2col rows are contiguous input rows
+//              (1x1 stride-1 convolutions, GEMMs) one thread issues a TMA box load of the
+//              K-tile's 128 activation rows; for other layers each thread copies its own
+//              row with 16-byte cp.async.  Thread t converts row t to fp16 in the
+//              128-byte-swizzled K-major layout the MMA reads; a staging slot is refilled
+//              by TMA only after every loader has released it (st_empty), so the loader
+//              warps never wait for each other otherwise.
 //   warp 12    TMEM allocation and the MMA issuer (one thread): 4 tcgen05.mma (K = 16)
 //              per K-tile into one of four 128-column TMEM accumulators.
+//   warp 13    streams the ternary operand: the codes are expanded to fp16 {0, +1, -1} once
+//              per call (a stream-ordered temporary) and reach a four-stage ring of their own
+//              by TMA in the MMA's swizzled layout, ahead of the K-tiles that use them.
+// The operand stages are released by the epilogue: the group's accumulator commit (one per
+// group) is seen by epilogue thread 0, which frees the group's A and B stages, so no commit
+// is spent on them.
 // Every mbarrier wait is bounded; on expiry the kernel records FGQ_ERR_TIMEOUT, each role
 // leaves its loop (uniformly within a role that uses named barriers), in-flight copies
 // and MMAs are waited for, and TMEM is freed.
@@ -51,7 +56,8 @@ using tc::u8pair_to_h2;
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 128;        // positions per tile (MMA N)
 constexpr int TC_KT = 64;         // reduction elements per K-tile
-constexpr int TC_NO = 3;          // operand ring depth
+constexpr int TC_NO = 3;          // activation operand (B) ring depth
+constexpr int TC_NAS = 4;         // ternary operand (A) ring depth
 constexpr int TC_NS_TMA = 6;      // staging ring depth of the TMA path (room for the output tile)
 constexpr int TC_NS_GATHER = 12;  // staging ring depth of the gather path (about 1.5 us of copies)
 constexpr int TC_NACC = 4;        // TMEM accumulator buffers
@@ -61,8 +67,9 @@ constexpr int TC_LOADERS = 32 * TC_LOAD_WARPS;  // loader threads
 constexpr int TC_LPR = TC_LOADERS / 128;         // loader threads per tile row
 static_assert(TC_LPR == 1, "the cp.async gather path reads only copies made by the same thread");
 constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // loaders: warps 8 .. 8 + TC_LOAD_WARPS - 1
-constexpr int TC_MMA_WARP = TC_EPI_WARPS + TC_LOAD_WARPS;  // warp 16
-constexpr int TC_THREADS = 32 * (TC_MMA_WARP + 1);
+constexpr int TC_MMA_WARP = TC_EPI_WARPS + TC_LOAD_WARPS;  // warp 12
+constexpr int TC_A_WARP = TC_MMA_WARP + 1;                 // warp 13: lane 0 streams the A boxes
+constexpr int TC_THREADS = 32 * (TC_A_WARP + 1);
 constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
 constexpr uint32_t TC_WAIT_LIMIT = 50000;        // polls of up to 20 us: about 1 s per wait
 constexpr uint32_t TC_WAIT_SLEEP_NS = 20000;     // suspend hint of one poll
@@ -70,26 +77,23 @@ constexpr uint32_t TC_DRAIN_LIMIT = 1u << 20;    // polls of the final drains (n
 constexpr uint32_t BAR_EPI = 2;                  // named barrier of the 256 epilogue threads
 
 constexpr int OP_TILE = TC_BM * TC_KT * 2;            // 16 KB: one fp16 operand tile
-constexpr int OP_STAGE = 2 * OP_TILE;                  // A (codes) + B (activations)
-constexpr int ST_ACT = TC_BN * TC_KT;                  // 8 KB raw activation bytes (8-bit)
-constexpr int ST_CODE = TC_BM * 16;                    // 2 KB raw code words
-constexpr int ST_STAGE = ST_ACT + ST_CODE;
+constexpr int ST_STAGE = TC_BN * TC_KT;                // 8 KB raw activation bytes (8-bit)
 constexpr int OUT_TILE = TC_BN * TC_BM * 4;            // 64 KB fp32 output tile
-constexpr int SMEM_OP = TC_NO * OP_STAGE;
-constexpr int SMEM_LUT = 16 * 32 * 4;                  // 2 codes -> 2 fp16, one copy per bank
-constexpr int SMEM_BAR = 8 * (2 * TC_NO + 2 * TC_NS_GATHER + 2 * TC_NACC + 1) + 16;
+constexpr int SMEM_A = TC_NAS * OP_TILE;
+constexpr int SMEM_B = TC_NO * OP_TILE;
+constexpr int SMEM_BAR = 8 * (2 * TC_NAS + 2 * TC_NO + 2 * TC_NS_GATHER + 2 * TC_NACC + 1) + 16;
 // TMA path: staging ring + fp32 output tile; gather path: a deeper staging ring, no tile.
 constexpr int SMEM_MID_TMA = TC_NS_TMA * ST_STAGE + OUT_TILE;
 constexpr int SMEM_MID_GATHER = TC_NS_GATHER * ST_STAGE;
 constexpr int SMEM_MID = SMEM_MID_TMA > SMEM_MID_GATHER ? SMEM_MID_TMA : SMEM_MID_GATHER;
-constexpr int TC_SMEM = 1024 + SMEM_OP + SMEM_MID + SMEM_LUT + SMEM_BAR;
+constexpr int TC_SMEM = 1024 + SMEM_A + SMEM_B + SMEM_MID + SMEM_BAR;
+static_assert(TC_SMEM <= 232448, "shared memory budget");
 
 struct TcArgs {
-  CUtensorMap codes_map;  // uint32 [M][wrow], box {4 words, 128 rows}
+  CUtensorMap a16_map;    // fp16 [M][Kp] expanded codes, box {64, 128 rows}, 128-byte swizzle
   CUtensorMap act_map;    // uint8 [pixels][row bytes], box {64 (or 32) bytes, 128 rows}; if act_tma
   CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 128 positions}; if out_tma
   const uint8_t* act;
-  const uint32_t* codes;
   const float* alpha;
   const float* act_scale;
   float* out;
@@ -124,14 +128,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
   constexpr int TC_NS = TMAP ? TC_NS_TMA : TC_NS_GATHER;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* op = smem;                               // TC_NO x {A tile, B tile}
-  uint8_t* st = smem + SMEM_OP;                     // TC_NS x {act bytes, code bytes}
-  float* otile = reinterpret_cast<float*>(smem + SMEM_OP + TC_NS_TMA * ST_STAGE);  // TMA path: [128 pos][128 filters]
-  uint32_t* lut = reinterpret_cast<uint32_t*>(smem + SMEM_OP + SMEM_MID);  // [16][32]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_OP + SMEM_MID + SMEM_LUT);
-  uint64_t* op_full = bars;
-  uint64_t* op_empty = bars + TC_NO;
-  uint64_t* st_full = bars + 2 * TC_NO;
+  uint8_t* abuf = smem;                             // TC_NAS A tiles
+  uint8_t* bbuf = smem + SMEM_A;                    // TC_NO B tiles
+  uint8_t* st = bbuf + SMEM_B;                      // TC_NS activation staging slots
+  float* otile = reinterpret_cast<float*>(st + TC_NS_TMA * ST_STAGE);  // TMA path: [128 pos][128 filters]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(st + SMEM_MID);
+  uint64_t* a_full = bars;
+  uint64_t* a_empty = bars + TC_NAS;
+  uint64_t* op_full = bars + 2 * TC_NAS;
+  uint64_t* op_empty = op_full + TC_NO;
+  uint64_t* st_full = op_empty + TC_NO;
   uint64_t* st_empty = st_full + TC_NS;
   uint64_t* acc_full = st_empty + TC_NS;
   uint64_t* acc_empty = acc_full + TC_NACC;
@@ -144,9 +150,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
   const Geom& g = a.g;
 
   if (threadIdx.x == 0) {
+    for (int i = 0; i < TC_NAS; ++i) {
+      mbar_init(&a_full[i], 1);   // the A box's byte count
+      mbar_init(&a_empty[i], 1);  // released by the epilogue (the group's MMAs completed)
+    }
     for (int i = 0; i < TC_NO; ++i) {
       mbar_init(&op_full[i], TC_LOADERS);
-      mbar_init(&op_empty[i], 1);
+      mbar_init(&op_empty[i], 1);  // released like a_empty
     }
     for (int i = 0; i < TC_NS; ++i) {
       mbar_init(&st_full[i], 1);
@@ -160,7 +170,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     *abort_flag = 0;
     fence_mbar_init();
   }
-  tc::fill_code_lut(lut);
   if (warp == TC_MMA_WARP) {
     tmem_alloc(tmem_slot, TC_TMEM_COLS);
     tmem_relinquish();
@@ -185,7 +194,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     constexpr int ROW_BYTES = TC_KT * ABITS / 8;     // 64 (8-bit) or 32 (4-bit)
     constexpr int CPR = ROW_BYTES / 16;              // 16-byte chunks per activation row
     constexpr int HC = CPR / TC_LPR;                 // activation chunks this thread handles
-    constexpr uint32_t TX_CODES = TC_BM * 16;
     constexpr uint32_t TX_ACT = TC_BN * ROW_BYTES;
 
     // per-tile state: conv group, first filter, this thread's row position; the filter
@@ -213,17 +221,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       }
       const int slot = j % TC_NS;
       uint8_t* sa = st + slot * ST_STAGE;
-      const int kk = j - tl * a.ktiles;
       if (TMAP && tid == 0) {
         // the slot's previous contents (K-tile j - TC_NS) have been released by every thread
         bool free_ok = true;
         if (j >= TC_NS)
           free_ok = mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns);
         if (free_ok) {
-          mbar_arrive_expect_tx(&st_full[slot], TX_CODES + (TMAP ? TX_ACT : 0u));
-          tma_load_2d(smem_u32(sa + ST_ACT), &a.codes_map, kk * (TC_KT / 16), m0, &st_full[slot]);
-          if (TMAP)
-            tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
+          mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
+          tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
           issued = j + 1;
         } else {
           if (!*abort_flag) fail();
@@ -245,13 +250,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
           const int ch = h * HC + c;
           cp_async16(smem_u32(sa + st_off<ABITS>(t, ch)), inside ? (const void*)(src + 16 * ch) : (const void*)a.act,
                      inside ? 16u : 0u);
-        }
-        // this thread's part of code row t (filter m0 + t): 16 / TC_LPR bytes of 4 code words
-        const int m = m0 + t;
-        const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
-        if (TC_LPR == 1 || h == 0) {
-          const uint32_t* csrc = mok ? a.codes + (int64_t)m * g.wrow + kk * (TC_KT / 16) : a.codes;
-          cp_async16(smem_u32(sa + ST_ACT + t * 16), csrc, mok ? 16u : 0u);
         }
       }
       tc0 += TC_KT;  // next K-tile of this tile
@@ -277,17 +275,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       const int slot = j % TC_NS;
       const int os = j % TC_NO;
       if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) ||
-          !(a.kt_per_group > 1
-                ? mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)
-                : (j < TC_NO || mbar_wait_or_abort(&acc_full[(j - TC_NO) % TC_NACC], ((j - TC_NO) / TC_NACC) & 1,
-                                                   a.wait_limit, abort_flag, a.wait_sleep_ns)))) {
+          !mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
         if (!*abort_flag) fail();
         break;
       }
       consumed = j + 1;
       const uint8_t* sa = st + slot * ST_STAGE;
-      uint8_t* A = op + os * OP_STAGE;
-      uint8_t* Bt = A + OP_TILE;
+      uint8_t* Bt = bbuf + os * OP_TILE;
       // activations -> fp16 (this thread's part of row t of B)
       if (ABITS == 8) {
         const uint32_t bias2 = SIGNED ? 0x64806480u : 0x64006400u;  // 1152 or 1024 in both halves
@@ -332,22 +326,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         }
         }
       }
-      // codes -> fp16 (this thread's part of row t of A): 8 codes per 16-byte chunk, 2 per
-      // table lookup
-      {
-        constexpr int CC = 8 / TC_LPR;  // 16-byte fp16 chunks of A converted by this thread
-        uint32_t cw[CC / 2];
-#pragma unroll
-        for (int i = 0; i < CC / 2; ++i) cw[i] = *reinterpret_cast<const uint32_t*>(sa + ST_ACT + t * 16 + 4 * (i + (CC / 2) * h));
-        const uint32_t* lt = lut + lane;
-#pragma unroll
-        for (int cc = 0; cc < CC; ++cc) {
-          const uint32_t bits = (cw[cc / 2] >> (16 * (cc & 1))) & 0xffffu;  // 8 codes
-          *reinterpret_cast<uint4*>(A + sw128(t, CC * h + cc)) =
-              make_uint4(lt[32 * (bits & 15u)], lt[32 * ((bits >> 4) & 15u)], lt[32 * ((bits >> 8) & 15u)],
-                         lt[32 * (bits >> 12)]);
-        }
-      }
       fence_proxy_async_smem();
       mbar_arrive(&op_full[os]);
       if (TMAP) mbar_arrive(&st_empty[slot]);  // done reading this TMA-filled staging slot
@@ -360,10 +338,35 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     }
   }
 
+  // ------------------------------------------------------------------ A boxes
+  if (warp == TC_A_WARP && lane == 0) {
+    const int total = my_tiles * a.ktiles;
+    int armed = 0;
+    bool ok = true;
+    for (int j = 0; j < total; ++j) {
+      const int as = j % TC_NAS;
+      if (!mbar_wait_or_abort(&a_empty[as], ((j / TC_NAS) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
+        ok = false;
+        break;
+      }
+      const int tl = j / a.ktiles;
+      int gj, mj;
+      int64_t pj;
+      tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gj, mj, pj);
+      mbar_arrive_expect_tx(&a_full[as], OP_TILE);
+      tma_load_2d(smem_u32(abuf + as * OP_TILE), &a.a16_map, (j - tl * a.ktiles) * TC_KT, mj, &a_full[as]);
+      armed = j + 1;
+    }
+    if (!ok && !*abort_flag) fail();
+    // boxes the MMA issuer may not have consumed: the last TC_NAS armed ones, one per stage,
+    // each the latest phase of its stage's barrier
+    for (int j = armed - TC_NAS < 0 ? 0 : armed - TC_NAS; j < armed; ++j)
+      mbar_wait_bounded(&a_full[j % TC_NAS], (j / TC_NAS) & 1, TC_DRAIN_LIMIT);
+  }
+
   // ------------------------------------------------------------------ MMA issuer
   if (warp == TC_MMA_WARP && lane == 0) {
     const uint32_t idesc = idesc_f16_f32(TC_BM, TC_BN);
-    const uint32_t op_base = smem_u32(op);
     int kt = 0, gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
@@ -377,24 +380,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(b * TC_BN);
         for (int sub = 0; sub < a.kt_per_group; ++sub, ++kt) {
-          const int os = kt % TC_NO;
-          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
+          const int os = kt % TC_NO, as = kt % TC_NAS;
+          if (!mbar_wait_or_abort(&op_full[os], (kt / TC_NO) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns) ||
+              !mbar_wait_or_abort(&a_full[as], (kt / TC_NAS) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
             if (!*abort_flag) fail();
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t abase = op_base + os * OP_STAGE;
-          const uint64_t ad = sdesc_k_sw128(abase);
-          const uint64_t bd = sdesc_k_sw128(abase + OP_TILE);
+          const uint64_t ad = sdesc_k_sw128(smem_u32(abuf + as * OP_TILE));
+          const uint64_t bd = sdesc_k_sw128(smem_u32(bbuf + os * OP_TILE));
 #pragma unroll
           for (int k = 0; k < TC_KT / 16; ++k) {
             // advance 16 fp16 (32 bytes) along K inside the swizzled rows
             mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (sub > 0 || k > 0) ? 1u : 0u);
           }
-          // with one K-tile per group the group's acc_full commit also frees the operand
-          // stage (the loaders wait on it), so a second commit is not spent on op_empty
-          if (a.kt_per_group > 1) mma_commit(&op_empty[os]);
         }
         if (ok) mma_commit(&acc_full[b]);
       }
@@ -433,6 +433,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
           if (!*abort_flag) fail();
           ok = false;
           continue;
+        }
+        if (leader) {
+          // the group's MMAs have completed: its K-tiles' A and B stages may be refilled
+          for (int k = gc * a.kt_per_group; k < (gc + 1) * a.kt_per_group; ++k) {
+            mbar_arrive(&a_empty[k % TC_NAS]);
+            mbar_arrive(&op_empty[k % TC_NO]);
+          }
         }
         tc_fence_after();
         uint32_t r[32];
@@ -562,7 +569,6 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   TcArgs a;
   memset(&a, 0, sizeof a);
   a.act = static_cast<const uint8_t*>(act);
-  a.codes = codes;
   a.alpha = alpha;
   a.act_scale = act_scale;
   a.out = out;
@@ -579,9 +585,16 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   a.wait_limit = lim_us < 0 ? TC_WAIT_LIMIT : (uint32_t)(lim_us / 20 + 1);
   a.wait_sleep_ns = lim_us < 0 ? TC_WAIT_SLEEP_NS : (uint32_t)(lim_us < 20 ? lim_us * 1000 : 20000);
   const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
-  if (!make_map_2d(&a.codes_map, CU_TENSOR_MAP_DATA_TYPE_UINT32, codes, (uint64_t)g.wrow, (uint64_t)g.M,
-                   (uint64_t)g.wrow * 4, TC_KT / 16, TC_BM, CU_TENSOR_MAP_SWIZZLE_NONE))
-    return FGQ_ERR_CUDA;
+  // expanded codes: fp16 [M][Kp] (Kp = 16 wrow), in a temporary from the stream-ordered pool
+  cudaMemPool_t pool = scratch_pool();
+  if (!pool) return FGQ_ERR_CUDA;
+  const int64_t nwords = (int64_t)g.M * g.wrow;
+  void* a16 = nullptr;
+  if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 32, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
+  fgq_status st = launch_expand_codes(codes, nwords, a16, s);
+  if (st == FGQ_OK && !make_map_2d(&a.a16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a16, (uint64_t)g.wrow * 16,
+                                   (uint64_t)g.M, (uint64_t)g.wrow * 32, TC_KT, TC_BM, CU_TENSOR_MAP_SWIZZLE_128B))
+    st = FGQ_ERR_CUDA;
   // im2col rows are consecutive input rows for a 1x1, stride-1, unpadded convolution or a GEMM
   if (g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
     const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
@@ -602,8 +615,15 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = a.ntiles < sms ? a.ntiles : sms;
   const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
-  if (abits == 4) return sgn ? launch_tc_path<4, true>(a, grid, s) : launch_tc_path<4, false>(a, grid, s);
-  return sgn ? launch_tc_path<8, true>(a, grid, s) : launch_tc_path<8, false>(a, grid, s);
+  if (st == FGQ_OK) {
+    if (abits == 4)
+      st = sgn ? launch_tc_path<4, true>(a, grid, s) : launch_tc_path<4, false>(a, grid, s);
+    else
+      st = sgn ? launch_tc_path<8, true>(a, grid, s) : launch_tc_path<8, false>(a, grid, s);
+  }
+  // the temporary returns to the pool once the work queued on s before this point is done
+  if (cudaFreeAsync(a16, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
+  return st;
 }
 
 fgq_status launch_wait_timeout_selftest(uint32_t max_iter, unsigned int* err, cudaStream_t s) {

@@ -596,6 +596,12 @@ fgq_status launch_tc4_path(const T4Args& args, int grid, cudaStream_t s) {
 
 }  // namespace
 
+fgq_status launch_expand_codes(const uint32_t* codes, int64_t nwords, void* a16, cudaStream_t s) {
+  if (nwords <= 0) return FGQ_OK;
+  expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
+  return after_launch();
+}
+
 bool tc4_supports(const Geom& g) {
   if (g.G != 4) return false;
   if (g.Cg % T4_KT != 0) return false;        // every K-tile inside one filter tap (conv) or row (GEMM)
@@ -643,9 +649,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
     a.row_scale = rs;
     st = launch_fold_alpha_split(codes, g.M, g.wrow, g.G, g.ng, alpha, parts, parts + part_bytes, rs, s);
   } else {
-    const int64_t nwords = (int64_t)g.M * g.wrow;
-    expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, reinterpret_cast<uint4*>(parts));
-    st = after_launch();
+    st = launch_expand_codes(codes, (int64_t)g.M * g.wrow, parts, s);
   }
   for (int part = 0; st == FGQ_OK && part < nparts; ++part)
     if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, parts + part * part_bytes,
