@@ -24,6 +24,8 @@ The same JSON line carries the other workloads, each measured in the same run:
             16384} x batch {1, 64, 1024}.
 
 Usage:  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+        python bench.py --layer res3b_branch2b[,...] --G 4 [--batch B] [--path auto|simt|tc] [--iters n]
+        (single convolutions, one JSON line each: the calls profiler captures select)
 N > 1 runs under torchrun, one rank per GPU, each rank its own batch of 64 (weak scaling,
 no data-path collective).  --impl reference times the CPU oracle (the reference statement of
 the method) on a bounded sample of the same workload, over all host cores.
@@ -64,6 +66,13 @@ def parse(argv=None):
     ap.add_argument("--cpu-workers", type=int, default=0, help="oracle processes (0: every host core)")
     ap.add_argument("--no-configs", action="store_true", help="skip the other workloads (configs 1, 2, 4, 5)")
     ap.add_argument("--only", default="", help="profiling captures: run only 'step' (the timed steps)")
+    ap.add_argument("--layer", default="", help="time single convolutions instead: ResNet-50 layer names, comma "
+                                               "separated (per call, L2 flushed before each; for profiler captures)")
+    ap.add_argument("--G", type=int, default=4, help="group size of the --layer calls")
+    ap.add_argument("--act", default="u8", help="activation type of the --layer calls")
+    ap.add_argument("--path", default="auto", choices=["auto", "simt", "tc", "dense"],
+                    help="kernel family of the --layer calls")
+    ap.add_argument("--iters", type=int, default=5, help="timed calls per --layer layer")
     ap.add_argument("--batch", type=int, default=BATCH,
                     help="images per GPU (the benchmark workload is 64; smaller batches serve profiler "
                          "captures that must stay small)")
@@ -753,11 +762,66 @@ def run_reference(args, ws, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_layers(args):
+    """Times single convolutions of the ResNet-50 stack (fgq_conv2d through the C ABI, the
+    weights ternarized and the input quantized beforehand), the L2 flushed before each call;
+    prints one JSON line per layer."""
+    import torch
+    from paper_1705_01462_gb300 import fgq, synth
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    L = fgq.lib()
+    peaks = load_peaks()
+    layers = {l.name: (i, l) for i, l in enumerate(synth.resnet50_convs())}
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+    path = {"auto": fgq.PATH_AUTO, "simt": fgq.PATH_SIMT, "tc": fgq.PATH_TC, "dense": fgq.PATH_DENSE}[args.path]
+    B, G = args.batch, args.G
+    for name in args.layer.split(","):
+        i, l = layers[name]
+        w = synth.torch_weights(l, synth.layer_seed(i), dev)
+        x = synth.torch_activations((B, l.H, l.W, l.C), synth.layer_seed(i, 1), dev)
+        with torch.cuda.stream(stream):
+            codes, alpha = fgq.fgq_ternarize(w, G, stream=stream)
+            q, sx = fgq.fgq_quantize_act(x, args.act, stream=stream)
+        out = torch.empty((B, l.Ho, l.Wo, l.M), dtype=torch.float32, device=dev)
+        torch.cuda.synchronize()
+        fgq.fgq_set_path(path)
+
+        def call():
+            st = L.fgq_conv2d(q.data_ptr(), fgq.ACT_TYPES[args.act], sx.data_ptr(), B, l.H, l.W, l.C, l.R, l.S,
+                              l.stride, l.pad, l.groups, codes.data_ptr(), alpha.data_ptr(), l.M, G, out.data_ptr(),
+                              stream.cuda_stream)
+            if st != 0:
+                raise RuntimeError(f"fgq_conv2d {name}: {L.fgq_status_string(st).decode()}")
+        for _ in range(2):
+            call()
+        per = []
+        for _ in range(args.iters):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            per.append(e0.elapsed_time(e1))
+        check_status(fgq, stream, name)
+        ms = statistics.median(per)
+        r = conv_roofline([l], B, G, peaks, ms / 1e3, ACT_BITS[args.act])
+        print(json.dumps({"layer": name, "batch": B, "G": G, "act": args.act, "path": L.fgq_last_path(),
+                          "ms": round(ms, 5), "value": round(r["achieved"], 2), "unit": UNIT,
+                          "roofline_frac": round(r["frac"], 4), "bound": r["bound"]}), flush=True)
+        fgq.fgq_set_path(fgq.PATH_AUTO)
+
+
 def main():
     args = parse()
     ws, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, ws, rank)
+        return
+    if args.layer:
+        run_layers(args)
         return
     import torch
     from paper_1705_01462_gb300 import fgq

@@ -317,15 +317,18 @@ fgq_status fgq_quantize_alpha(const float* alpha, int M, int ng, int bits, uint8
 /*
  * fgq_gemm and fgq_conv2d with fixed-point alphas (aq, abits, ascale as produced by
  * fgq_quantize_alpha): the same contraction with alpha'[m][g] = aq[m][g] * ascale[m] (exact
- * in fp32).  On the few-row path (P <= 8, see FGQ_PATH_GEMV) the weights stream as 2-bit
+ * in fp32).  On the few-row path (P <= 8, see FGQ_PATH_GEMV in fgq_debug.h) the weights stream as 2-bit
  * codes plus 1 (or 1/2) byte per group instead of 4, and sum_g aq * s is accumulated
  * exactly in 64-bit integers: y = act_scale * ascale[m] * sum, rounded once.  Otherwise, with
  * 8-bit activations and Cg a multiple of 64, the automatic choice is the dense tensor-core
  * path (FGQ_PATH_DENSE): the integer weights aq * t are folded into an fp16 matrix in a pool
- * temporary (2 * M * Kp bytes) and one dense contraction sums them exactly while
- * |sum aq t q| < 2^24, again y = act_scale * ascale[m] * sum rounded once.  On the group-sum
+ * temporary (2 * M * Kp bytes) and one dense contraction sums the exact integer products in
+ * an fp32 accumulator: y = act_scale * ascale[m] * sum is the exact value rounded once when
+ * sum_k |aq t q| < 2^24 (which bounds every partial sum; e.g. always for Kred * 255 * 255 <
+ * 2^24), and otherwise within (Kp / 16) * 2^-23 * act_scale * ascale[m] * sum_k |aq t q| of it
+ * (the accumulator rounds at most once per 16 reduction elements).  On the group-sum
  * paths (forced, or shapes the dense path does not cover) the alphas are expanded to fp32
- * in a pool temporary (2-bit codes stay as they are).  Tolerance as fgq_gemm with alpha';
+ * in a pool temporary (2-bit codes stay as they are) and the fgq_gemm tolerance holds with alpha';
  * errors as fgq_gemm / fgq_conv2d, FGQ_ERR_ARG for abits not 8 or 4.
  */
 fgq_status fgq_gemm_qa(const void* q, fgq_act_type type, const float* act_scale, int P, int Kred,

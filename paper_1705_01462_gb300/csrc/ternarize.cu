@@ -370,6 +370,10 @@ struct TernBatch {
   int n;
   int64_t total;
 };
+// Passed by value as a __grid_constant__ kernel parameter: above the 4 KB limit of older
+// toolkits, within the 32,764-byte parameter space of CUDA 12.1 and later (the toolkit this
+// library is built with is 13.0).
+static_assert(sizeof(TernBatch) <= 32764, "kernel parameter space");
 
 __device__ __forceinline__ int batch_layer(const TernBatch& b, int64_t i) {
   int lo = 0, hi = b.n - 1;

@@ -57,3 +57,30 @@ def test_noalloc_matches_workspace_entry_point_twice():
     # and once more on the first input after the second call reused the scratch
     q3, sc3 = _noalloc(x1, fgq.U8)
     assert torch.equal(q3, results[0][0]) and sc3.item() == results[0][1].item()
+
+
+def test_noalloc_given_scale_and_host_errors():
+    """A given power-of-two scale (the branch that needs no scratch) matches the workspace
+    entry point bit for bit; argument and alignment errors are those of fgq_quantize_act."""
+    dev = torch.device("cuda:0")
+    g = torch.Generator(device=dev)
+    g.manual_seed(1462)
+    x = torch.randn(33_333, generator=g, device=dev) * 3.0
+    n = x.numel()
+    L = fgq.lib()
+    s = torch.cuda.current_stream().cuda_stream
+    for t in (fgq.U8, fgq.S8, fgq.S4):
+        q = torch.empty(fgq.act_bytes(n, t), dtype=torch.uint8, device=dev)
+        q_ref = torch.empty_like(q)
+        assert L.fgq_quantize_act_noalloc(x.data_ptr(), n, t, 2.0 ** -3, q.data_ptr(), None, s) == fgq.FGQ_OK
+        assert L.fgq_quantize_act(x.data_ptr(), n, t, 2.0 ** -3, q_ref.data_ptr(), None, None, 0, s) == fgq.FGQ_OK
+        torch.cuda.synchronize()
+        assert torch.equal(q, q_ref)
+    q = torch.empty(n + 64, dtype=torch.uint8, device=dev)
+    sc = torch.empty(4, dtype=torch.float32, device=dev)
+    # misaligned input: FGQ_ERR_ALIGN; a derived scale without scale_out: FGQ_ERR_ARG
+    assert L.fgq_quantize_act_noalloc(x.data_ptr() + 4, n - 1, fgq.U8, 0.0, q.data_ptr(), sc.data_ptr(), s) == \
+        fgq.FGQ_ERR_ALIGN
+    assert L.fgq_quantize_act_noalloc(x.data_ptr(), n, fgq.U8, 0.0, q.data_ptr(), None, s) == fgq.FGQ_ERR_ARG
+    assert L.fgq_quantize_act_noalloc(x.data_ptr(), n, fgq.U8, 0.3, q.data_ptr(), sc.data_ptr(), s) == fgq.FGQ_ERR_ARG
+    assert fgq.fgq_stream_status() == fgq.FGQ_OK
