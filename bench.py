@@ -276,7 +276,7 @@ class Workload:
         self.dev, self.B, self.layers, self.groups, self.act = dev, B, list(layers) + list(fcs), groups, act
         self.first_w8 = first_w8
         self.nconv = len(layers)
-        self.w, self.x, self.q, self.sc, self.ws, self.types = [], [], [], [], [], []
+        self.w, self.x, self.q, self.sc, self.types = [], [], [], [], []
         self.codes = {G: [] for G in groups}
         self.alpha = {G: [] for G in groups}
         self.out = {G: [] for G in groups}
@@ -290,7 +290,6 @@ class Workload:
             n = self.x[-1].numel()
             self.q.append(torch.empty(fgq.act_bytes(n, typ), dtype=torch.uint8, device=dev))
             self.sc.append(torch.empty(1, dtype=torch.float32, device=dev))
-            self.ws.append(torch.empty(max(4, fgq.quantize_act_workspace_bytes(n)), dtype=torch.uint8, device=dev))
             for G in groups:
                 if w8:
                     self.codes[G].append(torch.empty((l.M, l.Kred), dtype=torch.int8, device=dev))
@@ -301,6 +300,16 @@ class Workload:
                     self.alpha[G].append(torch.empty((l.M, fgq.num_groups(l.Kred, G)), dtype=torch.float32,
                                                      device=dev))
                 self.out[G].append(torch.empty((B, l.Ho, l.Wo, l.M), dtype=torch.float32, device=dev))
+        # host tables of every layer's input for fgq_quantize_act_batch
+        nl = len(self.layers)
+        self.qb_n = nl
+        self.qb_x = (ctypes.c_void_p * nl)(*[x.data_ptr() for x in self.x])
+        self.qb_n_elem = (ctypes.c_size_t * nl)(*[x.numel() for x in self.x])
+        self.qb_types = (ctypes.c_int * nl)(*[fgq.ACT_TYPES[t] for t in self.types])
+        self.qb_q = (ctypes.c_void_p * nl)(*[q.data_ptr() for q in self.q])
+        self.qb_sc = (ctypes.c_void_p * nl)(*[s_.data_ptr() for s_ in self.sc])
+        self.qb_ws = torch.empty(max(4, fgq.lib().fgq_quantize_act_batch_workspace_bytes(nl)), dtype=torch.uint8,
+                                 device=dev)
         # host tables of the ternary layers for fgq_ternarize_batch (one launch per G)
         self.tl = [i for i in range(len(self.layers)) if not (first_w8 and i == 0)]
         n = len(self.tl)
@@ -341,10 +350,10 @@ class Workload:
             calls.append((f"ternarize_g{G}", lambda G=G: chk(L.fgq_ternarize_batch(
                 self.tern_n, self.tern_w, self.tern_M, self.tern_K, G, self.tern_codes[G], self.tern_alpha[G], sh),
                 "ternarize_batch")))
-        for i in range(len(self.layers)):
-            calls.append(("quantize_act", lambda i=i: chk(L.fgq_quantize_act(
-                self.x[i].data_ptr(), self.x[i].numel(), fgq.ACT_TYPES[self.types[i]], 0.0, self.q[i].data_ptr(),
-                self.sc[i].data_ptr(), self.ws[i].data_ptr(), self.ws[i].numel(), sh), "quantize")))
+        # every layer's input quantized with its own derived scale, in one batched call
+        calls.append(("quantize_act", lambda: chk(L.fgq_quantize_act_batch(
+            self.qb_n, self.qb_x, self.qb_n_elem, self.qb_types, self.qb_q, self.qb_sc, self.qb_ws.data_ptr(),
+            self.qb_ws.numel(), sh), "quantize_batch")))
         if self.first_w8:
             l = self.layers[0]
             for G in self.groups:

@@ -138,6 +138,31 @@ fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float s
                             float* scale_out, void* workspace, size_t workspace_bytes,
                             cudaStream_t stream);
 
+/* Largest number of tensors one fgq_quantize_act_batch call takes. */
+#define FGQ_QUANTIZE_BATCH_MAX 128
+
+/* Bytes of device workspace fgq_quantize_act_batch needs for n tensors (0 on bad n). */
+size_t fgq_quantize_act_batch_workspace_bytes(int n);
+
+/*
+ * fgq_quantize_act with a derived scale for n tensors (the inputs of a network's layers) in
+ * few launches: tensor i is x[i] fp32 [nelem[i]] -> q[i] (type[i]) and scale_out[i] (device
+ * fp32 [1]), with the results (bit for bit), layouts and non-finite handling of
+ * fgq_quantize_act.  x, nelem, type, q, scale_out are HOST arrays of n entries holding device
+ * pointers, sizes and types (read during the call, not kept); tensors with nelem[i] == 0 are
+ * skipped.  The tensors are processed in order in chunks of up to 64 MB of input (a larger
+ * tensor forms its own chunk), two kernel launches per chunk (the maxima, then the codes),
+ * so the second pass reads what the first left in the L2.  workspace: device scratch of
+ * fgq_quantize_act_batch_workspace_bytes(n) bytes, 4-byte aligned (its contents on entry
+ * do not matter).  The outputs must not overlap the inputs or one another.
+ * Errors: FGQ_ERR_ARG (n < 0 or n > FGQ_QUANTIZE_BATCH_MAX, a null array or pointer, a bad
+ * type, a short workspace), FGQ_ERR_ALIGN (x[i], q[i] not 16-byte aligned; scale_out[i],
+ * workspace not 4-byte aligned), FGQ_ERR_CUDA.
+ */
+fgq_status fgq_quantize_act_batch(int n, const float* const* x, const size_t* nelem, const fgq_act_type* type,
+                                  void* const* q, float* const* scale_out, void* workspace, size_t workspace_bytes,
+                                  cudaStream_t stream);
+
 /*
  * Allocation-free variant of fgq_quantize_act (no counterpart in the paper).  For callers
  * that cannot allocate device memory themselves -- hosts whose device memory is owned by a

@@ -355,6 +355,30 @@ fgq_status fgq_quantize_act(const float* x, size_t n, fgq_act_type type, float s
                          device_error_word(), stream);
 }
 
+size_t fgq_quantize_act_batch_workspace_bytes(int n) {
+  return n < 0 || n > FGQ_QUANTIZE_BATCH_MAX ? 0 : quantize_batch_workspace_bytes(n);
+}
+
+fgq_status fgq_quantize_act_batch(int n, const float* const* x, const size_t* nelem, const fgq_act_type* type,
+                                  void* const* q, float* const* scale_out, void* workspace, size_t workspace_bytes,
+                                  cudaStream_t stream) {
+  if (n < 0 || n > FGQ_QUANTIZE_BATCH_MAX) return FGQ_ERR_ARG;
+  if (n == 0) return FGQ_OK;
+  if (!x || !nelem || !type || !q || !scale_out) return FGQ_ERR_ARG;
+  if (!workspace || workspace_bytes < quantize_batch_workspace_bytes(n)) return FGQ_ERR_ARG;
+  if (!aligned(workspace, 4)) return FGQ_ERR_ALIGN;
+  int types[FGQ_QUANTIZE_BATCH_MAX];
+  for (int i = 0; i < n; ++i) {
+    if (!valid_type(type[i])) return FGQ_ERR_ARG;
+    types[i] = type[i];
+    if (nelem[i] == 0) continue;
+    if (!x[i] || !q[i] || !scale_out[i]) return FGQ_ERR_ARG;
+    if (!aligned(x[i], 16) || !aligned(q[i], 16) || !aligned(scale_out[i], 4)) return FGQ_ERR_ALIGN;
+  }
+  return launch_quantize_batch(n, x, nelem, types, q, scale_out, static_cast<unsigned int*>(workspace),
+                               device_error_word(), stream);
+}
+
 fgq_status fgq_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, float* wscale,
                                    cudaStream_t stream) {
   if (M < 0 || Kred < 0) return FGQ_ERR_ARG;

@@ -53,6 +53,10 @@ fgq_status launch_ternary_error(const float* w, int M, int Kred, int G, const ui
                                 double* errv, cudaStream_t s);
 fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool derive, void* q,
                            float* scale_out, uint32_t* partials, unsigned int* err, cudaStream_t s);
+// Batched derived-scale quantization of n tensors (tmax: n workspace words).
+size_t quantize_batch_workspace_bytes(int n);
+fgq_status launch_quantize_batch(int n, const float* const* x, const size_t* nelem, const int* type, void* const* q,
+                                 float* const* scale_out, unsigned int* tmax, unsigned int* err, cudaStream_t s);
 
 // CUDA-core contraction (dp4a).  codes/alpha for ternary weights, or wq/wscale for dense
 // 8-bit weights (dense != 0).  sums != nullptr writes the int32 group sums [M][ng][P]

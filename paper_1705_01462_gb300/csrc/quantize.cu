@@ -310,6 +310,232 @@ fgq_status launch_quantize(const float* x, size_t n, int type, int E_given, bool
 }  // namespace fgq
 
 // ----------------------------------------------------------------------------------------
+// fgq_quantize_act_batch: the same quantization for many tensors (the inputs of a network's
+// layers), with far fewer launches.  The tensors are taken in order in chunks of at most
+// kBatchChunkBytes of fp32 input (a larger tensor forms a chunk of its own), so that what pass
+// 1 reads is still in the L2 when pass 2 re-reads it.  The passes are pipelined: launch k
+// quantizes chunk k - 1 (pass 2, from the L2) while it reduces chunk k (pass 1, from HBM),
+// so C chunks take C + 1 launches and the two passes overlap.  Every block covers
+// kBatchElems consecutive elements of one tensor.  Pass 1 folds its maximum into the
+// tensor's word with atomicMax (magnitude bit patterns order like the floats); pass 2 takes
+// the tensor's exponent from that word and quantizes its elements, blocks in reverse order
+// (the data pass 1 read last first).
+namespace fgq {
+namespace {
+
+constexpr int kBatchThreads = 256;
+constexpr int64_t kBatchElems = 16384;             // elements per block (64 KB of fp32)
+constexpr int kBatchChunk = 32;                    // tensors per launch
+constexpr size_t kBatchChunkBytes = (size_t)48 << 20;  // two chunks (one per pass) share the L2
+
+struct QTensor {
+  const float* x;
+  uint8_t* q;
+  float* scale;
+  unsigned int* tmax;  // the tensor's maximum word
+  int64_t n;
+  int type;
+  int block0;   // first block of this tensor in the launch
+};
+
+struct QBatch {
+  QTensor t[kBatchChunk];
+  int n;
+  int nblocks;
+};
+
+__device__ __forceinline__ int qbatch_tensor(const QBatch& b, int blk) {
+  int lo = 0, hi = b.n - 1;
+  while (lo < hi) {  // largest tensor whose first block is <= blk
+    const int mid = (lo + hi + 1) >> 1;
+    if (b.t[mid].block0 <= blk) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ void qab_max_block(const QBatch& b, int blk, unsigned int* err) {
+  const QTensor& T = b.t[qbatch_tensor(b, blk)];
+  const int64_t e0 = (int64_t)(blk - T.block0) * kBatchElems;
+  const int64_t e1 = e0 + kBatchElems < T.n ? e0 + kBatchElems : T.n;
+  const bool is_unsigned = T.type == FGQ_U8 || T.type == FGQ_U4;
+  uint32_t mx = 0;
+  bool bad = false;
+  const float4* x4 = reinterpret_cast<const float4*>(T.x + e0);  // e0 is a multiple of 4: aligned
+  const int64_t n4 = (e1 - e0) / 4;
+  const uint64_t keep = policy_evict_last();
+  constexpr int U = 4;  // independent 16-byte loads in flight per thread
+  int64_t i = threadIdx.x;
+  for (; i + (U - 1) * kBatchThreads < n4; i += U * kBatchThreads) {
+    float4 f[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) f[u] = ld_f4_policy(x4 + i + u * kBatchThreads, keep);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const float e[4] = {f[u].x, f[u].y, f[u].z, f[u].w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        bad |= (__float_as_uint(e[j]) & 0x7fffffffu) >= 0x7f800000u;
+        mx = max(mx, mag_bits(e[j], is_unsigned));
+      }
+    }
+  }
+  for (; i < n4; i += kBatchThreads) {
+    const float4 f = ld_f4_policy(x4 + i, keep);
+    const float e[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      bad |= (__float_as_uint(e[j]) & 0x7fffffffu) >= 0x7f800000u;
+      mx = max(mx, mag_bits(e[j], is_unsigned));
+    }
+  }
+  for (int64_t i = e0 + n4 * 4 + threadIdx.x; i < e1; i += kBatchThreads) {
+    const float e = __ldg(T.x + i);
+    bad |= (__float_as_uint(e) & 0x7fffffffu) >= 0x7f800000u;
+    mx = max(mx, mag_bits(e, is_unsigned));
+  }
+  __shared__ uint32_t red[kBatchThreads / 32];
+  mx = __reduce_max_sync(FULL_MASK, mx);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+  if (__syncthreads_or(bad) && threadIdx.x == 0) record_error(err, FGQ_ERR_NONFINITE);
+  if (threadIdx.x == 0) {
+    uint32_t m = 0;
+    for (int i = 0; i < kBatchThreads / 32; ++i) m = max(m, red[i]);
+    atomicMax(T.tmax, m);
+  }
+}
+
+template <int TYPE>
+__device__ __forceinline__ void qab_quant_range(const QTensor& T, int64_t e0, int64_t e1, bool write_scale) {
+  using Tr = QTraits<TYPE>;
+  const int E = dfp_exponent(*reinterpret_cast<const volatile unsigned int*>(T.tmax), Tr::qmax);
+  if (write_scale && threadIdx.x == 0) *T.scale = pow2f(E);
+  const float mul1 = (-E <= 127) ? pow2f(-E) : pow2f(64);
+  const float mul2 = (-E <= 127) ? 1.0f : pow2f(-E - 64);
+  const int64_t n16 = (e1 - e0) / 16;
+  const float4* x4 = reinterpret_cast<const float4*>(T.x + e0);
+  const uint64_t drop = policy_evict_first();
+  for (int64_t c = threadIdx.x; c < n16; c += kBatchThreads) {
+    float e[16];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 f = ld_f4_policy(x4 + 4 * c + j, drop);
+      e[4 * j] = f.x; e[4 * j + 1] = f.y; e[4 * j + 2] = f.z; e[4 * j + 3] = f.w;
+    }
+    if (Tr::bits == 8) {
+      uint32_t wv[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        wv[j] = qcode<TYPE>(e[4 * j], mul1, mul2) | (qcode<TYPE>(e[4 * j + 1], mul1, mul2) << 8) |
+                (qcode<TYPE>(e[4 * j + 2], mul1, mul2) << 16) | (qcode<TYPE>(e[4 * j + 3], mul1, mul2) << 24);
+      reinterpret_cast<uint4*>(T.q + e0)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+    } else {
+      uint32_t wv[2] = {0u, 0u};
+#pragma unroll
+      for (int j = 0; j < 16; ++j) wv[j / 8] |= qcode<TYPE>(e[j], mul1, mul2) << (4 * (j % 8));
+      reinterpret_cast<uint2*>(T.q + e0 / 2)[c] = make_uint2(wv[0], wv[1]);
+    }
+  }
+  if (threadIdx.x == 0) {  // the tensor's ragged tail (last block only): fewer than 16 elements
+    for (int64_t i = e0 + n16 * 16; i < e1; ++i) {
+      const uint32_t code = qcode<TYPE>(T.x[i], mul1, mul2);
+      if (Tr::bits == 8) {
+        T.q[i] = (uint8_t)code;
+      } else if ((i & 1) == 0) {
+        T.q[i / 2] = (uint8_t)code;  // the high nibble of an odd tail stays 0
+      } else {
+        T.q[i / 2] = (uint8_t)(T.q[i / 2] | (code << 4));
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void qab_quant_block(const QBatch& b, int blk) {
+  const QTensor& T = b.t[qbatch_tensor(b, blk)];
+  const int64_t e0 = (int64_t)(blk - T.block0) * kBatchElems;
+  const int64_t e1 = e0 + kBatchElems < T.n ? e0 + kBatchElems : T.n;
+  const bool first = blk == T.block0;
+  switch (T.type) {
+    case FGQ_U8: qab_quant_range<FGQ_U8>(T, e0, e1, first); break;
+    case FGQ_S8: qab_quant_range<FGQ_S8>(T, e0, e1, first); break;
+    case FGQ_U4: qab_quant_range<FGQ_U4>(T, e0, e1, first); break;
+    default: qab_quant_range<FGQ_S4>(T, e0, e1, first); break;
+  }
+}
+
+// One pipelined launch: blocks [0, q.nblocks) quantize chunk q (reverse block order), the
+// rest reduce chunk m.
+struct QPair {
+  QBatch q, m;
+};
+
+__global__ void __launch_bounds__(kBatchThreads) qab_kernel(const __grid_constant__ QPair p, unsigned int* err) {
+  const int bx = (int)blockIdx.x;
+  if (bx < p.q.nblocks) qab_quant_block(p.q, p.q.nblocks - 1 - bx);
+  else qab_max_block(p.m, bx - p.q.nblocks, err);
+}
+
+}  // namespace
+
+size_t quantize_batch_workspace_bytes(int n) { return n > 0 ? sizeof(unsigned int) * (size_t)n : 0; }
+
+fgq_status launch_quantize_batch(int n, const float* const* x, const size_t* nelem, const int* type, void* const* q,
+                                 float* const* scale_out, unsigned int* tmax, unsigned int* err, cudaStream_t s) {
+  if (cudaMemsetAsync(tmax, 0, sizeof(unsigned int) * (size_t)n, s) != cudaSuccess) return FGQ_ERR_CUDA;
+  QPair p;
+  memset(&p, 0, sizeof p);  // p.q: the chunk waiting for pass 2 (none yet)
+  int i = 0;
+  auto launch = [&]() -> fgq_status {
+    const int64_t blocks = (int64_t)p.q.nblocks + p.m.nblocks;
+    if (blocks == 0) return FGQ_OK;
+    if (blocks > INT32_MAX) return FGQ_ERR_UNSUPPORTED;
+    qab_kernel<<<(unsigned)blocks, kBatchThreads, 0, s>>>(p, err);
+    return after_launch();
+  };
+  while (i < n) {
+    QBatch& b = p.m;
+    memset(&b, 0, sizeof b);
+    size_t bytes = 0;
+    int blocks = 0;
+    // a chunk: consecutive tensors up to kBatchChunkBytes of input (at least one tensor)
+    while (i < n && b.n < kBatchChunk) {
+      if (nelem[i] == 0) {
+        ++i;
+        continue;
+      }
+      const size_t tb = nelem[i] * sizeof(float);
+      if (b.n > 0 && bytes + tb > kBatchChunkBytes) break;
+      const int64_t nb = ((int64_t)nelem[i] + kBatchElems - 1) / kBatchElems;
+      if ((int64_t)blocks + nb > INT32_MAX) {
+        if (b.n == 0) return FGQ_ERR_UNSUPPORTED;  // one tensor beyond the grid's reach
+        break;
+      }
+      QTensor& T = b.t[b.n++];
+      T.x = x[i];
+      T.q = static_cast<uint8_t*>(q[i]);
+      T.scale = scale_out[i];
+      T.tmax = tmax + i;
+      T.n = (int64_t)nelem[i];
+      T.type = type[i];
+      T.block0 = blocks;
+      blocks += (int)nb;
+      bytes += tb;
+      ++i;
+    }
+    if (b.n == 0) continue;
+    b.nblocks = blocks;
+    // pass 2 of the previous chunk and pass 1 of this one
+    const fgq_status st = launch();
+    if (st != FGQ_OK) return st;
+    p.q = p.m;
+  }
+  memset(&p.m, 0, sizeof p.m);
+  return launch();  // pass 2 of the last chunk
+}
+
+}  // namespace fgq
+
+// ----------------------------------------------------------------------------------------
 // fgq_quantize_act_noalloc: the derived-scale quantizer for callers that cannot allocate
 // device memory.  Some hosts own every device allocation themselves (a framework's memory
 // pool with a fixed budget, a plugin that only receives pre-allocated tensors) or cannot

@@ -39,6 +39,8 @@ SIGNATURES = [
     ("fgq_quantize_act_workspace_bytes", _sz, [_sz]),
     ("fgq_quantize_act", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp, _sz, _vp]),
     ("fgq_quantize_act_noalloc", _i, [_vp, _sz, _i, _f, _vp, _vp, _vp]),
+    ("fgq_quantize_act_batch_workspace_bytes", _sz, [_i]),
+    ("fgq_quantize_act_batch", _i, [_i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     ("fgq_quantize_weights_w8", _i, [_vp, _i, _i, _vp, _vp, _vp]),
     ("fgq_gemm", _i, [_vp, _i, _vp, _i, _i, _vp, _vp, _i, _i, _vp, _vp]),
     ("fgq_conv2d", _i, [_vp, _i, _vp] + [_i] * 9 + [_vp, _vp, _i, _i, _vp, _vp]),
@@ -232,6 +234,23 @@ def fgq_quantize_act(x: torch.Tensor, act_type="u8", scale_in: float = 0.0, q: O
                                   _dev(scale_out, torch.float32, "scale_out") if scale_in <= 0 else None,
                                   ws_ptr, ws_len, _stream(stream)), "fgq_quantize_act")
     return q, scale_out
+
+
+def fgq_quantize_act_batch(xs, act_types, stream=None):
+    """fgq_quantize_act_batch over a list of fp32 device tensors with derived scales: returns
+    [(q, scale)] in the same order (q packed as fgq_quantize_act's)."""
+    _require_cuda()
+    n = len(xs)
+    types = [_act_type(t) for t in act_types]
+    qs = [torch.empty(act_bytes(x.numel(), t), dtype=torch.uint8, device=x.device) for x, t in zip(xs, types)]
+    scs = [torch.empty(1, dtype=torch.float32, device=x.device) for x in xs]
+    ws = torch.empty(max(4, int(lib().fgq_quantize_act_batch_workspace_bytes(n))), dtype=torch.uint8,
+                     device=xs[0].device if n else "cuda")
+    arr = lambda ts: (ctypes.c_void_p * n)(*[_dev(t, t.dtype, "tensor") for t in ts])
+    _check(lib().fgq_quantize_act_batch(n, arr(xs), (ctypes.c_size_t * n)(*[x.numel() for x in xs]),
+                                        (ctypes.c_int * n)(*types), arr(qs), arr(scs), ws.data_ptr(), ws.numel(),
+                                        _stream(stream)), "fgq_quantize_act_batch")
+    return list(zip(qs, scs))
 
 
 def fgq_quantize_weights_w8(w: torch.Tensor, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
