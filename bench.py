@@ -807,7 +807,8 @@ def run_layers(args):
             call()
         per = []
         for _ in range(args.iters):
-            flush.zero_()
+            with torch.cuda.stream(stream):
+                flush.zero_()  # on the timed stream, ahead of the event
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             call()

@@ -364,7 +364,7 @@ __device__ __forceinline__ void qab_max_block(const QBatch& b, int blk, unsigned
   const float4* x4 = reinterpret_cast<const float4*>(T.x + e0);  // e0 is a multiple of 4: aligned
   const int64_t n4 = (e1 - e0) / 4;
   const uint64_t keep = policy_evict_last();
-  constexpr int U = 4;  // independent 16-byte loads in flight per thread
+  constexpr int U = 8;  // independent 16-byte loads in flight per thread
   int64_t i = threadIdx.x;
   for (; i + (U - 1) * kBatchThreads < n4; i += U * kBatchThreads) {
     float4 f[U];
@@ -415,25 +415,35 @@ __device__ __forceinline__ void qab_quant_range(const QTensor& T, int64_t e0, in
   const int64_t n16 = (e1 - e0) / 16;
   const float4* x4 = reinterpret_cast<const float4*>(T.x + e0);
   const uint64_t drop = policy_evict_first();
-  for (int64_t c = threadIdx.x; c < n16; c += kBatchThreads) {
-    float e[16];
+  constexpr int CU = 2;  // 16-element chunks in flight per thread (8 independent 16-byte loads)
+  for (int64_t c0 = threadIdx.x; c0 < n16; c0 += CU * kBatchThreads) {
+    float e[CU][16];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float4 f = ld_f4_policy(x4 + 4 * c + j, drop);
-      e[4 * j] = f.x; e[4 * j + 1] = f.y; e[4 * j + 2] = f.z; e[4 * j + 3] = f.w;
+    for (int u = 0; u < CU; ++u) {
+      const int64_t c = c0 + u * kBatchThreads;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 f = c < n16 ? ld_f4_policy(x4 + 4 * c + j, drop) : make_float4(0.f, 0.f, 0.f, 0.f);
+        e[u][4 * j] = f.x; e[u][4 * j + 1] = f.y; e[u][4 * j + 2] = f.z; e[u][4 * j + 3] = f.w;
+      }
     }
-    if (Tr::bits == 8) {
-      uint32_t wv[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        wv[j] = qcode<TYPE>(e[4 * j], mul1, mul2) | (qcode<TYPE>(e[4 * j + 1], mul1, mul2) << 8) |
-                (qcode<TYPE>(e[4 * j + 2], mul1, mul2) << 16) | (qcode<TYPE>(e[4 * j + 3], mul1, mul2) << 24);
-      reinterpret_cast<uint4*>(T.q + e0)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
-    } else {
-      uint32_t wv[2] = {0u, 0u};
+    for (int u = 0; u < CU; ++u) {
+      const int64_t c = c0 + u * kBatchThreads;
+      if (c >= n16) break;
+      if (Tr::bits == 8) {
+        uint32_t wv[4];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) wv[j / 8] |= qcode<TYPE>(e[j], mul1, mul2) << (4 * (j % 8));
-      reinterpret_cast<uint2*>(T.q + e0 / 2)[c] = make_uint2(wv[0], wv[1]);
+        for (int j = 0; j < 4; ++j)
+          wv[j] = qcode<TYPE>(e[u][4 * j], mul1, mul2) | (qcode<TYPE>(e[u][4 * j + 1], mul1, mul2) << 8) |
+                  (qcode<TYPE>(e[u][4 * j + 2], mul1, mul2) << 16) | (qcode<TYPE>(e[u][4 * j + 3], mul1, mul2) << 24);
+        reinterpret_cast<uint4*>(T.q + e0)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+      } else {
+        uint32_t wv[2] = {0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 16; ++j) wv[j / 8] |= qcode<TYPE>(e[u][j], mul1, mul2) << (4 * (j % 8));
+        reinterpret_cast<uint2*>(T.q + e0 / 2)[c] = make_uint2(wv[0], wv[1]);
+      }
     }
   }
   if (threadIdx.x == 0) {  // the tensor's ragged tail (last block only): fewer than 16 elements

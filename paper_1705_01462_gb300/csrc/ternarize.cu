@@ -213,6 +213,129 @@ __global__ void __launch_bounds__(256) ternarize_small_kernel(const float* __res
     small_unit<G>(w, Kred, ng, wrow, codes, alpha, err, vec4, units_per_row, u);
 }
 
+// One group of G in {32, 64} weights (group grp = m ng + g of the layer) solved by one
+// thread: the G magnitudes sorted in registers (bitonic network, descending), then the exact
+// scan of solve_group_regs; the signs for the codes are read again (the group's bytes are
+// still in L1), so only the sorted magnitudes occupy registers.
+template <int G>
+__device__ __forceinline__ void thread_group(const float* __restrict__ w, int Kred, int ng, int wrow,
+                                             uint32_t* __restrict__ codes, float* __restrict__ alpha,
+                                             unsigned int* err, int vec4, int64_t grp) {
+  const int m = (int)(grp / ng);
+  const int g = (int)(grp - (int64_t)m * ng);
+  const float* src = w + (int64_t)m * Kred + (int64_t)g * G;
+  const int nvalid = Kred - g * G < G ? Kred - g * G : G;
+  uint32_t s[G];
+  bool bad = false;
+  if (vec4 && nvalid == G) {
+#pragma unroll
+    for (int i = 0; i < G; i += 4) {
+      const float4 f = __ldg(reinterpret_cast<const float4*>(src + i));
+      s[i] = __float_as_uint(f.x) & 0x7fffffffu;
+      s[i + 1] = __float_as_uint(f.y) & 0x7fffffffu;
+      s[i + 2] = __float_as_uint(f.z) & 0x7fffffffu;
+      s[i + 3] = __float_as_uint(f.w) & 0x7fffffffu;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < G; ++i) s[i] = i < nvalid ? __float_as_uint(__ldg(src + i)) & 0x7fffffffu : 0u;
+  }
+#pragma unroll
+  for (int i = 0; i < G; ++i) bad |= s[i] >= 0x7f800000u;
+  uint32_t* crow = codes + (int64_t)m * wrow + g * (G / 16);
+  if (bad) {
+    record_error(err, FGQ_ERR_NONFINITE);
+    alpha[grp] = 0.0f;
+#pragma unroll
+    for (int wd = 0; wd < G / 16; ++wd) crow[wd] = 0u;
+    return;
+  }
+  // bitonic sort, descending
+#pragma unroll
+  for (int size = 2; size <= G; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+#pragma unroll
+      for (int i = 0; i < G; ++i) {
+        if ((i & stride) == 0) {
+          const bool desc = (i & size) == 0;
+          const uint32_t a = s[i], b = s[i + stride];
+          const uint32_t mx = a > b ? a : b, mn = a > b ? b : a;
+          s[i] = desc ? mx : mn;
+          s[i + stride] = desc ? mn : mx;
+        }
+      }
+    }
+  }
+  uint32_t bk = 0, tau = 0;
+  uint64_t bS = 0;
+  float bJ = 0.0f;  // fp32 estimate of the best objective, within 2^-21 of bS^2 / bk
+  int F = 1;
+  if (s[0] != 0) {
+    F = max((int)(s[0] >> 23), 1);
+    uint64_t S = 0;
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      S += fixed_of(s[i], F);
+      const bool run_end = (i == G - 1) || (s[(i + 1) < G ? i + 1 : i] < s[i]);
+      if (run_end && in_window(s[i], F)) {
+        // candidates come in increasing k, so a strict comparison keeps the smaller k on ties.
+        // An fp32 estimate (relative error below 2^-21) decides every comparison whose two
+        // objectives differ by more than 2^-14; the rest are decided exactly in 128 bits.
+        const float fS = (float)S;
+        const float J = fS * fS * (1.0f / (float)(i + 1));
+        bool take;
+        if (bk == 0 || J > bJ * (1.0f + 0x1p-14f)) take = true;
+        else if (J < bJ * (1.0f - 0x1p-14f)) take = false;
+        else take = j_greater(S, (uint32_t)(i + 1), bS, bk);
+        if (take) {
+          bS = S;
+          bk = (uint32_t)(i + 1);
+          tau = s[i];
+          bJ = J;
+        }
+      }
+    }
+  }
+  alpha[grp] = bk ? round_ratio_f32(bS, bk, F - 158) : 0.0f;
+  // codes: t = sign(w) where |w| >= tau (tau > 0 whenever anything is kept)
+  const uint32_t thr = bk ? tau : 0xffffffffu;
+#pragma unroll
+  for (int wd = 0; wd < G / 16; ++wd) {
+    uint32_t b[16];
+    if (vec4 && nvalid == G) {
+#pragma unroll
+      for (int e = 0; e < 16; e += 4) {
+        const float4 f = __ldg(reinterpret_cast<const float4*>(src + 16 * wd + e));
+        b[e] = __float_as_uint(f.x);
+        b[e + 1] = __float_as_uint(f.y);
+        b[e + 2] = __float_as_uint(f.z);
+        b[e + 3] = __float_as_uint(f.w);
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) b[e] = 16 * wd + e < nvalid ? __float_as_uint(__ldg(src + 16 * wd + e)) : 0u;
+    }
+    uint32_t bits = 0;
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+      if ((b[e] & 0x7fffffffu) >= thr) bits |= ((b[e] >> 31) ? 3u : 1u) << (2 * e);
+    crow[wd] = bits;
+  }
+}
+
+// One thread per group for G in {32, 64}.
+template <int G>
+__global__ void __launch_bounds__(128) ternarize_thread_kernel(const float* __restrict__ w, int M, int Kred,
+                                                               int ng, int wrow, uint32_t* __restrict__ codes,
+                                                               float* __restrict__ alpha, unsigned int* err,
+                                                               int vec4) {
+  const int64_t total = (int64_t)M * ng;
+  for (int64_t grp = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; grp < total;
+       grp += (int64_t)gridDim.x * blockDim.x)
+    thread_group<G>(w, Kred, ng, wrow, codes, alpha, err, vec4, grp);
+}
+
 // One group of G in {32, 64, 128} weights (group grp = m ng + g of the layer) solved by one
 // warp: lane l holds elements l*E .. l*E+E-1.
 template <int G>
@@ -396,6 +519,16 @@ __global__ void __launch_bounds__(256) ternarize_small_batch_kernel(const __grid
 }
 
 template <int G>
+__global__ void __launch_bounds__(128) ternarize_thread_batch_kernel(const __grid_constant__ TernBatch b,
+                                                                     unsigned int* err) {
+  for (int64_t grp = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; grp < b.total;
+       grp += (int64_t)gridDim.x * blockDim.x) {
+    const TernLayer& L = b.l[batch_layer(b, grp)];
+    thread_group<G>(L.w, L.Kred, L.ng, L.wrow, L.codes, L.alpha, err, L.vec4, grp - L.first);
+  }
+}
+
+template <int G>
 __global__ void __launch_bounds__(256) ternarize_warp_batch_kernel(const __grid_constant__ TernBatch b,
                                                                    unsigned int* err) {
   const int lane = threadIdx.x & 31;
@@ -477,8 +610,8 @@ fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* co
     case 4: ternarize_small_kernel<4><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
     case 8: ternarize_small_kernel<8><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
     case 16: ternarize_small_kernel<16><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
-    case 32: ternarize_warp_kernel<32><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
-    case 64: ternarize_warp_kernel<64><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
+    case 32: ternarize_thread_kernel<32><<<grid_for((int64_t)M * ng, 128), 128, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
+    case 64: ternarize_thread_kernel<64><<<grid_for((int64_t)M * ng, 128), 128, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
     case 128: ternarize_warp_kernel<128><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
     default: return FGQ_ERR_ARG;
   }
@@ -515,8 +648,8 @@ fgq_status launch_ternarize_batch(int n, const float* const* w, const int* M, co
     case 4: ternarize_small_batch_kernel<4><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
     case 8: ternarize_small_batch_kernel<8><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
     case 16: ternarize_small_batch_kernel<16><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
-    case 32: ternarize_warp_batch_kernel<32><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
-    case 64: ternarize_warp_batch_kernel<64><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
+    case 32: ternarize_thread_batch_kernel<32><<<grid_for(total, 128), 128, 0, s>>>(b, err); break;
+    case 64: ternarize_thread_batch_kernel<64><<<grid_for(total, 128), 128, 0, s>>>(b, err); break;
     case 128: ternarize_warp_batch_kernel<128><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
     default: return FGQ_ERR_ARG;
   }
