@@ -113,30 +113,37 @@ __device__ __forceinline__ void tile_coords_d(const TDArgs& a, int tile, int& gi
 // 4-bit packed two per byte, element 2i in the low nibble) times t, and rs = ascale; MODE 0:
 // fp32 alphas split into hi + lo after scaling the row by 2^e, rs = 2^-e.  Row m of part i
 // is fp16 [Kp] at a_i + m Kp; codes 00 and padding give 0.
+constexpr int FOLD_THREADS = 128;  // one block per filter row
 template <int MODE>
-__global__ void __launch_bounds__(256) fold_weights_kernel(const uint32_t* __restrict__ codes, int M, int wrow, int G,
-                                                           int ng, const float* __restrict__ alpha,
-                                                           const uint8_t* __restrict__ aq,
-                                                           const float* __restrict__ ascale, __half* __restrict__ a0,
-                                                           __half* __restrict__ a1, float* __restrict__ row_scale) {
-  const int m = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (m >= M) return;
+__global__ void __launch_bounds__(FOLD_THREADS) fold_weights_kernel(const uint32_t* __restrict__ codes, int M,
+                                                                    int wrow, int G, int ng,
+                                                                    const float* __restrict__ alpha,
+                                                                    const uint8_t* __restrict__ aq,
+                                                                    const float* __restrict__ ascale,
+                                                                    __half* __restrict__ a0, __half* __restrict__ a1,
+                                                                    float* __restrict__ row_scale) {
+  const int m = blockIdx.x;
+  const int tid = threadIdx.x;
   float mul = 1.0f;
   if (MODE == 0) {
     float mx = 0.0f;
-    for (int g = lane; g < ng; g += 32) mx = fmaxf(mx, __ldg(alpha + (int64_t)m * ng + g));
+    for (int g = tid; g < ng; g += FOLD_THREADS) mx = fmaxf(mx, __ldg(alpha + (int64_t)m * ng + g));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    __shared__ float red[FOLD_THREADS / 32];
+    if ((tid & 31) == 0) red[tid >> 5] = mx;
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < FOLD_THREADS / 32; ++i) mx = fmaxf(mx, red[i]);
     int e = mx > 0.0f ? 14 - ilogbf(mx) : 0;  // mx 2^e in [2^14, 2^15)
     e = e < -100 ? -100 : (e > 100 ? 100 : e);
     mul = ldexpf(1.0f, e);
-    if (lane == 0) row_scale[m] = ldexpf(1.0f, -e);
-  } else if (lane == 0) {
+    if (tid == 0) row_scale[m] = ldexpf(1.0f, -e);
+  } else if (tid == 0) {
     row_scale[m] = __ldg(ascale + m);
   }
   const int64_t arow = MODE == 4 ? (ng + 1) / 2 : ng;
-  for (int w = lane; w < wrow; w += 32) {
+  for (int w = tid; w < wrow; w += FOLD_THREADS) {
     const uint32_t cw = __ldg(codes + (int64_t)m * wrow + w);
     uint32_t h0[8], h1[8];
 #pragma unroll
@@ -591,6 +598,71 @@ __global__ void __launch_bounds__(128) im2col_u8_kernel(const uint8_t* __restric
   }
 }
 
+// The same im2col rows, one block per output row (b, ho): the R input rows that output
+// row reads (zeros outside the image) are staged in shared memory with coalesced loads, and
+// the Wo consecutive col rows -- one contiguous range of Wo * Kc bytes -- are written in
+// 16-byte pieces by consecutive threads (coalesced stores), each piece gathered from the
+// staged rows through a per-element table (row offset r * W * C + c, tap column s).
+constexpr int IM2COL_ROWS_SMEM = 40 * 1024;
+__global__ void __launch_bounds__(256) im2col_rows_kernel(const uint8_t* __restrict__ act, int H, int W, int C,
+                                                         int R, int S, int stride, int pad, int Ho, int Wo, int Kred,
+                                                         int Kc, uint8_t* __restrict__ col) {
+  extern __shared__ uint8_t sm_i2c[];
+  const int rowb = W * C;
+  uint8_t* buf = sm_i2c;                                                       // [R][W * C]
+  uint16_t* tab_off = reinterpret_cast<uint16_t*>(sm_i2c + ((R * rowb + 15) & ~15));  // [Kc]
+  uint8_t* tab_s = reinterpret_cast<uint8_t*>(tab_off + Kc);                        // [Kc]
+  const int ho = blockIdx.x % Ho;
+  const int b = blockIdx.x / Ho;
+  const int h0 = ho * stride - pad;
+  for (int i = threadIdx.x; i < R * rowb; i += blockDim.x) {
+    const int r = i / rowb, e = i - r * rowb;
+    const int h = h0 + r;
+    buf[i] = (h >= 0 && h < H) ? __ldg(act + ((int64_t)b * H + h) * rowb + e) : (uint8_t)0;
+  }
+  for (int j = threadIdx.x; j < Kc; j += blockDim.x) {
+    if (j < Kred) {
+      const int r = j / (S * C), rem = j - r * S * C;
+      const int sx = rem / C, c = rem - sx * C;
+      tab_off[j] = (uint16_t)(r * rowb + c);
+      tab_s[j] = (uint8_t)sx;
+    } else {
+      tab_s[j] = 0xff;  // padding: zero
+    }
+  }
+  __syncthreads();
+  // thread t always writes piece jp = t % cpr of a row (its 16 table entries in registers),
+  // for rows wo = t / cpr, t / cpr + rows_per_pass, ...; consecutive threads write
+  // consecutive pieces
+  const int cpr = Kc / 16;  // 16-byte pieces per col row (<= 256)
+  const int rows_per_pass = blockDim.x / cpr;
+  const int jp = threadIdx.x % cpr;
+  const int wo0 = threadIdx.x / cpr;
+  if (wo0 >= rows_per_pass) return;
+  int off[16], sxs[16];
+#pragma unroll
+  for (int e = 0; e < 16; ++e) {
+    const int j = jp * 16 + e;
+    sxs[e] = tab_s[j];
+    off[e] = sxs[e] != 0xff ? tab_off[j] : 0;
+  }
+  uint4* dst = reinterpret_cast<uint4*>(col + ((int64_t)b * Ho + ho) * Wo * Kc);
+  for (int wo = wo0; wo < Wo; wo += rows_per_pass) {
+    const int wbase = wo * stride - pad;
+    uint32_t wv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      uint32_t byte = 0u;
+      const int w = wbase + sxs[e];
+      if (sxs[e] != 0xff && w >= 0 && w < W) byte = buf[off[e] + w * C];
+      wv[e >> 2] |= byte << (8 * (e & 3));
+    }
+    dst[wo * cpr + jp] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  }
+}
+
+size_t im2col_rows_smem(const Geom& g, int Kc) { return (size_t)((g.R * g.W * g.C + 15) & ~15) + 3 * (size_t)Kc; }
+
 // 8-bit weights wq [M][Kred] as fp16 [M][Kc] (zero-padded), rs = wscale: exact.
 __global__ void __launch_bounds__(256) fold_w8_kernel(const int8_t* __restrict__ wq, const float* __restrict__ wscale,
                                                       int M, int Kred, int Kc, __half* __restrict__ a0,
@@ -660,13 +732,16 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
   __half* a0 = static_cast<__half*>(tmp);
   __half* a1 = NA == 2 ? a0 + (size_t)g.M * g.Kp : nullptr;
   float* rs = reinterpret_cast<float*>(static_cast<uint8_t*>(tmp) + NA * part_bytes);
-  const unsigned fblocks = (unsigned)((g.M + 7) / 8);
+  const unsigned fblocks = (unsigned)g.M;
   if (!aq)
-    fold_weights_kernel<0><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, alpha, nullptr, nullptr, a0, a1, rs);
+    fold_weights_kernel<0><<<fblocks, FOLD_THREADS, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, alpha, nullptr, nullptr, a0,
+                                                            a1, rs);
   else if (abits == 8)
-    fold_weights_kernel<8><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1, rs);
+    fold_weights_kernel<8><<<fblocks, FOLD_THREADS, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1,
+                                                            rs);
   else
-    fold_weights_kernel<4><<<fblocks, 256, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1, rs);
+    fold_weights_kernel<4><<<fblocks, FOLD_THREADS, 0, s>>>(codes, g.M, g.wrow, g.G, g.ng, nullptr, aq, ascale, a0, a1,
+                                                            rs);
   fgq_status st = after_launch();
   if (st == FGQ_OK) st = run_dense(act, g, NA, a0, a1, rs, act_scale, out, err, s);
   // the temporary returns to the pool once the work queued on s before this point is done
@@ -676,7 +751,7 @@ fgq_status launch_dense_contract(const void* act, const Geom& g, const uint32_t*
 
 fgq_status launch_fold_alpha_split(const uint32_t* codes, int M, int wrow, int G, int ng, const float* alpha,
                                    void* a0, void* a1, float* rs, cudaStream_t s) {
-  fold_weights_kernel<0><<<(unsigned)((M + 7) / 8), 256, 0, s>>>(codes, M, wrow, G, ng, alpha, nullptr, nullptr,
+  fold_weights_kernel<0><<<(unsigned)M, FOLD_THREADS, 0, s>>>(codes, M, wrow, G, ng, alpha, nullptr, nullptr,
                                                                 static_cast<__half*>(a0), static_cast<__half*>(a1), rs);
   return after_launch();
 }
@@ -702,8 +777,14 @@ fgq_status launch_dense_w8(const void* act, const Geom& g, const int8_t* wq, con
   uint8_t* col = static_cast<uint8_t*>(tmp);
   __half* a0 = reinterpret_cast<__half*>(col + col_bytes);
   float* rs = reinterpret_cast<float*>(col + col_bytes + a_bytes);
-  im2col_u8_kernel<<<(unsigned)((g.P + 127) / 128), 128, 0, s>>>(
-      static_cast<const uint8_t*>(act), g.B, g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
+  const size_t rows_smem = im2col_rows_smem(g, Kc);
+  if (rows_smem <= (size_t)IM2COL_ROWS_SMEM && g.S <= 254 && g.R * g.W * g.C < 65536 &&
+      (int64_t)g.B * g.Ho < INT32_MAX)
+    im2col_rows_kernel<<<(unsigned)((int64_t)g.B * g.Ho), 256, rows_smem, s>>>(
+        static_cast<const uint8_t*>(act), g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
+  else
+    im2col_u8_kernel<<<(unsigned)((g.P + 127) / 128), 128, 0, s>>>(
+        static_cast<const uint8_t*>(act), g.B, g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
   fgq_status st = after_launch();
   if (st == FGQ_OK) {
     fold_w8_kernel<<<(unsigned)(((int64_t)g.M * Kc + 255) / 256), 256, 0, s>>>(wq, wscale, g.M, g.Kred, Kc, a0, rs);
