@@ -14,25 +14,25 @@
 // The group-sums variant (SUMS) stores each drained accumulator as the int32 s[m][g][p]
 // instead (the exact integers themselves, for verification).
 //
-// Warp roles (416 threads, one CTA per SM, persistent over tiles):
+// Warp roles (480 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
-//              64*(w/4).. (positions) of the drained buffer: one 64-column tcgen05.ld and
-//              two 32-column tcgen05.ld per group, release of the buffer, FMAs with alpha into
-//              fp32 registers.  At tile end the fp32 tile goes to shared memory and one
-//              thread writes it to HBM with a TMA box store (direct stores when the
-//              output has several conv groups or M % 4 != 0).
-//   warps 8-11 loaders/converters: for layers whose im2col rows are contiguous input rows
-//              (1x1 stride-1 convolutions, GEMMs) one thread issues a TMA box load of the
-//              K-tile's 128 activation rows; for other layers each thread copies its own
-//              row with 16-byte cp.async.  Thread t converts row t to fp16 in the
-//              128-byte-swizzled K-major layout the MMA reads; a staging slot is refilled
-//              by TMA only after every loader has released it (st_empty), so the loader
-//              warps never wait for each other otherwise.
+//              64*(w/4).. (positions) of the drained buffer: two 32-column tcgen05.ld per
+//              group, release of the buffer, FMAs with alpha into fp32 registers.  At tile end
+//              the fp32 tile goes to shared memory and one thread writes it to HBM with a TMA
+//              box store (direct stores when the output has several conv groups, M % 4 != 0,
+//              or the output is requantized).
+//   warps 8-11 converters: thread t converts tile row t (one output position, 64 reduction
+//              elements) of a staged K-tile to fp16 in the 128-byte-swizzled K-major layout
+//              the MMA reads.
 //   warp 12    TMEM allocation and the MMA issuer (one thread): 4 tcgen05.mma (K = 16)
 //              per K-tile into one of four 128-column TMEM accumulators.
 //   warp 13    streams the ternary operand: the codes are expanded to fp16 {0, +1, -1} once
 //              per call (a stream-ordered temporary) and reach a four-stage ring of their own
 //              by TMA in the MMA's swizzled layout, ahead of the K-tiles that use them.
+//   warp 14    streams the activations: one TMA load per K-tile into a six-slot staging ring,
+//              a 2D box of 128 consecutive input rows when the im2col rows are input rows
+//              (1x1 stride-1 convolutions, GEMMs), otherwise an im2col box (the 128 output
+//              positions' pixels at the K-tile's filter tap, zeros in the padding).
 // The operand stages are released by the epilogue: the group's accumulator commit (one per
 // group) is seen by epilogue thread 0, which frees the group's A and B stages, so no commit
 // is spent on them.
@@ -47,8 +47,11 @@
 namespace fgq {
 namespace {
 
+using tc::encode_im2col;
 using tc::encode_tiled;
+using tc::im2col_fits;
 using tc::make_map_2d;
+using tc::make_map_im2col;
 using tc::st_off;
 using tc::sw128;
 using tc::u8pair_to_h2;
@@ -58,18 +61,17 @@ constexpr int TC_BN = 128;        // positions per tile (MMA N)
 constexpr int TC_KT = 64;         // reduction elements per K-tile
 constexpr int TC_NO = 3;          // activation operand (B) ring depth
 constexpr int TC_NAS = 4;         // ternary operand (A) ring depth
-constexpr int TC_NS_TMA = 6;      // staging ring depth of the TMA path (room for the output tile)
-constexpr int TC_NS_GATHER = 12;  // staging ring depth of the gather path (about 1.5 us of copies)
+constexpr int TC_NS = 6;          // activation staging ring depth
 constexpr int TC_NACC = 4;        // TMEM accumulator buffers
 constexpr int TC_EPI_WARPS = 8;
 constexpr int TC_LOAD_WARPS = 4;
-constexpr int TC_LOADERS = 32 * TC_LOAD_WARPS;  // loader threads
-constexpr int TC_LPR = TC_LOADERS / 128;         // loader threads per tile row
-static_assert(TC_LPR == 1, "the cp.async gather path reads only copies made by the same thread");
-constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // loaders: warps 8 .. 8 + TC_LOAD_WARPS - 1
+constexpr int TC_LOADERS = 32 * TC_LOAD_WARPS;  // converter threads: one per tile row
+static_assert(TC_LOADERS == TC_BN, "one converter thread per tile row");
+constexpr int TC_LOAD_WARP0 = TC_EPI_WARPS;      // converters: warps 8 .. 8 + TC_LOAD_WARPS - 1
 constexpr int TC_MMA_WARP = TC_EPI_WARPS + TC_LOAD_WARPS;  // warp 12
 constexpr int TC_A_WARP = TC_MMA_WARP + 1;                 // warp 13: lane 0 streams the A boxes
-constexpr int TC_THREADS = 32 * (TC_A_WARP + 1);
+constexpr int TC_ACT_WARP = TC_A_WARP + 1;                 // warp 14: lane 0 streams the activation boxes
+constexpr int TC_THREADS = 32 * (TC_ACT_WARP + 1);
 constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
 constexpr uint32_t TC_WAIT_LIMIT = 50000;        // polls of up to 20 us: about 1 s per wait
 constexpr uint32_t TC_WAIT_SLEEP_NS = 20000;     // suspend hint of one poll
@@ -81,17 +83,15 @@ constexpr int ST_STAGE = TC_BN * TC_KT;                // 8 KB raw activation by
 constexpr int OUT_TILE = TC_BN * TC_BM * 4;            // 64 KB fp32 output tile
 constexpr int SMEM_A = TC_NAS * OP_TILE;
 constexpr int SMEM_B = TC_NO * OP_TILE;
-constexpr int SMEM_BAR = 8 * (2 * TC_NAS + 2 * TC_NO + 2 * TC_NS_GATHER + 2 * TC_NACC + 1) + 16;
-// TMA path: staging ring + fp32 output tile; gather path: a deeper staging ring, no tile.
-constexpr int SMEM_MID_TMA = TC_NS_TMA * ST_STAGE + OUT_TILE;
-constexpr int SMEM_MID_GATHER = TC_NS_GATHER * ST_STAGE;
-constexpr int SMEM_MID = SMEM_MID_TMA > SMEM_MID_GATHER ? SMEM_MID_TMA : SMEM_MID_GATHER;
+constexpr int SMEM_BAR = 8 * (2 * TC_NAS + 2 * TC_NO + 2 * TC_NS + 2 * TC_NACC + 1) + 16;
+constexpr int SMEM_MID = TC_NS * ST_STAGE + OUT_TILE;  // staging ring + fp32 output tile
 constexpr int TC_SMEM = 1024 + SMEM_A + SMEM_B + SMEM_MID + SMEM_BAR;
 static_assert(TC_SMEM <= 232448, "shared memory budget");
 
 struct TcArgs {
   CUtensorMap a16_map;    // fp16 [M][Kp] expanded codes, box {64, 128 rows}, 128-byte swizzle
-  CUtensorMap act_map;    // uint8 [pixels][row bytes], box {64 (or 32) bytes, 128 rows}; if act_tma
+  CUtensorMap act_map;    // act_tma: 2D uint8 [pixels][row bytes], box {64 (or 32) bytes, 128 rows};
+                          // otherwise the im2col map of the NHWC tensor, 128 pixels x 64 (32) bytes
   CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 128 positions}; if out_tma
   const uint8_t* act;
   const float* alpha;
@@ -105,7 +105,7 @@ struct TcArgs {
   int ntiles;       // groups * mtiles * ptiles
   int ktiles;       // K-tiles per tile (= ng * G / 64)
   int kt_per_group; // G / 64
-  int act_tma;      // activation rows by TMA (im2col rows are consecutive input rows)
+  int act_tma;      // 2D activation map (im2col rows are consecutive input rows); else im2col map
   int out_tma;      // output tile by TMA store (one conv group, M % 4 == 0)
   uint32_t wait_limit;     // polls per wait (each up to wait_sleep_ns)
   uint32_t wait_sleep_ns;
@@ -121,17 +121,17 @@ __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, 
   p0 = (int64_t)pt * TC_BN;
 }
 
-// TMAP: the layer's im2col rows are contiguous input rows (TMA loads, TMA-store epilogue);
-// otherwise rows are gathered with cp.async.
+// TMAP: the layer's im2col rows are contiguous input rows (2D box loads); otherwise the
+// activation boxes come from an im2col map (one load per K-tile: 128 output positions at
+// one filter tap and 64 channels, padding read as zeros).
 template <int ABITS, bool SIGNED, bool TMAP, bool SUMS>
 __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid_constant__ TcArgs a) {
-  constexpr int TC_NS = TMAP ? TC_NS_TMA : TC_NS_GATHER;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* abuf = smem;                             // TC_NAS A tiles
   uint8_t* bbuf = smem + SMEM_A;                    // TC_NO B tiles
   uint8_t* st = bbuf + SMEM_B;                      // TC_NS activation staging slots
-  float* otile = reinterpret_cast<float*>(st + TC_NS_TMA * ST_STAGE);  // TMA path: [128 pos][128 filters]
+  float* otile = reinterpret_cast<float*>(st + TC_NS * ST_STAGE);  // [128 positions][128 filters]
   uint64_t* bars = reinterpret_cast<uint64_t*>(st + SMEM_MID);
   uint64_t* a_full = bars;
   uint64_t* a_empty = bars + TC_NAS;
@@ -185,74 +185,46 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     record_error(a.err, FGQ_ERR_TIMEOUT);
   };
 
-  // ------------------------------------------------------------------ loaders/converters
-  if (warp >= TC_LOAD_WARP0 && warp < TC_MMA_WARP) {
-    const int tid = threadIdx.x - 32 * TC_LOAD_WARP0;
-    const int t = tid & (TC_BN - 1);  // tile row converted (and gathered) by this thread
-    const int h = tid >> 7;           // which part of the row (when TC_LPR > 1)
+  // ------------------------------------------------------------------ activation boxes
+  if (warp == TC_ACT_WARP && lane == 0) {
     const int total = my_tiles * a.ktiles;
-    constexpr int ROW_BYTES = TC_KT * ABITS / 8;     // 64 (8-bit) or 32 (4-bit)
-    constexpr int CPR = ROW_BYTES / 16;              // 16-byte chunks per activation row
-    constexpr int HC = CPR / TC_LPR;                 // activation chunks this thread handles
-    constexpr uint32_t TX_ACT = TC_BN * ROW_BYTES;
-
-    // per-tile state: conv group, first filter, this thread's row position; the filter
-    // tap (tr, ts) and channel offset tc0 of the next issued K-tile advance incrementally
-    int cur_tile = -1, gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0;
+    constexpr uint32_t TX_ACT = TC_BN * TC_KT * ABITS / 8;
+    // per tile: conv group and first position; the filter tap (tr, ts) and channel offset
+    // tc0 of the next K-tile advance incrementally
+    int gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0, kt = 0, tl = 0;
     int64_t p0 = 0;
-    int pb = 0, phb = 0, pwb = 0;
-    bool pvalid = false;
-    int issued = 0;  // K-tiles whose copies have been started
-    auto issue = [&](int j) {
-      const int tl = j / a.ktiles;
-      if (tl != cur_tile) {
-        cur_tile = tl;
+    int n0 = 0, h0 = 0, w0 = 0;  // im2col: the tile's first window origin (input pixel coordinates)
+    int issued = 0;
+    bool ok = true;
+    for (int j = 0; j < total; ++j) {
+      if (kt == 0) {
         tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
         tr = ts = tc0 = 0;
-        const int64_t p = p0 + t;
-        pvalid = p < g.P;
-        const int pp = pvalid ? (int)p : 0;
-        const int wo = pp % g.Wo;
-        const int q = pp / g.Wo;
-        const int ho = q % g.Ho;
-        pb = q / g.Ho;
-        phb = ho * g.stride - g.pad;
-        pwb = wo * g.stride - g.pad;
+        if (!TMAP) {
+          const int pp = (int)p0;  // < P < 2^31
+          const int wo = pp % g.Wo;
+          const int q = pp / g.Wo;
+          n0 = q / g.Ho;
+          h0 = (q - n0 * g.Ho) * g.stride - g.pad;
+          w0 = wo * g.stride - g.pad;
+        }
       }
       const int slot = j % TC_NS;
+      // the slot's previous contents (K-tile j - TC_NS) have been released by every converter
+      if (j >= TC_NS &&
+          !mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
+        ok = false;
+        break;
+      }
       uint8_t* sa = st + slot * ST_STAGE;
-      if (TMAP && tid == 0) {
-        // the slot's previous contents (K-tile j - TC_NS) have been released by every thread
-        bool free_ok = true;
-        if (j >= TC_NS)
-          free_ok = mbar_wait_or_abort(&st_empty[slot], ((j / TC_NS) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns);
-        if (free_ok) {
-          mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
-          tma_load_2d(smem_u32(sa), &a.act_map, (gi * g.Cg + tc0) * ABITS / 8, (int)p0, &st_full[slot]);
-          issued = j + 1;
-        } else {
-          if (!*abort_flag) fail();
-        }
-      }
-      if (!TMAP) {
-        const uint8_t* src = a.act;
-        bool inside = false;
-        if (pvalid) {
-          const int hi = phb + tr, wi = pwb + ts;
-          if (hi >= 0 && hi < g.H && wi >= 0 && wi < g.W) {
-            const int64_t e = (((int64_t)pb * g.H + hi) * g.W + wi) * g.C + (int64_t)gi * g.Cg + tc0;
-            src = a.act + e * ABITS / 8;
-            inside = true;
-          }
-        }
-#pragma unroll
-        for (int c = 0; c < HC; ++c) {
-          const int ch = h * HC + c;
-          cp_async16(smem_u32(sa + st_off<ABITS>(t, ch)), inside ? (const void*)(src + 16 * ch) : (const void*)a.act,
-                     inside ? 16u : 0u);
-        }
-      }
-      tc0 += TC_KT;  // next K-tile of this tile
+      const int cbyte = (gi * g.Cg + tc0) * ABITS / 8;  // a multiple of 32 bytes
+      mbar_arrive_expect_tx(&st_full[slot], TX_ACT);
+      if (TMAP)
+        tma_load_2d(smem_u32(sa), &a.act_map, cbyte, (int)p0, &st_full[slot]);
+      else
+        tma_load_im2col_4d(smem_u32(sa), &a.act_map, cbyte, w0, h0, n0, (uint16_t)ts, (uint16_t)tr, &st_full[slot]);
+      issued = j + 1;
+      tc0 += TC_KT;
       if (tc0 == g.Cg) {
         tc0 = 0;
         if (++ts == g.S) {
@@ -260,34 +232,39 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
           ++tr;
         }
       }
-    };
-
-    for (int j = 0; j < TC_NS - 1; ++j) {
-      if (j < total) issue(j);
-      cp_async_commit();
+      if (++kt == a.ktiles) {
+        kt = 0;
+        ++tl;
+      }
     }
-    int consumed = 0;
+    if (!ok && !*abort_flag) fail();
+    // loads the converters may not have consumed: the last TC_NS issued, one per slot, each
+    // the latest phase of its slot's barrier; none may outlive the CTA
+    for (int j = issued - TC_NS < 0 ? 0 : issued - TC_NS; j < issued; ++j)
+      mbar_wait_bounded(&st_full[j % TC_NS], (j / TC_NS) & 1, TC_DRAIN_LIMIT);
+  }
+
+  // ------------------------------------------------------------------ converters
+  if (warp >= TC_LOAD_WARP0 && warp < TC_MMA_WARP) {
+    const int tid = threadIdx.x - 32 * TC_LOAD_WARP0;
+    const int t = tid & (TC_BN - 1);  // tile row converted by this thread
+    const int total = my_tiles * a.ktiles;
     for (int j = 0; j < total; ++j) {
       if (*abort_flag) break;
-      if (j + TC_NS - 1 < total) issue(j + TC_NS - 1);
-      cp_async_commit();
-      if (!TMAP) cp_async_wait<TC_NS - 1>();  // this thread's copies for K-tile j have landed
       const int slot = j % TC_NS;
       const int os = j % TC_NO;
-      if ((TMAP && !mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) ||
+      if (!mbar_wait_or_abort(&st_full[slot], (j / TC_NS) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns) ||
           !mbar_wait_or_abort(&op_empty[os], ((j / TC_NO) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
         if (!*abort_flag) fail();
         break;
       }
-      consumed = j + 1;
       const uint8_t* sa = st + slot * ST_STAGE;
       uint8_t* Bt = bbuf + os * OP_TILE;
-      // activations -> fp16 (this thread's part of row t of B)
+      // activations of row t -> fp16, 128-byte-swizzled K-major
       if (ABITS == 8) {
         const uint32_t bias2 = SIGNED ? 0x64806480u : 0x64006400u;  // 1152 or 1024 in both halves
 #pragma unroll
-        for (int cc = 0; cc < HC; ++cc) {
-          const int c = HC * h + cc;
+        for (int c = 0; c < 4; ++c) {
           uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<8>(t, c));
           if (SIGNED) {
             v.x ^= 0x80808080u; v.y ^= 0x80808080u; v.z ^= 0x80808080u; v.w ^= 0x80808080u;
@@ -303,38 +280,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       } else {
         const uint32_t bias2 = SIGNED ? 0x64086408u : 0x64006400u;  // 1032 or 1024
 #pragma unroll
-        for (int cc = 0; cc < HC; ++cc) {
-        const int c = HC * h + cc;
-        const uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<4>(t, c));
-        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+        for (int c = 0; c < 2; ++c) {
+          const uint4 v = *reinterpret_cast<const uint4*>(sa + st_off<4>(t, c));
+          const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          // 8 nibbles -> 8 bytes (element order preserved), then 8 fp16
-          const uint32_t x = w4[q];
-          const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
-          const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
-          uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                            // e0 e1 e2 e3
-          uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                                    // e4 e5 e6 e7
-          if (SIGNED) {
-            b0 ^= 0x08080808u;
-            b1 ^= 0x08080808u;
+          for (int q = 0; q < 4; ++q) {
+            // 8 nibbles -> 8 bytes (element order preserved), then 8 fp16
+            const uint32_t x = w4[q];
+            const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
+            const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
+            uint32_t b0 = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                            // e0 e1 e2 e3
+            uint32_t b1 = (lo >> 16) | (hi & 0xffff0000u);                                    // e4 e5 e6 e7
+            if (SIGNED) {
+              b0 ^= 0x08080808u;
+              b1 ^= 0x08080808u;
+            }
+            uint4 o;
+            o.x = u8pair_to_h2(b0, 0x4140, bias2); o.y = u8pair_to_h2(b0, 0x4342, bias2);
+            o.z = u8pair_to_h2(b1, 0x4140, bias2); o.w = u8pair_to_h2(b1, 0x4342, bias2);
+            *reinterpret_cast<uint4*>(Bt + sw128(t, 4 * c + q)) = o;
           }
-          uint4 o;
-          o.x = u8pair_to_h2(b0, 0x4140, bias2); o.y = u8pair_to_h2(b0, 0x4342, bias2);
-          o.z = u8pair_to_h2(b1, 0x4140, bias2); o.w = u8pair_to_h2(b1, 0x4342, bias2);
-          *reinterpret_cast<uint4*>(Bt + sw128(t, 4 * c + q)) = o;
-        }
         }
       }
       fence_proxy_async_smem();
       mbar_arrive(&op_full[os]);
-      if (TMAP) mbar_arrive(&st_empty[slot]);  // done reading this TMA-filled staging slot
-    }
-    cp_async_wait_all();
-    // TMA loads issued but not consumed (only after a failure): wait, bounded, for their
-    // bytes to land so that no copy into this CTA's shared memory outlives it
-    if (tid == 0) {
-      for (int j = consumed; j < issued; ++j) mbar_wait_bounded(&st_full[j % TC_NS], (j / TC_NS) & 1, TC_DRAIN_LIMIT);
+      mbar_arrive(&st_empty[slot]);  // done reading this staging slot
     }
   }
 
@@ -480,7 +450,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       }
       if (named_bar_or(BAR_EPI, 32 * TC_EPI_WARPS, !ok)) break;  // leave together
       if (SUMS) continue;  // the group sums are stored already
-      if (TMAP && a.out_tma) {
+      if (a.out_tma) {
         // the previous tile's store has finished reading the staging tile
         if (leader) bulk_wait_read_all();
         named_bar_sync(BAR_EPI, 32 * TC_EPI_WARPS);
@@ -559,6 +529,9 @@ bool tc_supports(const Geom& g) {
   if (g.C % 16 != 0) return false;            // 16-byte aligned activation rows
   if (g.P >= (int64_t)1 << 31) return false;  // positions decoded in 32 bits
   if (encode_tiled() == nullptr) return false;
+  if (!(g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) &&
+      (encode_im2col() == nullptr || !im2col_fits(g.R, g.S, g.stride, g.pad)))
+    return false;
   return true;
 }
 
@@ -596,15 +569,20 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                                    (uint64_t)g.M, (uint64_t)g.wrow * 32, TC_KT, TC_BM, CU_TENSOR_MAP_SWIZZLE_128B))
     st = FGQ_ERR_CUDA;
   // im2col rows are consecutive input rows for a 1x1, stride-1, unpadded convolution or a GEMM
+  const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
+  const CUtensorMapSwizzle act_sw = abits == 8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B;
+  bool act_ok;
   if (g.R == 1 && g.S == 1 && g.stride == 1 && g.pad == 0) {
-    const uint64_t row_bytes = (uint64_t)g.C * abits / 8;
-    a.act_tma = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, row_bytes, (uint64_t)g.B * g.H * g.W,
-                            row_bytes, (uint32_t)(TC_KT * abits / 8), TC_BN,
-                            abits == 8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B)
-                    ? 1
-                    : 0;
+    a.act_tma = 1;
+    act_ok = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_UINT8, act, row_bytes, (uint64_t)g.B * g.H * g.W,
+                         row_bytes, (uint32_t)(TC_KT * abits / 8), TC_BN, act_sw);
+  } else {
+    a.act_tma = 0;
+    act_ok = make_map_im2col(&a.act_map, act, row_bytes, g.B, g.H, g.W, g.R, g.S, g.stride, g.pad,
+                             (uint32_t)(TC_KT * abits / 8), TC_BN, act_sw);
   }
-  if (a.act_tma && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums) {
+  if (st == FGQ_OK && !act_ok) st = FGQ_ERR_CUDA;
+  if (g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums) {
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, TC_BM, TC_BN, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1

@@ -265,6 +265,17 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst_smem, const void* tmap,
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
       : "memory");
 }
+// im2col load of a 4D NHWC tensor: pixelsPerColumn pixels (the map's column) starting at
+// pixel (n, h, w) of the map's bounding box, each shifted by the filter tap (dw, dh), with
+// the map's channelsPerPixel channels from channel c; pixels outside the tensor read as 0.
+__device__ __forceinline__ void tma_load_im2col_4d(uint32_t dst_smem, const void* tmap, int c, int w, int h, int n,
+                                                   uint16_t dw, uint16_t dh, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
+      "%5}], [%6], {%7, %8};" ::"r"(dst_smem),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c), "r"(w), "r"(h), "r"(n), "r"(smem_u32(bar)), "h"(dw), "h"(dh)
+      : "memory");
+}
 // Store a box from shared memory; out-of-range rows/columns of the box are not written.
 __device__ __forceinline__ void tma_store_2d(const void* tmap, int c0, int c1, uint32_t src_smem) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(

@@ -108,6 +108,46 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_tiled() {
   return fn;
 }
 
+// cuTensorMapEncodeIm2col from the driver, looked up once through the runtime.
+inline PFN_cuTensorMapEncodeIm2col_v12000 encode_im2col() {
+  static PFN_cuTensorMapEncodeIm2col_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeIm2col_v12000>(p);
+  });
+  return fn;
+}
+
+// im2col map of a byte tensor [B][H][W][row_bytes] for a convolution with an R x S filter,
+// stride and zero padding pad: the bounding box of the filter windows' top-left pixels runs
+// from -pad to W + pad - S (H + pad - R), walked with the convolution's stride, so that
+// consecutive pixels of a column are consecutive output positions; each pixel contributes
+// `pixel_bytes` bytes (channels) to a row of the box.
+inline bool make_map_im2col(CUtensorMap* m, const void* base, uint64_t row_bytes, int B, int H, int W, int R, int S,
+                            int stride, int pad, uint32_t pixel_bytes, uint32_t pixels, CUtensorMapSwizzle sw) {
+  auto enc = encode_im2col();
+  if (!enc) return false;
+  const cuuint64_t dims[4] = {row_bytes, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)B};
+  const cuuint64_t strides[3] = {row_bytes, row_bytes * (cuuint64_t)W, row_bytes * (cuuint64_t)W * (cuuint64_t)H};
+  const int lower[2] = {-pad, -pad};                   // {W, H}
+  const int upper[2] = {pad - (S - 1), pad - (R - 1)};  // {W, H}
+  const cuuint32_t estr[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(base), dims, strides, lower, upper, pixel_bytes,
+             pixels, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Whether a convolution's geometry fits an im2col map (the corner offsets of a 4D map are
+// 8-bit signed, the traversal stride at most 8).
+inline bool im2col_fits(int R, int S, int stride, int pad) {
+  const int lo = -pad, up_w = pad - (S - 1), up_h = pad - (R - 1);
+  return stride >= 1 && stride <= 8 && lo >= -128 && up_w >= -128 && up_w <= 127 && up_h >= -128 && up_h <= 127;
+}
+
 // 2D tiled map: dims {d0 (innermost), d1}, row pitch in bytes, box {b0, b1}.
 inline bool make_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t d0, uint64_t d1,
                  uint64_t pitch, uint32_t b0, uint32_t b1, CUtensorMapSwizzle sw) {

@@ -166,6 +166,13 @@ CONV_CASES = [
     (1, 10, 10, 128, 64, 3, 3, 1, 1, 1, 64, "u4"),
     (1, 8, 8, 64, 32, 3, 3, 1, 1, 1, 4, "s4"),
     (1, 9, 9, 6, 8, 3, 3, 1, 1, 1, 4, "u4"),         # 4-bit with C % 4 != 0
+    # G >= 64 tensor-core im2col boxes: H != W, R != S, strides, conv groups, packed 4-bit
+    (2, 9, 13, 64, 64, 3, 3, 1, 1, 1, 64, "u8"),
+    (1, 9, 12, 64, 64, 1, 3, 1, 1, 1, 64, "u8"),
+    (2, 11, 10, 128, 72, 3, 1, 2, 1, 1, 64, "s8"),
+    (2, 12, 12, 128, 64, 3, 3, 2, 1, 1, 128, "u4"),
+    (1, 8, 8, 256, 128, 3, 3, 1, 1, 2, 64, "u8"),
+    (1, 15, 15, 64, 64, 5, 5, 3, 2, 1, 64, "s4"),
 ]
 
 
