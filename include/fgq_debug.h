@@ -70,6 +70,13 @@ int64_t fgq_debug_set_wait_limit_us(int64_t us);
  */
 int fgq_debug_allow_split_fold(int allow);
 
+/*
+ * The CUDA runtime error (a cudaError_t value) behind the last FGQ_ERR_CUDA that a kernel
+ * launch of this thread returned, 0 if none; reading it clears it.  `name` receives the
+ * runtime's name of that error (at most `len` bytes including the terminator) when non-null.
+ */
+int fgq_debug_last_cuda_error(char* name, size_t len);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,6 +24,7 @@ thread_local int t_path = FGQ_PATH_AUTO;
 thread_local int t_last_path = FGQ_PATH_AUTO;
 thread_local int64_t t_wait_limit_us = -1;
 thread_local int t_split_fold = 0;
+thread_local int t_last_cuda_error = 0;  // cudaError_t of the last failed launch on this thread
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
@@ -180,7 +181,10 @@ unsigned int* device_error_word() {
 
 fgq_status after_launch() {
   g_launches.fetch_add(1);
-  return cudaGetLastError() == cudaSuccess ? FGQ_OK : FGQ_ERR_CUDA;
+  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) return FGQ_OK;
+  t_last_cuda_error = (int)e;
+  return FGQ_ERR_CUDA;
 }
 
 int64_t debug_wait_limit_us() { return t_wait_limit_us; }
@@ -670,6 +674,18 @@ int fgq_debug_allow_split_fold(int allow) {
   const int prev = t_split_fold;
   t_split_fold = allow ? 1 : 0;
   return prev;
+}
+
+int fgq_debug_last_cuda_error(char* name, size_t len) {
+  const int e = t_last_cuda_error;
+  t_last_cuda_error = 0;
+  if (name && len > 0) {
+    const char* n = e ? cudaGetErrorName((cudaError_t)e) : "";
+    size_t i = 0;
+    for (; n[i] && i + 1 < len; ++i) name[i] = n[i];
+    name[i] = 0;
+  }
+  return e;
 }
 
 int fgq_last_path(void) { return t_last_path; }

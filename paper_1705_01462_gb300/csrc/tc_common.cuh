@@ -122,22 +122,24 @@ inline PFN_cuTensorMapEncodeIm2col_v12000 encode_im2col() {
   return fn;
 }
 
-// im2col map of a byte tensor [B][H][W][row_bytes] for a convolution with an R x S filter,
-// stride and zero padding pad: the bounding box of the filter windows' top-left pixels runs
-// from -pad to W + pad - S (H + pad - R), walked with the convolution's stride, so that
-// consecutive pixels of a column are consecutive output positions; each pixel contributes
-// `pixel_bytes` bytes (channels) to a row of the box.
-inline bool make_map_im2col(CUtensorMap* m, const void* base, uint64_t row_bytes, int B, int H, int W, int R, int S,
-                            int stride, int pad, uint32_t pixel_bytes, uint32_t pixels, CUtensorMapSwizzle sw) {
+// im2col map of an NHWC tensor [B][H][W][C] (elements of elem_bytes bytes) for a
+// convolution with an R x S filter, stride and zero padding pad: the bounding box of the
+// filter windows' top-left pixels runs from -pad to W + pad - S (H + pad - R), walked with
+// the convolution's stride, so that consecutive pixels of a column are consecutive output
+// positions; each pixel contributes `pixel_elems` channels to a row of the box.
+inline bool make_map_im2col(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t C, uint64_t elem_bytes,
+                            int B, int H, int W, int R, int S, int stride, int pad, uint32_t pixel_elems,
+                            uint32_t pixels, CUtensorMapSwizzle sw) {
   auto enc = encode_im2col();
   if (!enc) return false;
-  const cuuint64_t dims[4] = {row_bytes, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)B};
-  const cuuint64_t strides[3] = {row_bytes, row_bytes * (cuuint64_t)W, row_bytes * (cuuint64_t)W * (cuuint64_t)H};
+  const uint64_t row = C * elem_bytes;
+  const cuuint64_t dims[4] = {C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)B};
+  const cuuint64_t strides[3] = {row, row * (cuuint64_t)W, row * (cuuint64_t)W * (cuuint64_t)H};
   const int lower[2] = {-pad, -pad};                   // {W, H}
   const int upper[2] = {pad - (S - 1), pad - (R - 1)};  // {W, H}
   const cuuint32_t estr[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<void*>(base), dims, strides, lower, upper, pixel_bytes,
-             pixels, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+  return enc(m, dt, 4, const_cast<void*>(base), dims, strides, lower, upper, pixel_elems, pixels, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 

@@ -64,6 +64,7 @@ SIGNATURES = [
     ("fgq_selftest_wait_timeout", _i, [_u32, _vp]),
     ("fgq_debug_set_wait_limit_us", _i64, [_i64]),
     ("fgq_debug_allow_split_fold", _i, [_i]),
+    ("fgq_debug_last_cuda_error", _i, [_vp, _sz]),
 ]
 
 
@@ -488,6 +489,13 @@ def fgq_debug_set_wait_limit_us(us: int) -> int:
 def fgq_debug_allow_split_fold(allow: bool) -> int:
     """Lets FGQ_PATH_DENSE run fp32 alphas as the split-fp16 ablation on this thread."""
     return int(lib().fgq_debug_allow_split_fold(1 if allow else 0))
+
+
+def fgq_debug_last_cuda_error() -> tuple:
+    """(cudaError_t value, name) behind this thread's last FGQ_ERR_CUDA from a launch; clears it."""
+    buf = ctypes.create_string_buffer(64)
+    code = int(lib().fgq_debug_last_cuda_error(buf, 64))
+    return code, buf.value.decode()
 
 
 def fgq_last_path() -> int:
