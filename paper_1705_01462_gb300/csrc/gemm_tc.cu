@@ -21,16 +21,17 @@
 // R * S filter taps and M / 128 filter tiles; converting it once instead of at every use
 // takes the conversion off the MMA's path.
 //
-// Warp roles (320 threads, one CTA per SM, persistent over tiles):
+// Warp roles (352 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
 //              128*(w/4).. (positions) of the drained buffer in four 32-column tcgen05.ld,
 //              frees the buffer, and adds alpha * s into 128 fp32 registers.  At tile end
 //              it stores the tile directly (32 lanes = 32 consecutive filters: one 128-byte
 //              segment per position), requantized when asked.
-//   warp 8     TMEM allocation and the MMA issuer (one thread): 4 tcgen05.mma (M = 128,
-//              N = 256, K = 16) per K-tile into one of the two accumulators, one commit per
-//              group.
-//   warp 9     the producer (one thread): per K-tile, the ternary box (64 reduction
+//   warps 8, 9 the MMA issuers (one thread each; warp 8 also allocates TMEM): the even groups
+//              into accumulator 0 and the odd groups into accumulator 1, 4 tcgen05.mma
+//              (M = 128, N = 256, K = 16) per K-tile and one commit per group; while one
+//              thread waits on its barriers, the other's MMAs keep the tensor pipe busy.
+//   warp 10    the producer (one thread): per K-tile, the ternary box (64 reduction
 //              elements x 128 filters) and the activation box (64 channels x 256 positions)
 //              into one four-stage ring: a 2D box of consecutive input rows when the im2col
 //              rows are input rows (1x1 stride-1 convolutions, GEMMs), otherwise an im2col
@@ -62,8 +63,8 @@ constexpr int TC_KT = 64;         // reduction elements per K-tile
 constexpr int TC_NST = 3;         // operand ring depth (stages of A + B)
 constexpr int TC_NACC = 2;        // TMEM accumulator buffers
 constexpr int TC_EPI_WARPS = 8;
-constexpr int TC_MMA_WARP = TC_EPI_WARPS;       // warp 8
-constexpr int TC_PROD_WARP = TC_EPI_WARPS + 1;  // warp 9: lane 0 streams both operands
+constexpr int TC_MMA_WARP = TC_EPI_WARPS;       // warps 8 and 9: MMA issuers of even and odd groups
+constexpr int TC_PROD_WARP = TC_EPI_WARPS + 2;  // warp 10: lane 0 streams both operands
 constexpr int TC_THREADS = 32 * (TC_PROD_WARP + 1);
 constexpr int TC_TMEM_COLS = TC_NACC * TC_BN;    // 512: all of TMEM
 constexpr int TC_EPI_COLS = TC_BN / 2;           // positions per epilogue thread
@@ -232,7 +233,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], TC_EPI_WARPS);  // one arrival per epilogue warp
     }
-    mbar_init(drain_bar, 1);
+    mbar_init(drain_bar, TC_NACC);  // one commit per MMA issuer
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -310,14 +311,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       mbar_wait_bounded(&full[j % TC_NST], (j / TC_NST) & 1, TC_DRAIN_LIMIT);
   }
 
-  // ------------------------------------------------------------------ MMA issuer
-  if (warp == TC_MMA_WARP && lane == 0) {
+  // ------------------------------------------------------------------ MMA issuers
+  // Two threads issue the MMAs, one for the even and one for the odd groups, each into its
+  // own TMEM accumulator: one thread's barrier waits and commit overlap the other's MMAs.
+  if ((warp == TC_MMA_WARP || warp == TC_MMA_WARP + 1) && lane == 0) {
+    const int b = warp - TC_MMA_WARP;  // accumulator = parity of the groups this thread issues
     const uint32_t idesc = idesc_f16_f32(TC_BM, TC_BN);
     int kt = 0, gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
       for (int grp = 0; grp < g.ng && ok; ++grp, ++gc) {
-        const int b = gc & 1;
+        if ((gc & 1) != b) {
+          kt += a.kt_per_group;  // the other issuer's group
+          continue;
+        }
         if (!mbar_wait_or_abort(&acc_empty[b], ((gc >> 1) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
           if (!*abort_flag) fail();
           ok = false;
@@ -344,7 +351,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
         if (ok) mma_commit(&acc_full[b]);
       }
     }
-    // all MMAs issued by this thread are complete once the drain barrier flips
+    // all MMAs issued by both threads are complete once the drain barrier flips
     mma_commit(drain_bar);
     mbar_wait_bounded(drain_bar, 0, TC_DRAIN_LIMIT);
   }
@@ -533,20 +540,48 @@ __global__ void wait_timeout_selftest_kernel(uint32_t max_iter, unsigned int* er
   if (!ok && threadIdx.x == 0) record_error(err, FGQ_ERR_TIMEOUT);
 }
 
-// A 1x1 unpadded convolution (any stride) or a GEMM: one activation row per output position
-// (gathered when strided), loaded by 2D boxes.
-bool pointwise(const Geom& g) { return g.R == 1 && g.S == 1 && g.pad == 0; }
-
 }  // namespace
+
+namespace tc {
+
+bool act_pointwise(const Geom& g) { return g.R == 1 && g.S == 1 && g.pad == 0; }
+
+int64_t act16_elems(const Geom& g) {
+  return act_pointwise(g) && g.stride > 1 ? g.P * g.C : (int64_t)g.B * g.H * g.W * g.C;
+}
+
+fgq_status expand_act16(const void* act, const Geom& g, void* x16, cudaStream_t s) {
+  const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
+  const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
+  if (abits == 4)
+    return sgn ? expand_activations<4, true>(act, g, x16, s) : expand_activations<4, false>(act, g, x16, s);
+  return sgn ? expand_activations<8, true>(act, g, x16, s) : expand_activations<8, false>(act, g, x16, s);
+}
+
+bool act16_map(CUtensorMap* m, const void* x16, const Geom& g, uint32_t pixels) {
+  if (act_pointwise(g))
+    return make_map_2d(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)g.C, (uint64_t)(act16_elems(g) / g.C),
+                       (uint64_t)g.C * 2, 64, pixels, CU_TENSOR_MAP_SWIZZLE_128B);
+  return make_map_im2col(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)g.C, 2, g.B, g.H, g.W, g.R, g.S, g.stride,
+                         g.pad, 64, pixels, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+bool act16_supported(const Geom& g) {
+  if (g.C % 16 != 0 || g.Cg % 64 != 0) return false;
+  if (encode_tiled() == nullptr) return false;
+  return act_pointwise(g) || (encode_im2col() != nullptr && im2col_fits(g.R, g.S, g.stride, g.pad));
+}
+
+}  // namespace tc
+
+using tc::act_pointwise;
 
 bool tc_supports(const Geom& g) {
   if (g.G != 64 && g.G != 128) return false;
-  if (g.Cg % TC_KT != 0) return false;        // every K-tile inside one filter tap (conv) or row (GEMM)
-  if (g.C % 16 != 0) return false;            // 16-element chunks of the activation expansion
   if (g.P >= (int64_t)1 << 31) return false;  // positions decoded in 32 bits
-  if (encode_tiled() == nullptr) return false;
-  if (!pointwise(g) && (encode_im2col() == nullptr || !im2col_fits(g.R, g.S, g.stride, g.pad))) return false;
-  return true;
+  // every K-tile inside one filter tap (conv) or row (GEMM); 16-element expansion chunks;
+  // activation boxes by 2D or im2col maps
+  return tc::act16_supported(g);
 }
 
 fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* codes, const float* alpha,
@@ -570,15 +605,12 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   const int64_t lim_us = debug_wait_limit_us();
   a.wait_limit = lim_us < 0 ? TC_WAIT_LIMIT : (uint32_t)(lim_us / 20 + 1);
   a.wait_sleep_ns = lim_us < 0 ? TC_WAIT_SLEEP_NS : (uint32_t)(lim_us < 20 ? lim_us * 1000 : 20000);
-  const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
-  const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
   // temporaries from the stream-ordered pool: the codes as fp16 [M][Kp] (Kp = 16 wrow) and
   // the activations as fp16 NHWC (a strided 1x1 convolution: only the pixels it reads, [P][C])
   cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
   const int64_t nwords = (int64_t)g.M * g.wrow;
-  const bool gathered = pointwise(g) && g.stride > 1;
-  const int64_t nact = gathered ? g.P * g.C : (int64_t)g.B * g.H * g.W * g.C;
+  const int64_t nact = tc::act16_elems(g);
   void* a16 = nullptr;
   void* x16 = nullptr;
   if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 32, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
@@ -587,28 +619,12 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
     return FGQ_ERR_CUDA;
   }
   fgq_status st = launch_expand_codes(codes, nwords, a16, s);
-  if (st == FGQ_OK) {
-    if (abits == 4)
-      st = sgn ? expand_activations<4, true>(act, g, x16, s) : expand_activations<4, false>(act, g, x16, s);
-    else
-      st = sgn ? expand_activations<8, true>(act, g, x16, s) : expand_activations<8, false>(act, g, x16, s);
-  }
+  if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
   if (st == FGQ_OK && !make_map_2d(&a.a16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a16, (uint64_t)g.wrow * 16,
                                    (uint64_t)g.M, (uint64_t)g.wrow * 32, TC_KT, TC_BM, CU_TENSOR_MAP_SWIZZLE_128B))
     st = FGQ_ERR_CUDA;
-  if (st == FGQ_OK) {
-    bool act_ok;
-    if (pointwise(g)) {
-      a.act_tma = 1;
-      act_ok = make_map_2d(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)g.C, (uint64_t)(nact / g.C),
-                           (uint64_t)g.C * 2, TC_KT, TC_BN, CU_TENSOR_MAP_SWIZZLE_128B);
-    } else {
-      a.act_tma = 0;
-      act_ok = make_map_im2col(&a.act_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x16, (uint64_t)g.C, 2, g.B, g.H, g.W,
-                               g.R, g.S, g.stride, g.pad, TC_KT, TC_BN, CU_TENSOR_MAP_SWIZZLE_128B);
-    }
-    if (!act_ok) st = FGQ_ERR_CUDA;
-  }
+  a.act_tma = act_pointwise(g) ? 1 : 0;
+  if (st == FGQ_OK && !tc::act16_map(&a.act_map, x16, g, TC_BN)) st = FGQ_ERR_CUDA;
   if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums)
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, TC_BM, OUT_POS, CU_TENSOR_MAP_SWIZZLE_NONE)

@@ -163,5 +163,15 @@ inline bool make_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base
              CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The activations of the tensor-core kernels as fp16 integers (defined with the G >= 64
+// kernel): NHWC, or [P][C] -- only the pixels a strided 1x1 unpadded convolution reads.
+bool act_pointwise(const Geom& g);         // 1x1, unpadded (any stride), or a GEMM: 2D rows
+int64_t act16_elems(const Geom& g);        // elements of the fp16 copy
+fgq_status expand_act16(const void* act, const Geom& g, void* x16, cudaStream_t s);
+// 2D map (pointwise) or im2col map of the fp16 copy: boxes of `pixels` output positions x 64
+// channels, 128-byte swizzle
+bool act16_map(CUtensorMap* m, const void* x16, const Geom& g, uint32_t pixels);
+bool act16_supported(const Geom& g);       // C % 16 == 0, Cg % 64 == 0, a map for the geometry
+
 }  // namespace tc
 }  // namespace fgq
