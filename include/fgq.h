@@ -13,8 +13,12 @@
  * weight (Section 4.1).
  *
  * Conventions for every call
- *   - All array pointers are DEVICE pointers owned by the caller; the library allocates
- *     nothing.  Calls are asynchronous and ordered on the given CUDA stream.
+ *   - All array pointers are DEVICE pointers owned by the caller (fgq_conv2d_host: host
+ *     pointers).  Calls are asynchronous and ordered on the given CUDA stream.  The only
+ *     allocations of the library are per-call temporaries (operands expanded or folded for
+ *     the tensor cores) from a library-owned stream-ordered memory pool of the current
+ *     device, allocated and freed on the call's stream; fgq_quantize_act_noalloc allocates
+ *     nothing.
  *   - The return value reports errors found on the host (argument, alignment, unsupported
  *     shape, CUDA launch failure).  Errors found by a kernel (non-finite input, a bounded
  *     wait that ran out) are recorded in a device error word and returned by
@@ -244,10 +248,13 @@ fgq_status fgq_quantize_weights_w8(const float* w, int M, int Kred, int8_t* wq, 
  *   codes, alpha as produced by fgq_ternarize for (M, Kred, G).
  *   y          out, fp32 [P][M].
  * The fp32 result is within 1e-5 * act_scale * sum_g |alpha_g * s_g| of the exact value.
- * Memory: the tensor-core G = 4 kernel expands the codes to fp16 (2 * M * Kred bytes) in a
- * temporary taken from a library-owned stream-ordered pool of the current device and
- * returned to it on the same stream; the pool keeps freed blocks, so only a call that needs
- * more than the pool holds reaches the device allocator.  No other path allocates.
+ * Memory: the tensor-core kernels take per-call temporaries from a library-owned
+ * stream-ordered pool of the current device and return them on the same stream: the
+ * activations as fp16 (2 bytes per element read), and the ternary operand -- at G >= 64
+ * the codes as fp16 (2 * M * Kp bytes), at G = 4 its block-diagonal form (4 * 2 * M' * Kp
+ * bytes per fp16 part, two parts for fp32 alphas, M' = M rounded up to 32 per conv group).
+ * The pool keeps freed blocks, so only a call that needs more than the pool holds reaches
+ * the device allocator.  The dp4a and few-row paths allocate nothing.
  * Errors: FGQ_ERR_ARG (null pointers, bad sizes, Kred odd for 4-bit types),
  * FGQ_ERR_ALIGN (any pointer not 16-byte aligned), FGQ_ERR_CUDA.
  */

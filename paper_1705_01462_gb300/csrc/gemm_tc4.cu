@@ -44,6 +44,8 @@
 // no commit is spent on the stages.  Every mbarrier wait is bounded in time; on expiry the
 // kernel records FGQ_ERR_TIMEOUT, each role leaves its loop (uniformly within the epilogue,
 // which uses named barriers), in-flight copies and MMAs are waited for, and TMEM is freed.
+#include <cuda_fp16.h>
+
 #include <cstdint>
 #include <cstring>
 
@@ -132,12 +134,35 @@ __global__ void __launch_bounds__(256) expand_codes_kernel(const uint32_t* __res
   a16[2 * i + 1] = make_uint4(h[4], h[5], h[6], h[7]);
 }
 
-// Block-diagonal A' from a dense fp16 operand src [M][Kp]: row 4 m' + j of tile (gi, mt)
-// keeps, of filter gi Mg + mt 32 + m', the elements of the groups whose index is j modulo 4
-// (slot j of every K = 16 step) and zeros elsewhere.  One thread per 16-byte chunk (8
-// elements = 2 groups) of A'.
-__global__ void __launch_bounds__(256) diag_kernel(const uint2* __restrict__ src, int Kp, int Mg, int mtiles,
-                                                   int64_t nchunks, uint4* __restrict__ dst) {
+// Row scales of the folded operand, one warp per filter row: e_m puts the row's largest
+// alpha in [2^14, 2^15) (clamped to [-100, 100]; an all-zero row keeps e = 0), so that the
+// low fp16 part of every alpha stays clear of fp16's subnormal range; rs[m] = 2^-e_m.
+__global__ void __launch_bounds__(256) row_scale_kernel(const float* __restrict__ alpha, int M, int ng,
+                                                        float* __restrict__ rs) {
+  const int m = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  float mx = 0.0f;
+  for (int g = lane; g < ng; g += 32) mx = fmaxf(mx, __ldg(alpha + (int64_t)m * ng + g));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  int e = mx > 0.0f ? 14 - ilogbf(mx) : 0;
+  e = e < -100 ? -100 : (e > 100 ? 100 : e);
+  if (lane == 0) rs[m] = ldexpf(1.0f, -e);
+}
+
+// The block-diagonal ternary operand A', straight from the 2-bit codes: row 4 m' + j of tile
+// (gi, mt) holds, for filter gi Mg + mt 32 + m', the elements of the groups whose index is j
+// modulo 4 (slot j of every K = 16 step) and zeros elsewhere.  FOLD: the elements are
+// alpha(m, g) 2^e_m t split into fp16 hi + lo (hi the fp16 nearest, lo the fp16 nearest the
+// remainder), parts a0 and a1; otherwise the codes as fp16 {0, +1, -1} in a0.  One thread
+// per 16-byte chunk (8 elements = 2 groups, at most one of them in the row's slot).
+template <bool FOLD>
+__global__ void __launch_bounds__(256) fold_diag_kernel(const uint32_t* __restrict__ codes, int wrow,
+                                                        const float* __restrict__ alpha, int ng,
+                                                        const float* __restrict__ rs, int Kp, int Mg, int mtiles,
+                                                        int64_t nchunks, uint4* __restrict__ a0,
+                                                        uint4* __restrict__ a1) {
   const int cpr = Kp / 8;  // chunks per row
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = i / cpr;
@@ -147,21 +172,44 @@ __global__ void __launch_bounds__(256) diag_kernel(const uint2* __restrict__ src
     const int mp = rr >> 2, j = rr & 3;
     const int gi = (int)(tile / mtiles), mt = (int)(tile - (int64_t)gi * mtiles);
     const int local = mt * T4_FM + mp;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (local < Mg) {
+    uint32_t h0[4] = {0u, 0u, 0u, 0u}, h1[4] = {0u, 0u, 0u, 0u};
+    // group 2c occupies halves 0-3 of the chunk, group 2c + 1 halves 4-7; slot = group % 4
+    const int grp = ((2 * c) & 3) == j ? 2 * c : (((2 * c + 1) & 3) == j ? 2 * c + 1 : -1);
+    if (local < Mg && grp >= 0 && grp < ng) {
       const int64_t m = (int64_t)gi * Mg + local;
-      const int g0 = 2 * c;  // first group of the chunk; slot = group % 4
-      if ((g0 & 3) == j) {
-        const uint2 h = __ldg(src + (m * Kp + 8 * c) / 4);
-        v.x = h.x;
-        v.y = h.y;
-      } else if (((g0 + 1) & 3) == j) {
-        const uint2 h = __ldg(src + (m * Kp + 8 * c + 4) / 4);
-        v.z = h.x;
-        v.w = h.y;
+      const int k0 = 4 * grp;  // the group's 4 codes lie in one word, bits 2 (k0 % 16) ..
+      const uint32_t cw = (__ldg(codes + m * wrow + k0 / 16) >> (2 * (k0 % 16))) & 0xffu;
+      uint32_t hi = 0x3C00u, lo = 0u;  // fp16 +1 and 0: the codes themselves
+      if (FOLD) {
+        const float v = __ldg(alpha + m * ng + grp) / __ldg(rs + m);  // exact: a power-of-two scaling
+        const __half hh = __float2half_rn(v);
+        hi = __half_as_ushort(hh);
+        lo = __half_as_ushort(__float2half_rn(v - __half2float(hh)));  // the remainder, exact in fp32
       }
+      uint32_t e0[4], e1[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t t = (cw >> (2 * e)) & 3u;  // 00 = 0, 01 = +1, 11 = -1
+        const uint32_t sgn = t == 3u ? 0x8000u : 0u;
+        const bool nz = t == 1u || t == 3u;
+        e0[e] = nz ? (hi ^ sgn) : 0u;
+        e1[e] = nz && lo ? (lo ^ sgn) : 0u;
+      }
+      // the group fills 32-bit words 0-1 of the chunk (group 2c) or 2-3 (group 2c + 1)
+      const bool first = grp == 2 * c;
+      const uint32_t p0 = e0[0] | (e0[1] << 16), p1 = e0[2] | (e0[3] << 16);
+      const uint32_t q0 = e1[0] | (e1[1] << 16), q1 = e1[2] | (e1[3] << 16);
+      h0[0] = first ? p0 : 0u;
+      h0[1] = first ? p1 : 0u;
+      h0[2] = first ? 0u : p0;
+      h0[3] = first ? 0u : p1;
+      h1[0] = first ? q0 : 0u;
+      h1[1] = first ? q1 : 0u;
+      h1[2] = first ? 0u : q0;
+      h1[3] = first ? 0u : q1;
     }
-    dst[i] = v;
+    a0[i] = make_uint4(h0[0], h0[1], h0[2], h0[3]);
+    if (FOLD) a1[i] = make_uint4(h1[0], h1[1], h1[2], h1[3]);
   }
 }
 
@@ -459,16 +507,28 @@ fgq_status launch_tc4(const T4Args& args, int grid, cudaStream_t s) {
   return after_launch();
 }
 
-fgq_status launch_diag(const void* src, int Kp, int Mg, int mtiles, int64_t rows, void* dst, cudaStream_t s) {
-  const int64_t nchunks = rows * (Kp / 8);
+// A' (both parts when folded) and, folded, the row scales rs.
+fgq_status launch_fold_diag(const Geom& g, const uint32_t* codes, const float* alpha, float* rs, int mtiles,
+                            int64_t rows, void* a0, void* a1, cudaStream_t s) {
+  const bool fold = a1 != nullptr;
+  if (fold) {
+    row_scale_kernel<<<(unsigned)((g.M + 7) / 8), 256, 0, s>>>(alpha, g.M, g.ng, rs);
+    const fgq_status st = after_launch();
+    if (st != FGQ_OK) return st;
+  }
+  const int64_t nchunks = rows * (g.Kp / 8);
   if (nchunks <= 0) return FGQ_OK;
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (nchunks + 255) / 256;
-  const int blocks = (int)(want < 8LL * sms ? want : 8LL * sms);
-  diag_kernel<<<blocks, 256, 0, s>>>(static_cast<const uint2*>(src), Kp, Mg, mtiles, nchunks,
-                                     static_cast<uint4*>(dst));
+  const int blocks = (int)(want < 16LL * sms ? want : 16LL * sms);
+  if (fold)
+    fold_diag_kernel<true><<<blocks, 256, 0, s>>>(codes, g.wrow, alpha, g.ng, rs, g.Kp, g.Mg, mtiles, nchunks,
+                                                  static_cast<uint4*>(a0), static_cast<uint4*>(a1));
+  else
+    fold_diag_kernel<false><<<blocks, 256, 0, s>>>(codes, g.wrow, nullptr, g.ng, nullptr, g.Kp, g.Mg, mtiles, nchunks,
+                                                   static_cast<uint4*>(a0), nullptr);
   return after_launch();
 }
 
@@ -508,33 +568,23 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   a.timeout_ns = lim_us < 0 ? T4_TIMEOUT_NS : (uint64_t)lim_us * 1000u;
   const bool fold = sums == nullptr;
 
-  // temporaries from the stream-ordered pool: the dense ternary operand fp16 [M][Kp] per part
-  // (folded hi, lo; or the codes) and the row scales, its block-diagonal form A' per part, and
-  // the activations in fp16
+  // temporaries from the stream-ordered pool: the block-diagonal ternary operand A' per part
+  // (folded hi, lo; or the codes), the row scales, and the activations in fp16
   cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
   const int nparts = fold ? 2 : 1;
-  const size_t dense_bytes = (size_t)g.M * g.Kp * 2;
   const int64_t arows = (int64_t)g.groups * a.mtiles * T4_ROWS;
   const size_t diag_bytes = (size_t)arows * g.Kp * 2;
   const size_t x16_bytes = (size_t)tc::act16_elems(g) * 2;
   const size_t rs_bytes = fold ? ((size_t)g.M * 4 + 255) / 256 * 256 : 0;
-  const size_t total = nparts * (dense_bytes + diag_bytes) + rs_bytes + x16_bytes;
+  const size_t total = nparts * diag_bytes + rs_bytes + x16_bytes;
   void* tmp = nullptr;
   if (cudaMallocFromPoolAsync(&tmp, total, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
-  uint8_t* dense = static_cast<uint8_t*>(tmp);
-  uint8_t* diag = dense + nparts * dense_bytes;
+  uint8_t* diag = static_cast<uint8_t*>(tmp);
   float* rs = reinterpret_cast<float*>(diag + nparts * diag_bytes);
   uint8_t* x16 = diag + nparts * diag_bytes + rs_bytes;
-  fgq_status st;
-  if (fold) {
-    a.row_scale = rs;
-    st = launch_fold_alpha_split(codes, g.M, g.wrow, g.G, g.ng, alpha, dense, dense + dense_bytes, rs, s);
-  } else {
-    st = launch_expand_codes(codes, (int64_t)g.M * g.wrow, dense, s);
-  }
-  for (int part = 0; st == FGQ_OK && part < nparts; ++part)
-    st = launch_diag(dense + part * dense_bytes, g.Kp, g.Mg, a.mtiles, arows, diag + part * diag_bytes, s);
+  if (fold) a.row_scale = rs;
+  fgq_status st = launch_fold_diag(g, codes, alpha, rs, a.mtiles, arows, diag, fold ? diag + diag_bytes : nullptr, s);
   if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
   for (int part = 0; st == FGQ_OK && part < nparts; ++part)
     if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, diag + part * diag_bytes, (uint64_t)g.Kp,
