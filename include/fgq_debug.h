@@ -71,6 +71,14 @@ int64_t fgq_debug_set_wait_limit_us(int64_t us);
 int fgq_debug_allow_split_fold(int allow);
 
 /*
+ * Runs the G = 4 tensor-core output kernel of this thread's calls on CTA pairs (on != 0: two
+ * SMs share each 64-filter x 256-position tile through cta_group::2 MMAs) or on single CTAs
+ * (0, the default: 32-filter tiles), the same results either way.  Returns the previous
+ * setting.
+ */
+int fgq_debug_cta_pairs(int on);
+
+/*
  * The CUDA runtime error (a cudaError_t value) behind the last FGQ_ERR_CUDA that a kernel
  * launch of this thread returned, 0 if none; reading it clears it.  `name` receives the
  * runtime's name of that error (at most `len` bytes including the terminator) when non-null.

@@ -25,6 +25,7 @@ thread_local int t_last_path = FGQ_PATH_AUTO;
 thread_local int64_t t_wait_limit_us = -1;
 thread_local int t_split_fold = 0;
 thread_local int t_last_cuda_error = 0;  // cudaError_t of the last failed launch on this thread
+thread_local int t_cta_pairs = 0;        // G = 4 output kernel on CTA pairs (off: single CTAs)
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
@@ -188,6 +189,8 @@ fgq_status after_launch() {
 }
 
 int64_t debug_wait_limit_us() { return t_wait_limit_us; }
+
+bool debug_cta_pairs() { return t_cta_pairs != 0; }
 
 namespace {
 
@@ -673,6 +676,12 @@ int64_t fgq_debug_set_wait_limit_us(int64_t us) {
 int fgq_debug_allow_split_fold(int allow) {
   const int prev = t_split_fold;
   t_split_fold = allow ? 1 : 0;
+  return prev;
+}
+
+int fgq_debug_cta_pairs(int on) {
+  const int prev = t_cta_pairs;
+  t_cta_pairs = on ? 1 : 0;
   return prev;
 }
 

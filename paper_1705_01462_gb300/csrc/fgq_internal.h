@@ -36,6 +36,8 @@ fgq_status after_launch();
 // Wait limit, in microseconds, that a test set on this host thread for the tensor-core
 // kernels' mbarrier waits (fgq_debug_set_wait_limit_us), or -1 for the kernels' own limits.
 int64_t debug_wait_limit_us();
+// Whether the G = 4 output kernel runs on CTA pairs (this thread's setting, default off).
+bool debug_cta_pairs();
 
 // Kernel launchers (each returns FGQ_OK or FGQ_ERR_CUDA / FGQ_ERR_UNSUPPORTED).
 fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,

@@ -100,6 +100,7 @@ struct T4Args {
   unsigned int* err;
   Geom g;
   int mtiles, ptiles, ntiles, ktiles;  // mtiles: 32-filter tiles per conv group
+  int mtiles2;                         // CTA pairs: 64-filter tiles per conv group (ntiles counts pair tiles)
   int out_tma;
   uint64_t timeout_ns;
 };
@@ -210,6 +211,63 @@ __global__ void __launch_bounds__(256) fold_diag_kernel(const uint32_t* __restri
     }
     a0[i] = make_uint4(h0[0], h0[1], h0[2], h0[3]);
     if (FOLD) a1[i] = make_uint4(h1[0], h1[1], h1[2], h1[3]);
+  }
+}
+
+// Tile end of the output variant: the four slot rows 4 m' .. 4 m' + 3 of a filter are lanes
+// 4 (lane / 4) .. + 3 of the warp; reduce them so that lane j ends with positions 4 i + j
+// (i < 32) of its half, summed over the slots (two exchange rounds, each keeping half of the
+// positions), scale by s_x 2^-e_m and store: one 32-filter x 256-position TMA box through
+// shared memory (every epilogue thread of the CTA takes part), or direct / requantized stores.
+__device__ __forceinline__ void store_tile4(const T4Args& a, float (&acc)[T4_EPI_COLS], float* otile, int gi, int mt,
+                                            int64_t p0, int half, int mp, int j, bool mok, int m, float sx,
+                                            bool leader) {
+  const Geom& g = a.g;
+  const bool b1 = (j >> 1) & 1, b0 = j & 1;
+#pragma unroll
+  for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      // positions 4 q + e (slot bit 1 clear) and 4 q + 2 + e (set): keep the one whose bit 1
+      // matches b1, send the other to lane ^ 2; the result goes to 4 q + e
+      const float lo = acc[4 * q + e], hi = acc[4 * q + 2 + e];
+      const float sent = __shfl_xor_sync(0xffffffffu, b1 ? lo : hi, 2);
+      acc[4 * q + e] = (b1 ? hi : lo) + sent;
+    }
+    // positions 4 q + 2 b1 + 0 / + 1 (now at 4 q, 4 q + 1): keep bit 0 = b0
+    const float e0 = acc[4 * q], e1 = acc[4 * q + 1];
+    const float sent = __shfl_xor_sync(0xffffffffu, b0 ? e0 : e1, 1);
+    acc[4 * q] = (b0 ? e1 : e0) + sent;  // position 4 q + j, all four slots
+  }
+  const float sc_m = mok ? sx * __ldg(a.row_scale + m) : 0.0f;
+  const int64_t pbase = p0 + T4_EPI_COLS * half;
+  if (a.out_tma) {
+    if (leader) bulk_wait_read_all();  // the previous tile's box has been read out
+    named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
+    float* ob = otile + (T4_EPI_COLS * half + j) * T4_FM + mp;
+#pragma unroll
+    for (int q = 0; q < T4_EPI_COLS / 4; ++q) ob[4 * q * T4_FM] = sc_m * acc[4 * q];
+    fence_proxy_async_smem();
+    named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
+    if (leader) {  // rows past P and filters past M are clipped by the tensor map
+      tma_store_2d(&a.out_map, gi * g.Mg + mt * T4_FM, (int)p0, smem_u32(otile));
+      bulk_commit();
+    }
+  } else if (mok) {
+    if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
+      const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
+#pragma unroll
+      for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
+        const int64_t p = pbase + 4 * q + j;
+        if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sc_m * acc[4 * q], r);
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
+        const int64_t p = pbase + 4 * q + j;
+        if (p < g.P) a.out[p * g.M + m] = sc_m * acc[4 * q];
+      }
+    }
   }
 }
 
@@ -437,56 +495,8 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
       }
       if (!ok && !*abort_flag) fail();
       if (named_bar_or(BAR_EPI4, 32 * T4_EPI_WARPS, !ok)) break;
-      if constexpr (FOLD) {
-        // the four slot rows 4 m' .. 4 m' + 3 of a filter are lanes 4 (lane / 4) .. + 3 of the
-        // warp: reduce them so that lane j ends with positions 4 i + j (i < 32) of its half,
-        // summed over the slots; two exchange rounds, each keeping half of the positions
-        const bool b1 = (j >> 1) & 1, b0 = j & 1;
-#pragma unroll
-        for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
-#pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            // positions 4 q + e (slot bit 1 clear) and 4 q + 2 + e (set): keep the one whose
-            // bit 1 matches b1, send the other to lane ^ 2; the result goes to 4 q + e
-            const float lo = acc[4 * q + e], hi = acc[4 * q + 2 + e];
-            const float sent = __shfl_xor_sync(0xffffffffu, b1 ? lo : hi, 2);
-            acc[4 * q + e] = (b1 ? hi : lo) + sent;
-          }
-          // positions 4 q + 2 b1 + 0 / + 1 (now at 4 q, 4 q + 1): keep bit 0 = b0
-          const float e0 = acc[4 * q], e1 = acc[4 * q + 1];
-          const float sent = __shfl_xor_sync(0xffffffffu, b0 ? e0 : e1, 1);
-          acc[4 * q] = (b0 ? e1 : e0) + sent;  // position 4 q + j, all four slots
-        }
-        const float sc_m = mok ? sx * __ldg(a.row_scale + m) : 0.0f;
-        if (a.out_tma) {
-          if (leader) bulk_wait_read_all();  // the previous tile's box has been read out
-          named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
-          float* ob = otile + (T4_EPI_COLS * half + j) * T4_FM + mp;
-#pragma unroll
-          for (int q = 0; q < T4_EPI_COLS / 4; ++q) ob[4 * q * T4_FM] = sc_m * acc[4 * q];
-          fence_proxy_async_smem();
-          named_bar_sync(BAR_EPI4, 32 * T4_EPI_WARPS);
-          if (leader) {  // rows past P and filters past M are clipped by the tensor map
-            tma_store_2d(&a.out_map, gi * g.Mg + mt * T4_FM, (int)p0, smem_u32(otile));
-            bulk_commit();
-          }
-        } else if (mok) {
-          if (g.rq_out) {  // fused requantization: 8-bit codes instead of fp32
-            const RqMul r = rq_mul(g.rq_scale, g.rq_signed);
-#pragma unroll
-            for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
-              const int64_t p = pbase + 4 * q + j;
-              if (p < g.P) g.rq_out[p * g.M + m] = rq_code(sc_m * acc[4 * q], r);
-            }
-          } else {
-#pragma unroll
-            for (int q = 0; q < T4_EPI_COLS / 4; ++q) {
-              const int64_t p = pbase + 4 * q + j;
-              if (p < g.P) a.out[p * g.M + m] = sc_m * acc[4 * q];
-            }
-          }
-        }
-      }
+      if constexpr (FOLD)
+        store_tile4(a, acc, otile, gi, mt, p0, half, mp, j, mok, m, sx, leader);
     }
     if (leader) bulk_wait_all();
   }
@@ -497,6 +507,301 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
     tc_fence_after();
     tmem_dealloc(tmem, T4_TMEM_COLS);
   }
+}
+
+// CTA-pair variant of the output kernel.  Two CTAs (a cluster) share a 64-filter x
+// 256-position tile: CTA r holds the block-diagonal rows of filters 32 r .. of the pair's 64
+// and positions 128 r .. of the 256, and one thread of CTA 0 issues M = 256, N = 256 MMAs
+// (cta_group::2) that read both CTAs' operands and write each CTA's 128 TMEM lanes.  Per SM,
+// a K-tile moves 48 KB into shared memory instead of 64 KB and each MMA reads 8 KB of it
+// instead of 12 KB.  Synchronisation across the pair: CTA 1's loads complete on its own
+// barriers and a forwarding thread passes each completion to CTA 0 (pfull); the MMA commit
+// arrives on both CTAs' acc_full; CTA 1's epilogue warps free an accumulator with remote
+// arrivals on CTA 0's acc_empty.  Each CTA frees its own stages (the epilogue relay).
+constexpr int P4_NST = 4;
+constexpr int P4_STAGE = 2 * A_TILE4 + B_TILE4 / 2;  // A' hi, lo + this CTA's 128 positions
+constexpr int P4_BAR = 8 * (3 * P4_NST + 2 * T4_NACC + 1) + 16;
+constexpr int P4_SMEM = 1024 + P4_NST * P4_STAGE + OUT_BOX4 + P4_BAR;
+static_assert(P4_SMEM <= 232448, "shared memory budget");
+
+__device__ __forceinline__ void pair_tile_coords(const T4Args& a, int tile, uint32_t rank, int& gi, int& mt,
+                                                 int64_t& p0) {
+  const int per_p = a.g.groups * a.mtiles2;
+  const int pt = tile / per_p;
+  const int r = tile - pt * per_p;
+  gi = r / a.mtiles2;
+  mt = 2 * (r - gi * a.mtiles2) + (int)rank;
+  p0 = (int64_t)pt * T4_BN;
+}
+
+template <bool TMAP>
+__global__ void __launch_bounds__(T4_THREADS, 1) tc4_pair_kernel(const __grid_constant__ T4Args a) {
+  constexpr int NST = P4_NST;
+  extern __shared__ uint8_t smem_raw4p[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw4p) + 1023) & ~uintptr_t(1023));
+  float* otile = reinterpret_cast<float*>(smem + NST * P4_STAGE);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NST * P4_STAGE + OUT_BOX4);
+  uint64_t* full = bars;                // this CTA's stage loaded
+  uint64_t* empty = bars + NST;         // this CTA's stage free
+  uint64_t* pfull = bars + 2 * NST;     // CTA 0: CTA 1's stage loaded (forwarded)
+  uint64_t* acc_full = bars + 3 * NST;
+  uint64_t* acc_empty = acc_full + T4_NACC;  // CTA 0: both CTAs' epilogues drained
+  uint64_t* drain_bar = acc_empty + T4_NACC;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  volatile uint32_t* abort_flag = tmem_slot + 1;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const Geom& g = a.g;
+  const uint64_t tmo = a.timeout_ns;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = (int)blockIdx.x >> 1, npairs = (int)gridDim.x >> 1;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < NST; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+      mbar_init(&pfull[i], 1);
+    }
+    for (int i = 0; i < T4_NACC; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 2 * T4_EPI_WARPS);  // the epilogue warps of both CTAs
+    }
+    mbar_init(drain_bar, T4_NACC);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == T4_MMA_WARP) {
+    tmem_alloc_pair(tmem_slot, T4_TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers exist before any remote arrival
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int my_tiles = (a.ntiles - pair + npairs - 1) / npairs;
+  const int total = my_tiles * a.ktiles;
+
+  auto fail = [&]() {
+    *abort_flag = 1;
+    record_error(a.err, FGQ_ERR_TIMEOUT);
+  };
+
+  // ------------------------------------------------------------------ producer (each CTA)
+  if (warp == T4_PROD_WARP && lane == 0) {
+    int gi = 0, mt = 0, tr = 0, ts = 0, tc0 = 0, kt = 0, tl = 0;
+    int64_t p0 = 0;
+    int n0 = 0, h0 = 0, w0 = 0;
+    int issued = 0;
+    bool ok = true;
+    for (int j = 0; j < total; ++j) {
+      if (kt == 0) {
+        pair_tile_coords(a, pair + tl * npairs, rank, gi, mt, p0);
+        tr = ts = tc0 = 0;
+        if (!TMAP) {
+          const int pp = (int)p0 + (T4_BN / 2) * (int)rank;  // this CTA's first position
+          const int wo = pp % g.Wo;
+          const int q = pp / g.Wo;
+          n0 = q / g.Ho;
+          h0 = (q - n0 * g.Ho) * g.stride - g.pad;
+          w0 = wo * g.stride - g.pad;
+        }
+      }
+      const int s = j % NST;
+      if (j >= NST && !mbar_wait_timed(&empty[s], ((j / NST) & 1) ^ 1, tmo, abort_flag, 64)) {
+        ok = false;
+        break;
+      }
+      uint8_t* sa = smem + s * P4_STAGE;
+      const int arow = (gi * a.mtiles + mt) * T4_ROWS;  // past the group's filters: masked at the end
+      const int ch = gi * g.Cg + tc0;
+      mbar_arrive_expect_tx(&full[s], P4_STAGE);
+      tma_load_2d(smem_u32(sa), &a.a_map[0], kt * T4_KT, arow, &full[s]);
+      tma_load_2d(smem_u32(sa + A_TILE4), &a.a_map[1], kt * T4_KT, arow, &full[s]);
+      uint8_t* sb = sa + 2 * A_TILE4;
+      if (TMAP)
+        tma_load_2d(smem_u32(sb), &a.act_map, ch, (int)p0 + (T4_BN / 2) * (int)rank, &full[s]);
+      else
+        tma_load_im2col_4d(smem_u32(sb), &a.act_map, ch, w0, h0, n0, (uint16_t)ts, (uint16_t)tr, &full[s]);
+      issued = j + 1;
+      tc0 += T4_KT;
+      if (tc0 == g.Cg) {
+        tc0 = 0;
+        if (++ts == g.S) {
+          ts = 0;
+          ++tr;
+        }
+      }
+      if (++kt == a.ktiles) {
+        kt = 0;
+        ++tl;
+      }
+    }
+    if (!ok && !*abort_flag) fail();
+    for (int j = issued - NST < 0 ? 0 : issued - NST; j < issued; ++j)
+      mbar_wait_bounded(&full[j % NST], (j / NST) & 1, T4_DRAIN_LIMIT);
+  }
+
+  // ------------------------------------------------------------------ CTA 1: forwarder
+  if (rank == 1 && warp == T4_MMA_WARP && lane == 0) {
+    const uint32_t lead_pfull = mapa_shared(pfull, 0);
+    bool ok = true;
+    for (int j = 0; j < total; ++j) {
+      const int s = j % NST;
+      if (!mbar_wait_timed(&full[s], (j / NST) & 1, tmo, abort_flag, 0)) {
+        ok = false;
+        break;
+      }
+      mbar_arrive_cluster(lead_pfull + 8u * (uint32_t)s);
+    }
+    if (!ok && !*abort_flag) fail();
+  }
+
+  // ------------------------------------------------------------------ CTA 0: MMA issuers
+  if (rank == 0 && (warp == T4_MMA_WARP || warp == T4_MMA_WARP + 1) && lane == 0) {
+    const int b = warp - T4_MMA_WARP;
+    const uint32_t idesc = idesc_f16_f32(2 * T4_ROWS, T4_BN);
+    const uint32_t d = tmem + (uint32_t)(b * T4_BN);
+    bool ok = true;
+    for (int u = b; u < total && ok; u += 2) {
+      if (!mbar_wait_timed(&acc_empty[b], ((u >> 1) & 1) ^ 1, tmo, abort_flag, 0)) {
+        ok = false;
+        break;
+      }
+      const int s = u % NST;
+      if (!mbar_wait_timed(&full[s], (u / NST) & 1, tmo, abort_flag, 0) ||
+          !mbar_wait_timed(&pfull[s], (u / NST) & 1, tmo, abort_flag, 0)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t abase = smem_u32(smem + s * P4_STAGE);
+      const uint64_t bd = sdesc_k_sw128(abase + 2 * A_TILE4);
+#pragma unroll
+      for (int st = 0; st < 4; ++st)
+#pragma unroll
+        for (int part = 0; part < 2; ++part)
+          mma_f16_pair(d, sdesc_k_sw128(abase + part * A_TILE4) + 2 * st, bd + 2 * st, idesc, (st | part) != 0 ? 1u : 0u);
+      mma_commit_pair(&acc_full[b], 3);
+    }
+    if (!ok && !*abort_flag) fail();
+    mma_commit_pair(drain_bar, 1);
+    mbar_wait_bounded(drain_bar, 0, T4_DRAIN_LIMIT);
+  }
+
+  // ------------------------------------------------------------------ epilogue (each CTA)
+  if (warp < T4_EPI_WARPS) {
+    const int quarter = warp & 3, half = warp >> 2;
+    const int mp = 8 * quarter + (lane >> 2);
+    const int j = lane & 3;
+    const uint32_t tbase = tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(T4_EPI_COLS * half);
+    const uint32_t lead_acc_empty = mapa_shared(acc_empty, 0);
+    const float sx = __ldg(a.act_scale);
+    const bool leader = threadIdx.x == 0;
+    int u = 0;
+    bool ok = true;
+    for (int tl = 0; tl < my_tiles; ++tl) {
+      int gi, mt;
+      int64_t p0;
+      pair_tile_coords(a, pair + tl * npairs, rank, gi, mt, p0);
+      const int local = mt * T4_FM + mp;
+      const int m = gi * g.Mg + local;
+      const bool mok = local < g.Mg;
+      float acc[T4_EPI_COLS];
+#pragma unroll
+      for (int i = 0; i < T4_EPI_COLS; ++i) acc[i] = 0.0f;
+      for (int k = 0; k < a.ktiles; ++k, ++u) {
+        if (!ok) continue;
+        const int b = u & 1;
+        if (!mbar_wait_timed(&acc_full[b], (u >> 1) & 1, tmo, abort_flag, 0)) {
+          ok = false;
+          continue;
+        }
+        if (leader) mbar_arrive(&empty[u % NST]);  // the K-tile's MMAs are complete: free this CTA's stage
+        tc_fence_after();
+        const uint32_t ta = tbase + (uint32_t)(b * T4_BN);
+#pragma unroll
+        for (int c = 0; c < T4_EPI_COLS / 16; ++c) {
+          uint32_t r[16];
+          tmem_ld16(ta + 16 * c, r);
+          tmem_ld_wait_regs16(r);
+          if (c == T4_EPI_COLS / 16 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {  // the accumulator is free once both CTAs have it in registers
+              if (rank == 0) mbar_arrive(&acc_empty[b]);
+              else mbar_arrive_cluster(lead_acc_empty + 8u * (uint32_t)b);
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[16 * c + i] += __uint_as_float(r[i]);
+        }
+      }
+      if (!ok && !*abort_flag) fail();
+      if (named_bar_or(BAR_EPI4, 32 * T4_EPI_WARPS, !ok)) break;
+      store_tile4(a, acc, otile, gi, mt, p0, half, mp, j, mok, m, sx, leader);
+    }
+    if (leader) bulk_wait_all();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // no CTA leaves while the pair's MMAs or arrivals may still reach it
+  if (warp == T4_MMA_WARP) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, T4_TMEM_COLS);
+  }
+}
+
+// CTA pairs the device runs at once: not every SM can pair with a neighbour of its cluster
+// domain, so a persistent grid of SMs / 2 pairs would leave some pairs waiting for others to
+// finish all their tiles.  Queried once per device and kernel.
+template <bool TMAP>
+int resident_pairs() {
+  constexpr int kDev = 64;
+  static std::once_flag once[kDev];
+  static int n[kDev];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDev) return 0;
+  std::call_once(once[dev], [&] {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2);
+    cfg.blockDim = dim3(T4_THREADS);
+    cfg.dynamicSmemBytes = P4_SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int c = 0;
+    n[dev] = cudaOccupancyMaxActiveClusters(&c, tc4_pair_kernel<TMAP>, &cfg) == cudaSuccess ? c : 0;
+  });
+  return n[dev];
+}
+
+template <bool TMAP>
+fgq_status launch_tc4_pair(const T4Args& args, int ntiles, cudaStream_t s) {
+  if (!tc::smem_attr_once<tc4_pair_kernel<TMAP>>(P4_SMEM)) return FGQ_ERR_CUDA;
+  const int resident = resident_pairs<TMAP>();
+  if (resident <= 0) return FGQ_ERR_CUDA;
+  const int npairs = ntiles < resident ? ntiles : resident;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(2 * npairs));
+  cfg.blockDim = dim3(T4_THREADS);
+  cfg.dynamicSmemBytes = P4_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, tc4_pair_kernel<TMAP>, args) != cudaSuccess) return FGQ_ERR_CUDA;
+  return after_launch();
 }
 
 template <bool TMAP, bool FOLD>
@@ -561,12 +866,16 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   a.g = g;
   a.mtiles = (g.Mg + T4_FM - 1) / T4_FM;
   a.ptiles = (int)((g.P + T4_BN - 1) / T4_BN);
-  a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.ktiles = g.Kp / T4_KT;
+  const bool fold = sums == nullptr;
+  // fp32 outputs run on CTA pairs (64 filters x 256 positions per pair) unless a test asked
+  // for single CTAs; the group sums always on single CTAs
+  const bool pairs = fold && debug_cta_pairs();
+  a.mtiles2 = (a.mtiles + 1) / 2;
+  a.ntiles = g.groups * (pairs ? a.mtiles2 : a.mtiles) * a.ptiles;
   // a test may shorten the waits (debug_wait_limit_us), never the final drains
   const int64_t lim_us = debug_wait_limit_us();
   a.timeout_ns = lim_us < 0 ? T4_TIMEOUT_NS : (uint64_t)lim_us * 1000u;
-  const bool fold = sums == nullptr;
 
   // temporaries from the stream-ordered pool: the block-diagonal ternary operand A' per part
   // (folded hi, lo; or the codes), the row scales, and the activations in fp16
@@ -591,7 +900,7 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
                      (uint64_t)arows, (uint64_t)g.Kp * 2, T4_KT, T4_ROWS, CU_TENSOR_MAP_SWIZZLE_128B))
       st = FGQ_ERR_CUDA;
   const bool tmap = tc::act_pointwise(g);
-  if (st == FGQ_OK && !tc::act16_map(&a.act_map, x16, g, T4_BN)) st = FGQ_ERR_CUDA;
+  if (st == FGQ_OK && !tc::act16_map(&a.act_map, x16, g, pairs ? T4_BN / 2 : T4_BN)) st = FGQ_ERR_CUDA;
   if (st == FGQ_OK && fold && g.groups == 1 && g.M % 4 == 0 && !g.rq_out)
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, T4_FM, T4_BN, CU_TENSOR_MAP_SWIZZLE_NONE)
@@ -602,7 +911,9 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = a.ntiles < sms ? a.ntiles : sms;
-    if (fold)
+    if (pairs)
+      st = tmap ? launch_tc4_pair<true>(a, a.ntiles, s) : launch_tc4_pair<false>(a, a.ntiles, s);
+    else if (fold)
       st = tmap ? launch_tc4<true, true>(a, grid, s) : launch_tc4<false, true>(a, grid, s);
     else
       st = tmap ? launch_tc4<true, false>(a, grid, s) : launch_tc4<false, false>(a, grid, s);

@@ -65,6 +65,7 @@ SIGNATURES = [
     ("fgq_debug_set_wait_limit_us", _i64, [_i64]),
     ("fgq_debug_allow_split_fold", _i, [_i]),
     ("fgq_debug_last_cuda_error", _i, [_vp, _sz]),
+    ("fgq_debug_cta_pairs", _i, [_i]),
 ]
 
 
@@ -489,6 +490,11 @@ def fgq_debug_set_wait_limit_us(us: int) -> int:
 def fgq_debug_allow_split_fold(allow: bool) -> int:
     """Lets FGQ_PATH_DENSE run fp32 alphas as the split-fp16 ablation on this thread."""
     return int(lib().fgq_debug_allow_split_fold(1 if allow else 0))
+
+
+def fgq_debug_cta_pairs(on: bool) -> int:
+    """G = 4 output kernel on CTA pairs or single CTAs (the default) for this thread's calls."""
+    return int(lib().fgq_debug_cta_pairs(1 if on else 0))
 
 
 def fgq_debug_last_cuda_error() -> tuple:

@@ -338,21 +338,28 @@ def test_tc_forced_on_unsupported_shape():
     assert e.value.code == fgq.FGQ_ERR_UNSUPPORTED
 
 
-@pytest.mark.parametrize("path", ["simt", "tc"])
+@pytest.mark.parametrize("path", ["simt", "tc", "tc_cta_pairs"])
 @pytest.mark.parametrize("case", [(1, 56, 56, 64, 64, 3, 3, 1, 1, 1, 4, "u8"), (2, 28, 28, 128, 96, 1, 1, 1, 0, 1, 4, "u8"),
-                                  (2, 14, 14, 256, 64, 1, 1, 2, 0, 1, 4, "s8")],
+                                  (2, 14, 14, 256, 64, 1, 1, 2, 0, 1, 4, "s8"), (1, 9, 13, 128, 160, 3, 3, 1, 1, 2, 4, "u4"),
+                                  (3, 7, 7, 64, 96, 3, 3, 2, 1, 1, 4, "s8")],
                          ids=lambda c: "x".join(map(str, c)))
 def test_g4_both_kernel_families(case, path):
-    """G = 4 through the dp4a kernel and through the block-diagonal tensor-core kernel."""
+    """G = 4 through the dp4a kernel and through the block-diagonal tensor-core kernel, the
+    latter on single CTAs (the default) and on CTA pairs."""
     B, H, W, C, M, R, S, stride, pad, groups, G, act = case
     rng = np.random.default_rng(zlib.crc32(repr(case).encode()) + 2)
-    w = (rng.standard_normal((M, R * S * C)) * np.sqrt(2.0 / (R * S * C))).astype(np.float32)
+    Kred = R * S * (C // groups)
+    w = (rng.standard_normal((M, Kred)) * np.sqrt(2.0 / Kred)).astype(np.float32)
     t, al, codes = make_codes(w, G)
     x = random_acts((B, H, W, C), act, rng)
     q, sc, packed = quantize_oracle(x, act)
     y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
     fgq.fgq_set_path(fgq.PATH_SIMT if path == "simt" else fgq.PATH_TC)
-    gout = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride,
-                          pad, groups, to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    prev = fgq.fgq_debug_cta_pairs(path == "tc_cta_pairs")
+    try:
+        gout = fgq.fgq_conv2d(to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride,
+                              pad, groups, to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    finally:
+        fgq.fgq_debug_cta_pairs(bool(prev))
     assert fgq.fgq_last_path() == (fgq.PATH_SIMT if path == "simt" else fgq.PATH_TC)
     check_within(gout.cpu().numpy(), y, ym, f"G=4 {path} {case}")
