@@ -60,7 +60,6 @@ using tc::u8pair_to_h2;
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 256;        // positions per tile (MMA N)
 constexpr int TC_KT = 64;         // reduction elements per K-tile
-constexpr int TC_NST = 3;         // operand ring depth (stages of A + B)
 constexpr int TC_NACC = 2;        // TMEM accumulator buffers
 constexpr int TC_EPI_WARPS = 8;
 constexpr int TC_MMA_WARP = TC_EPI_WARPS;       // warps 8 and 9: MMA issuers of even and odd groups
@@ -73,21 +72,34 @@ constexpr uint32_t TC_WAIT_SLEEP_NS = 20000;     // suspend hint of one poll
 constexpr uint32_t TC_DRAIN_LIMIT = 1u << 20;    // polls of the final drains (never shortened)
 constexpr uint32_t BAR_EPI = 2;                  // named barrier of the 256 epilogue threads
 
-constexpr int A_TILE = TC_BM * TC_KT * 2;        // 16 KB fp16 ternary operand
-constexpr int B_TILE = TC_BN * TC_KT * 2;        // 32 KB fp16 activation operand
-constexpr int STAGE = A_TILE + B_TILE;
 constexpr int OUT_POS = 64;                      // positions per output box
 constexpr int OUT_BOX = OUT_POS * TC_BM * 4;     // 32 KB fp32 [64 positions][128 filters]
 constexpr int SMEM_OUT = 2 * OUT_BOX;            // one box per position half of the tile
-constexpr int SMEM_BAR = 8 * (2 * TC_NST + 2 * TC_NACC + 1) + 16;
-constexpr int TC_SMEM = 1024 + TC_NST * STAGE + SMEM_OUT + SMEM_BAR;
-static_assert(TC_SMEM <= 232448, "shared memory budget");
-static_assert(A_TILE % 1024 == 0 && STAGE % 1024 == 0, "128-byte-swizzle atoms stay 1024-byte aligned");
+
+// Operand plan of a variant.  fp16 operands (8-bit activations): 128-byte rows of 64
+// elements, 128-byte swizzle, 4 MMAs of K = 16 per K-tile.  e4m3 operands (4-bit
+// activations, F8): every 4-bit value and every code is exact in e4m3, so the K-tile is
+// 64-byte rows with the 64-byte swizzle and 2 MMAs of K = 32 (kind::f8f6f4) -- half the bytes
+// per K-tile in HBM, L2 and shared memory, twice the ring depth.
+template <bool F8>
+struct TcCfg {
+  static constexpr int ES = F8 ? 1 : 2;                 // bytes per operand element
+  static constexpr int A_TILE = TC_BM * TC_KT * ES;     // ternary operand
+  static constexpr int B_TILE = TC_BN * TC_KT * ES;     // activation operand
+  static constexpr int STAGE = A_TILE + B_TILE;
+  static constexpr int NST = F8 ? 6 : 3;                // operand ring depth
+  static constexpr int SMEM_BAR = 8 * (2 * NST + 2 * TC_NACC + 1) + 16;
+  static constexpr int SMEM = 1024 + NST * STAGE + SMEM_OUT + SMEM_BAR;
+};
+static_assert(TcCfg<false>::SMEM <= 232448 && TcCfg<true>::SMEM <= 232448, "shared memory budget");
+static_assert(TcCfg<false>::A_TILE % 1024 == 0 && TcCfg<false>::STAGE % 1024 == 0 &&
+                  TcCfg<true>::A_TILE % 1024 == 0 && TcCfg<true>::STAGE % 1024 == 0,
+              "swizzle atoms stay 1024-byte aligned");
 
 struct TcArgs {
-  CUtensorMap a16_map;    // fp16 [M][Kp] expanded codes, box {64, 128 rows}, 128-byte swizzle
-  CUtensorMap act_map;    // fp16 activations: act_tma: 2D [positions][C], box {64, 256 rows}; otherwise
-                          // the im2col map of the NHWC tensor, 256 pixels x 64 channels; 128-byte swizzle
+  CUtensorMap a16_map;    // expanded codes [M][Kp] (fp16, or e4m3 for F8), box {64, 128 rows}
+  CUtensorMap act_map;    // expanded activations: act_tma: 2D [positions][C], box {64, 256 rows}; otherwise
+                          // the im2col map of the NHWC tensor, 256 pixels x 64 channels
   CUtensorMap out_map;    // fp32 [P][M], box {128 filters, 64 positions}; if out_tma
   const float* alpha;
   const float* act_scale;
@@ -203,11 +215,94 @@ __global__ void __launch_bounds__(256) expand_act_strided_kernel(const uint8_t* 
   }
 }
 
+// 16 packed 4-bit activation codes (8 bytes, element 2i in the low nibble of byte i) -> 16
+// e4m3 bytes in element order.  Every 4-bit value is exact in e4m3: 0 -> 0x00, 1 -> 0x38 (1.0),
+// n = 2^e (1 + f/8) -> (e + 7) << 3 | f; negative s4 values carry the sign bit.  The 16-entry
+// table is looked up with byte permutes (low and high half of the table, chosen per byte by
+// the value's bit 3).
+template <bool SIGNED>
+__device__ __forceinline__ uint4 expand16_e4m3(uint32_t x0, uint32_t x1) {
+  constexpr uint32_t T0 = 0x44403800u, T1 = 0x4E4C4A48u;  // 0 .. 7
+  constexpr uint32_t T2 = SIGNED ? 0xCACCCED0u : 0x53525150u;  // 8 .. 11 (s4: -8 .. -5)
+  constexpr uint32_t T3 = SIGNED ? 0xB8C0C4C8u : 0x57565554u;  // 12 .. 15 (s4: -4 .. -1)
+  const uint32_t xs[2] = {x0, x1};
+  uint32_t o[4];
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const uint32_t x = xs[q];
+    const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
+    const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
+    const uint32_t bw[2] = {(lo & 0xffffu) | ((hi & 0xffffu) << 16), (lo >> 16) | (hi & 0xffff0000u)};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const uint32_t b = bw[h];  // four values 0 .. 15, one per byte
+      const uint32_t sel = (b & 7u) | ((b >> 4) & 0x70u) | ((b >> 8) & 0x700u) | ((b >> 12) & 0x7000u);
+      const uint32_t vlo = __byte_perm(T0, T1, sel), vhi = __byte_perm(T2, T3, sel);
+      const uint32_t mask = ((b >> 3) & 0x01010101u) * 0xffu;
+      o[2 * q + h] = (vhi & mask) | (vlo & ~mask);
+    }
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+template <bool SIGNED>
+__global__ void __launch_bounds__(256) expand_act_e4m3_kernel(const uint8_t* __restrict__ act, int64_t nchunks,
+                                                              uint4* __restrict__ out) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + i);
+    out[i] = expand16_e4m3<SIGNED>(v.x, v.y);
+  }
+}
+
+// The pixels a strided 1x1 unpadded convolution reads, gathered: [P][C] e4m3.
+template <bool SIGNED>
+__global__ void __launch_bounds__(256) expand_act_e4m3_strided_kernel(const uint8_t* __restrict__ act, int H, int W,
+                                                                      int C, int Ho, int Wo, int stride,
+                                                                      int64_t nchunks, uint4* __restrict__ out) {
+  const int cpp = C / 16;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t p = i / cpp;
+    const int c = (int)(i - p * cpp);
+    const int wo = (int)(p % Wo);
+    const int64_t q = p / Wo;
+    const int ho = (int)(q % Ho);
+    const int64_t b = q / Ho;
+    const int64_t src = ((b * H + (int64_t)ho * stride) * W + (int64_t)wo * stride) * cpp + c;
+    const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + src);
+    out[i] = expand16_e4m3<SIGNED>(v.x, v.y);
+  }
+}
+
+// 2-bit codes -> e4m3 {0, +1, -1}: 00 -> 0x00, 01 -> 0x38, 11 -> 0xB8; one word (16 codes) per
+// thread, 16 bytes out.
+__global__ void __launch_bounds__(256) expand_codes_e4m3_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
+                                                                uint4* __restrict__ out) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= nwords) return;
+  const uint32_t w = __ldg(codes + i);
+  uint32_t o[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    uint32_t v = 0;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t c = (w >> (2 * (4 * q + e))) & 3u;
+      v |= (((c & 1u) ? 0x38u : 0u) | ((c & 2u) << 6)) << (8 * e);
+    }
+    o[q] = v;
+  }
+  out[i] = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
 // TMAP: the layer's im2col rows are contiguous input rows (2D box loads); otherwise the
 // activation boxes come from an im2col map (one load per K-tile: 256 output positions at
 // one filter tap and 64 channels, padding read as zeros).
-template <bool TMAP, bool SUMS>
+template <bool TMAP, bool SUMS, bool F8>
 __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid_constant__ TcArgs a) {
+  using Cfg = TcCfg<F8>;
+  constexpr int TC_NST = Cfg::NST;
+  constexpr int STAGE = Cfg::STAGE;
+  constexpr int A_TILE = Cfg::A_TILE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float* otile = reinterpret_cast<float*>(smem + TC_NST * STAGE);  // two [64 positions][128 filters] boxes
@@ -340,12 +435,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
             break;
           }
           tc_fence_after();
-          const uint64_t ad = sdesc_k_sw128(smem_u32(smem + s * STAGE));
-          const uint64_t bd = sdesc_k_sw128(smem_u32(smem + s * STAGE + A_TILE));
+          if constexpr (F8) {
+            const uint64_t ad = sdesc_k_sw64(smem_u32(smem + s * STAGE));
+            const uint64_t bd = sdesc_k_sw64(smem_u32(smem + s * STAGE + A_TILE));
 #pragma unroll
-          for (int k = 0; k < TC_KT / 16; ++k) {
-            // advance 16 fp16 (32 bytes) along K inside the swizzled rows
-            mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (sub > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < TC_KT / 32; ++k)  // advance 32 e4m3 (32 bytes) along K
+              mma_e4m3(d, ad + 2 * k, bd + 2 * k, idesc, (sub > 0 || k > 0) ? 1u : 0u);
+          } else {
+            const uint64_t ad = sdesc_k_sw128(smem_u32(smem + s * STAGE));
+            const uint64_t bd = sdesc_k_sw128(smem_u32(smem + s * STAGE + A_TILE));
+#pragma unroll
+            for (int k = 0; k < TC_KT / 16; ++k)  // advance 16 fp16 (32 bytes) along K
+              mma_f16(d, ad + 2 * k, bd + 2 * k, idesc, (sub > 0 || k > 0) ? 1u : 0u);
           }
         }
         if (ok) mma_commit(&acc_full[b]);
@@ -485,11 +586,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
   }
 }
 
-template <bool TMAP, bool SUMS>
+template <bool TMAP, bool SUMS, bool F8>
 fgq_status launch_tc(const TcArgs& args, int grid, cudaStream_t s) {
-  if (!tc::smem_attr_once<tc_contract_kernel<TMAP, SUMS>>(TC_SMEM)) return FGQ_ERR_CUDA;
-  tc_contract_kernel<TMAP, SUMS><<<grid, TC_THREADS, TC_SMEM, s>>>(args);
+  constexpr int smem = TcCfg<F8>::SMEM;
+  if (!tc::smem_attr_once<tc_contract_kernel<TMAP, SUMS, F8>>(smem)) return FGQ_ERR_CUDA;
+  tc_contract_kernel<TMAP, SUMS, F8><<<grid, TC_THREADS, smem, s>>>(args);
   return after_launch();
+}
+
+template <bool F8>
+fgq_status launch_tc_variant(const TcArgs& a, bool sums, int grid, cudaStream_t s) {
+  if (sums) return a.act_tma ? launch_tc<true, true, F8>(a, grid, s) : launch_tc<false, true, F8>(a, grid, s);
+  return a.act_tma ? launch_tc<true, false, F8>(a, grid, s) : launch_tc<false, false, F8>(a, grid, s);
 }
 
 template <int ABITS, bool SIGNED>
@@ -525,6 +633,31 @@ template <int ABITS, bool SIGNED>
 fgq_status expand_activations(const void* act, const Geom& g, void* act16, cudaStream_t s) {
   if (g.R == 1 && g.S == 1 && g.pad == 0 && g.stride > 1) return launch_expand_act_strided<ABITS, SIGNED>(act, g, act16, s);
   return launch_expand_act<ABITS, SIGNED>(act, (int64_t)g.B * g.H * g.W * g.C, act16, s);
+}
+
+int expand_blocks(int64_t nchunks) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (nchunks + 255) / 256;
+  return (int)(want < 8LL * sms ? want : 8LL * sms);
+}
+
+// 4-bit activations as e4m3 bytes: NHWC, or [P][C] for a strided 1x1 unpadded convolution.
+template <bool SIGNED>
+fgq_status expand_activations_e4m3(const void* act, const Geom& g, void* x8, cudaStream_t s) {
+  const uint8_t* a8 = static_cast<const uint8_t*>(act);
+  if (g.R == 1 && g.S == 1 && g.pad == 0 && g.stride > 1) {
+    const int64_t nchunks = g.P * (g.C / 16);
+    if (nchunks <= 0) return FGQ_OK;
+    expand_act_e4m3_strided_kernel<SIGNED><<<expand_blocks(nchunks), 256, 0, s>>>(a8, g.H, g.W, g.C, g.Ho, g.Wo, g.stride,
+                                                                                   nchunks, static_cast<uint4*>(x8));
+  } else {
+    const int64_t nchunks = (int64_t)g.B * g.H * g.W * g.C / 16;
+    if (nchunks <= 0) return FGQ_OK;
+    expand_act_e4m3_kernel<SIGNED><<<expand_blocks(nchunks), 256, 0, s>>>(a8, nchunks, static_cast<uint4*>(x8));
+  }
+  return after_launch();
 }
 
 // One block waits on an mbarrier that nothing arrives on; every wait is bounded, so the
@@ -605,26 +738,52 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   const int64_t lim_us = debug_wait_limit_us();
   a.wait_limit = lim_us < 0 ? TC_WAIT_LIMIT : (uint32_t)(lim_us / 20 + 1);
   a.wait_sleep_ns = lim_us < 0 ? TC_WAIT_SLEEP_NS : (uint32_t)(lim_us < 20 ? lim_us * 1000 : 20000);
-  // temporaries from the stream-ordered pool: the codes as fp16 [M][Kp] (Kp = 16 wrow) and
-  // the activations as fp16 NHWC (a strided 1x1 convolution: only the pixels it reads, [P][C])
+  // 4-bit activations run on e4m3 operands (exact), 8-bit ones on fp16 (exact)
+  const bool f8 = g.act_type == FGQ_U4 || g.act_type == FGQ_S4;
+  const int es = f8 ? 1 : 2;
+  // temporaries from the stream-ordered pool: the codes expanded [M][Kp] (Kp = 16 wrow) and the
+  // activations expanded NHWC (a strided 1x1 convolution: only the pixels it reads, [P][C])
   cudaMemPool_t pool = scratch_pool();
   if (!pool) return FGQ_ERR_CUDA;
   const int64_t nwords = (int64_t)g.M * g.wrow;
   const int64_t nact = tc::act16_elems(g);
   void* a16 = nullptr;
   void* x16 = nullptr;
-  if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 32, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
-  if (cudaMallocFromPoolAsync(&x16, (size_t)nact * 2, pool, s) != cudaSuccess) {
+  if (cudaMallocFromPoolAsync(&a16, (size_t)nwords * 16 * es, pool, s) != cudaSuccess) return FGQ_ERR_CUDA;
+  if (cudaMallocFromPoolAsync(&x16, (size_t)nact * es, pool, s) != cudaSuccess) {
     cudaFreeAsync(a16, s);
     return FGQ_ERR_CUDA;
   }
-  fgq_status st = launch_expand_codes(codes, nwords, a16, s);
-  if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
-  if (st == FGQ_OK && !make_map_2d(&a.a16_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a16, (uint64_t)g.wrow * 16,
-                                   (uint64_t)g.M, (uint64_t)g.wrow * 32, TC_KT, TC_BM, CU_TENSOR_MAP_SWIZZLE_128B))
+  fgq_status st = FGQ_OK;
+  if (f8) {
+    if (nwords > 0) {
+      expand_codes_e4m3_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
+      st = after_launch();
+    }
+    if (st == FGQ_OK)
+      st = g.act_type == FGQ_S4 ? expand_activations_e4m3<true>(act, g, x16, s)
+                                : expand_activations_e4m3<false>(act, g, x16, s);
+  } else {
+    st = launch_expand_codes(codes, nwords, a16, s);
+    if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
+  }
+  const CUtensorMapDataType dt = f8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+  const CUtensorMapSwizzle sw = f8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
+  if (st == FGQ_OK && !make_map_2d(&a.a16_map, dt, a16, (uint64_t)g.wrow * 16, (uint64_t)g.M,
+                                   (uint64_t)g.wrow * 16 * es, TC_KT, TC_BM, sw))
     st = FGQ_ERR_CUDA;
   a.act_tma = act_pointwise(g) ? 1 : 0;
-  if (st == FGQ_OK && !tc::act16_map(&a.act_map, x16, g, TC_BN)) st = FGQ_ERR_CUDA;
+  bool act_ok = true;
+  if (st == FGQ_OK) {
+    if (!f8)
+      act_ok = tc::act16_map(&a.act_map, x16, g, TC_BN);
+    else if (a.act_tma)
+      act_ok = make_map_2d(&a.act_map, dt, x16, (uint64_t)g.C, (uint64_t)(nact / g.C), (uint64_t)g.C, TC_KT, TC_BN, sw);
+    else
+      act_ok = make_map_im2col(&a.act_map, dt, x16, (uint64_t)g.C, 1, g.B, g.H, g.W, g.R, g.S, g.stride, g.pad, TC_KT,
+                               TC_BN, sw);
+  }
+  if (!act_ok) st = FGQ_ERR_CUDA;
   if (st == FGQ_OK && g.groups == 1 && g.M % 4 == 0 && !g.rq_out && !sums)
     a.out_tma = make_map_2d(&a.out_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, out, (uint64_t)g.M, (uint64_t)g.P,
                             (uint64_t)g.M * 4, TC_BM, OUT_POS, CU_TENSOR_MAP_SWIZZLE_NONE)
@@ -634,12 +793,8 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = a.ntiles < sms ? a.ntiles : sms;
-  if (st == FGQ_OK) {
-    if (sums)
-      st = a.act_tma ? launch_tc<true, true>(a, grid, s) : launch_tc<false, true>(a, grid, s);
-    else
-      st = a.act_tma ? launch_tc<true, false>(a, grid, s) : launch_tc<false, false>(a, grid, s);
-  }
+  if (st == FGQ_OK)
+    st = f8 ? launch_tc_variant<true>(a, sums != nullptr, grid, s) : launch_tc_variant<false>(a, sums != nullptr, grid, s);
   // the temporaries return to the pool once the work queued on s before this point is done
   if (cudaFreeAsync(x16, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;
   if (cudaFreeAsync(a16, s) != cudaSuccess && st == FGQ_OK) st = FGQ_ERR_CUDA;

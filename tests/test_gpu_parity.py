@@ -173,6 +173,8 @@ CONV_CASES = [
     (2, 12, 12, 128, 64, 3, 3, 2, 1, 1, 128, "u4"),
     (1, 8, 8, 256, 128, 3, 3, 1, 1, 2, 64, "u8"),
     (1, 15, 15, 64, 64, 5, 5, 3, 2, 1, 64, "s4"),
+    (2, 14, 14, 128, 64, 1, 1, 2, 0, 1, 64, "s4"),    # strided 1x1, 4-bit: gathered e4m3 rows
+    (2, 9, 9, 192, 96, 1, 1, 1, 0, 1, 64, "u4"),      # 1x1 stride 1, 4-bit: 2D e4m3 boxes
 ]
 
 
