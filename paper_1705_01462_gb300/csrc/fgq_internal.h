@@ -74,9 +74,6 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                               const float* alpha, const float* act_scale, float* out,
                               int32_t* sums, unsigned int* err, cudaStream_t s);
 
-// The 2-bit codes of nwords code words expanded to fp16 {0, +1, -1}: 16 halves (32 bytes) per
-// word at a16 (the ternary operand the tensor-core kernels load by TMA).
-fgq_status launch_expand_codes(const uint32_t* codes, int64_t nwords, void* a16, cudaStream_t s);
 
 // Tensor-core contraction for G = 4 (block-diagonal activation operand).
 bool tc4_supports(const Geom& g);

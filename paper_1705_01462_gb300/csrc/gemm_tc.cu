@@ -14,12 +14,13 @@
 // drains.  The group-sums variant (SUMS) stores each drained accumulator as the int32
 // s[m][g][p] instead (the exact integers themselves, for verification).
 //
-// Both operands reach shared memory by TMA, already in fp16: the codes are expanded to
-// {0, +1, -1} and the activations to their integer values once per call (stream-ordered
-// temporaries, one elementwise pass each), so every K-tile is two box loads into one ring
-// stage and no thread converts operands inside the contraction.  An activation is read by
-// R * S filter taps and M / 128 filter tiles; converting it once instead of at every use
-// takes the conversion off the MMA's path.
+// Both operands reach shared memory by TMA, already as MMA operands: the codes are expanded
+// to {0, +1, -1} and the activations to their integer values once per call (stream-ordered
+// temporaries written by one launch, prep64_kernel), fp16 for 8-bit activations and e4m3
+// (kind::f8f6f4) for 4-bit ones, so every K-tile is two box loads into one ring stage and
+// no thread converts operands inside the contraction.  An activation is read by R * S filter
+// taps and M / 128 filter tiles; converting it once instead of at every use takes the
+// conversion off the MMA's path.
 //
 // Warp roles (352 threads, one CTA per SM, persistent over tiles):
 //   warps 0-7  epilogue: warp w reads TMEM lanes 32*(w%4).. (filter rows) and columns
@@ -45,6 +46,7 @@
 #include <cstdint>
 #include <cstring>
 
+#include "operand_prep.cuh"
 #include "tc_common.cuh"
 
 namespace fgq {
@@ -55,7 +57,6 @@ using tc::encode_tiled;
 using tc::im2col_fits;
 using tc::make_map_2d;
 using tc::make_map_im2col;
-using tc::u8pair_to_h2;
 
 constexpr int TC_BM = 128;        // filters per tile (MMA M, TMEM lanes)
 constexpr int TC_BN = 256;        // positions per tile (MMA N)
@@ -130,168 +131,26 @@ __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, 
   p0 = (int64_t)pt * TC_BN;
 }
 
-// Activation codes -> fp16 integers, 16 elements per thread and step (NHWC order kept):
-// 8-bit: 16 bytes in, 32 out; 4-bit: 8 bytes (16 nibbles, element 2i in the low nibble of
-// byte i) in, 32 out.  Signed codes are offset to unsigned and the offset subtracted in
-// fp16 (1024 + v - bias, exact).
-template <int ABITS, bool SIGNED>
-__device__ __forceinline__ void expand16(uint32_t (&w)[4], uint4& o0, uint4& o1) {
-  if (ABITS == 8) {
-    if (SIGNED) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) w[q] ^= 0x80808080u;
+// One launch prepares both operands of a call: blocks [0, code_blocks) expand the ternary
+// codes (one 16-code word per thread and step), the others the activations (16 elements per
+// thread and step); fp16 operands, or e4m3 for 4-bit activations (F8).
+template <bool F8>
+__global__ void __launch_bounds__(256) prep64_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
+                                                     uint4* __restrict__ a_op, const prep::ActSrc src,
+                                                     uint4* __restrict__ x_op, int code_blocks) {
+  if ((int)blockIdx.x < code_blocks) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nwords; i += (int64_t)code_blocks * blockDim.x) {
+      if (F8) prep::codes_e4m3(codes, i, a_op);
+      else prep::codes_f16(codes, i, a_op);
     }
   } else {
-    const uint32_t x2[2] = {w[0], w[1]};
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      // 8 nibbles -> 8 bytes (element order preserved)
-      const uint32_t x = x2[q];
-      const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
-      const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
-      w[2 * q] = (lo & 0xffffu) | ((hi & 0xffffu) << 16);                               // e0 e1 e2 e3
-      w[2 * q + 1] = (lo >> 16) | (hi & 0xffff0000u);                                   // e4 e5 e6 e7
-      if (SIGNED) {
-        w[2 * q] ^= 0x08080808u;
-        w[2 * q + 1] ^= 0x08080808u;
-      }
+    const int64_t nb = (int64_t)gridDim.x - code_blocks;
+    for (int64_t i = ((int64_t)blockIdx.x - code_blocks) * blockDim.x + threadIdx.x; i < src.nchunks;
+         i += nb * blockDim.x) {
+      if (F8) prep::act_e4m3(src, i, x_op);
+      else prep::act_f16(src, i, x_op);
     }
   }
-  constexpr uint32_t bias2 =
-      ABITS == 8 ? (SIGNED ? 0x64806480u : 0x64006400u) : (SIGNED ? 0x64086408u : 0x64006400u);
-  o0.x = u8pair_to_h2(w[0], 0x4140, bias2); o0.y = u8pair_to_h2(w[0], 0x4342, bias2);
-  o0.z = u8pair_to_h2(w[1], 0x4140, bias2); o0.w = u8pair_to_h2(w[1], 0x4342, bias2);
-  o1.x = u8pair_to_h2(w[2], 0x4140, bias2); o1.y = u8pair_to_h2(w[2], 0x4342, bias2);
-  o1.z = u8pair_to_h2(w[3], 0x4140, bias2); o1.w = u8pair_to_h2(w[3], 0x4342, bias2);
-}
-
-template <int ABITS, bool SIGNED>
-__global__ void __launch_bounds__(256) expand_act_kernel(const uint8_t* __restrict__ act, int64_t nchunks,
-                                                         uint4* __restrict__ out) {
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
-    uint32_t w[4];
-    if (ABITS == 8) {
-      const uint4 v = __ldg(reinterpret_cast<const uint4*>(act) + i);
-      w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
-    } else {
-      const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + i);
-      w[0] = v.x; w[1] = v.y;
-    }
-    uint4 o0, o1;
-    expand16<ABITS, SIGNED>(w, o0, o1);
-    out[2 * i] = o0;
-    out[2 * i + 1] = o1;
-  }
-}
-
-// A 1x1 unpadded convolution with stride > 1 reads one input pixel per output position:
-// the expansion gathers those pixels into a dense fp16 [P][C] tensor (16 channels per
-// thread and step), so that the contraction loads its rows with 2D boxes.
-template <int ABITS, bool SIGNED>
-__global__ void __launch_bounds__(256) expand_act_strided_kernel(const uint8_t* __restrict__ act, int H, int W,
-                                                                 int C, int Ho, int Wo, int stride,
-                                                                 int64_t nchunks, uint4* __restrict__ out) {
-  const int cpp = C / 16;  // 16-channel chunks per pixel
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t p = i / cpp;
-    const int c = (int)(i - p * cpp);
-    const int wo = (int)(p % Wo);
-    const int64_t q = p / Wo;
-    const int ho = (int)(q % Ho);
-    const int64_t b = q / Ho;
-    const int64_t src = ((b * H + (int64_t)ho * stride) * W + (int64_t)wo * stride) * cpp + c;  // 16-channel chunk
-    uint32_t w[4];
-    if (ABITS == 8) {
-      const uint4 v = __ldg(reinterpret_cast<const uint4*>(act) + src);
-      w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
-    } else {
-      const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + src);
-      w[0] = v.x; w[1] = v.y;
-    }
-    uint4 o0, o1;
-    expand16<ABITS, SIGNED>(w, o0, o1);
-    out[2 * i] = o0;
-    out[2 * i + 1] = o1;
-  }
-}
-
-// 16 packed 4-bit activation codes (8 bytes, element 2i in the low nibble of byte i) -> 16
-// e4m3 bytes in element order.  Every 4-bit value is exact in e4m3: 0 -> 0x00, 1 -> 0x38 (1.0),
-// n = 2^e (1 + f/8) -> (e + 7) << 3 | f; negative s4 values carry the sign bit.  The 16-entry
-// table is looked up with byte permutes (low and high half of the table, chosen per byte by
-// the value's bit 3).
-template <bool SIGNED>
-__device__ __forceinline__ uint4 expand16_e4m3(uint32_t x0, uint32_t x1) {
-  constexpr uint32_t T0 = 0x44403800u, T1 = 0x4E4C4A48u;  // 0 .. 7
-  constexpr uint32_t T2 = SIGNED ? 0xCACCCED0u : 0x53525150u;  // 8 .. 11 (s4: -8 .. -5)
-  constexpr uint32_t T3 = SIGNED ? 0xB8C0C4C8u : 0x57565554u;  // 12 .. 15 (s4: -4 .. -1)
-  const uint32_t xs[2] = {x0, x1};
-  uint32_t o[4];
-#pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    const uint32_t x = xs[q];
-    const uint32_t lo = (x & 0x000f000fu) | ((x & 0x00f000f0u) << 4);                // e0 e1 e4 e5
-    const uint32_t hi = ((x >> 8) & 0x000f000fu) | (((x >> 8) & 0x00f000f0u) << 4);  // e2 e3 e6 e7
-    const uint32_t bw[2] = {(lo & 0xffffu) | ((hi & 0xffffu) << 16), (lo >> 16) | (hi & 0xffff0000u)};
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const uint32_t b = bw[h];  // four values 0 .. 15, one per byte
-      const uint32_t sel = (b & 7u) | ((b >> 4) & 0x70u) | ((b >> 8) & 0x700u) | ((b >> 12) & 0x7000u);
-      const uint32_t vlo = __byte_perm(T0, T1, sel), vhi = __byte_perm(T2, T3, sel);
-      const uint32_t mask = ((b >> 3) & 0x01010101u) * 0xffu;
-      o[2 * q + h] = (vhi & mask) | (vlo & ~mask);
-    }
-  }
-  return make_uint4(o[0], o[1], o[2], o[3]);
-}
-
-template <bool SIGNED>
-__global__ void __launch_bounds__(256) expand_act_e4m3_kernel(const uint8_t* __restrict__ act, int64_t nchunks,
-                                                              uint4* __restrict__ out) {
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
-    const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + i);
-    out[i] = expand16_e4m3<SIGNED>(v.x, v.y);
-  }
-}
-
-// The pixels a strided 1x1 unpadded convolution reads, gathered: [P][C] e4m3.
-template <bool SIGNED>
-__global__ void __launch_bounds__(256) expand_act_e4m3_strided_kernel(const uint8_t* __restrict__ act, int H, int W,
-                                                                      int C, int Ho, int Wo, int stride,
-                                                                      int64_t nchunks, uint4* __restrict__ out) {
-  const int cpp = C / 16;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t p = i / cpp;
-    const int c = (int)(i - p * cpp);
-    const int wo = (int)(p % Wo);
-    const int64_t q = p / Wo;
-    const int ho = (int)(q % Ho);
-    const int64_t b = q / Ho;
-    const int64_t src = ((b * H + (int64_t)ho * stride) * W + (int64_t)wo * stride) * cpp + c;
-    const uint2 v = __ldg(reinterpret_cast<const uint2*>(act) + src);
-    out[i] = expand16_e4m3<SIGNED>(v.x, v.y);
-  }
-}
-
-// 2-bit codes -> e4m3 {0, +1, -1}: 00 -> 0x00, 01 -> 0x38, 11 -> 0xB8; one word (16 codes) per
-// thread, 16 bytes out.
-__global__ void __launch_bounds__(256) expand_codes_e4m3_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
-                                                                uint4* __restrict__ out) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= nwords) return;
-  const uint32_t w = __ldg(codes + i);
-  uint32_t o[4];
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    uint32_t v = 0;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const uint32_t c = (w >> (2 * (4 * q + e))) & 3u;
-      v |= (((c & 1u) ? 0x38u : 0u) | ((c & 2u) << 6)) << (8 * e);
-    }
-    o[q] = v;
-  }
-  out[i] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // TMAP: the layer's im2col rows are contiguous input rows (2D box loads); otherwise the
@@ -600,66 +459,6 @@ fgq_status launch_tc_variant(const TcArgs& a, bool sums, int grid, cudaStream_t 
   return a.act_tma ? launch_tc<true, false, F8>(a, grid, s) : launch_tc<false, false, F8>(a, grid, s);
 }
 
-template <int ABITS, bool SIGNED>
-fgq_status launch_expand_act(const void* act, int64_t nelem, void* act16, cudaStream_t s) {
-  const int64_t nchunks = nelem / 16;  // nelem is a multiple of 16 (C % 16 == 0)
-  if (nchunks <= 0) return FGQ_OK;
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t want = (nchunks + 255) / 256;
-  const int blocks = (int)(want < 8LL * sms ? want : 8LL * sms);
-  expand_act_kernel<ABITS, SIGNED>
-      <<<blocks, 256, 0, s>>>(static_cast<const uint8_t*>(act), nchunks, static_cast<uint4*>(act16));
-  return after_launch();
-}
-
-// The pixels a strided 1x1 unpadded convolution reads, gathered and expanded: [P][C] fp16.
-template <int ABITS, bool SIGNED>
-fgq_status launch_expand_act_strided(const void* act, const Geom& g, void* act16, cudaStream_t s) {
-  const int64_t nchunks = g.P * (g.C / 16);
-  if (nchunks <= 0) return FGQ_OK;
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t want = (nchunks + 255) / 256;
-  const int blocks = (int)(want < 8LL * sms ? want : 8LL * sms);
-  expand_act_strided_kernel<ABITS, SIGNED><<<blocks, 256, 0, s>>>(
-      static_cast<const uint8_t*>(act), g.H, g.W, g.C, g.Ho, g.Wo, g.stride, nchunks, static_cast<uint4*>(act16));
-  return after_launch();
-}
-
-template <int ABITS, bool SIGNED>
-fgq_status expand_activations(const void* act, const Geom& g, void* act16, cudaStream_t s) {
-  if (g.R == 1 && g.S == 1 && g.pad == 0 && g.stride > 1) return launch_expand_act_strided<ABITS, SIGNED>(act, g, act16, s);
-  return launch_expand_act<ABITS, SIGNED>(act, (int64_t)g.B * g.H * g.W * g.C, act16, s);
-}
-
-int expand_blocks(int64_t nchunks) {
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t want = (nchunks + 255) / 256;
-  return (int)(want < 8LL * sms ? want : 8LL * sms);
-}
-
-// 4-bit activations as e4m3 bytes: NHWC, or [P][C] for a strided 1x1 unpadded convolution.
-template <bool SIGNED>
-fgq_status expand_activations_e4m3(const void* act, const Geom& g, void* x8, cudaStream_t s) {
-  const uint8_t* a8 = static_cast<const uint8_t*>(act);
-  if (g.R == 1 && g.S == 1 && g.pad == 0 && g.stride > 1) {
-    const int64_t nchunks = g.P * (g.C / 16);
-    if (nchunks <= 0) return FGQ_OK;
-    expand_act_e4m3_strided_kernel<SIGNED><<<expand_blocks(nchunks), 256, 0, s>>>(a8, g.H, g.W, g.C, g.Ho, g.Wo, g.stride,
-                                                                                   nchunks, static_cast<uint4*>(x8));
-  } else {
-    const int64_t nchunks = (int64_t)g.B * g.H * g.W * g.C / 16;
-    if (nchunks <= 0) return FGQ_OK;
-    expand_act_e4m3_kernel<SIGNED><<<expand_blocks(nchunks), 256, 0, s>>>(a8, nchunks, static_cast<uint4*>(x8));
-  }
-  return after_launch();
-}
-
 // One block waits on an mbarrier that nothing arrives on; every wait is bounded, so the
 // kernel always returns and records FGQ_ERR_TIMEOUT.
 __global__ void wait_timeout_selftest_kernel(uint32_t max_iter, unsigned int* err) {
@@ -681,14 +480,6 @@ bool act_pointwise(const Geom& g) { return g.R == 1 && g.S == 1 && g.pad == 0; }
 
 int64_t act16_elems(const Geom& g) {
   return act_pointwise(g) && g.stride > 1 ? g.P * g.C : (int64_t)g.B * g.H * g.W * g.C;
-}
-
-fgq_status expand_act16(const void* act, const Geom& g, void* x16, cudaStream_t s) {
-  const int abits = (g.act_type == FGQ_U4 || g.act_type == FGQ_S4) ? 4 : 8;
-  const bool sgn = g.act_type == FGQ_S8 || g.act_type == FGQ_S4;
-  if (abits == 4)
-    return sgn ? expand_activations<4, true>(act, g, x16, s) : expand_activations<4, false>(act, g, x16, s);
-  return sgn ? expand_activations<8, true>(act, g, x16, s) : expand_activations<8, false>(act, g, x16, s);
 }
 
 bool act16_map(CUtensorMap* m, const void* x16, const Geom& g, uint32_t pixels) {
@@ -754,19 +545,14 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
     cudaFreeAsync(a16, s);
     return FGQ_ERR_CUDA;
   }
-  fgq_status st = FGQ_OK;
-  if (f8) {
-    if (nwords > 0) {
-      expand_codes_e4m3_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
-      st = after_launch();
-    }
-    if (st == FGQ_OK)
-      st = g.act_type == FGQ_S4 ? expand_activations_e4m3<true>(act, g, x16, s)
-                                : expand_activations_e4m3<false>(act, g, x16, s);
-  } else {
-    st = launch_expand_codes(codes, nwords, a16, s);
-    if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
-  }
+  // both operands in one launch, the blocks split by the two jobs' sizes
+  const prep::ActSrc src = prep::act_src(act, g);
+  const int cb = prep::blocks_for(nwords), xb = prep::blocks_for(src.nchunks);
+  if (f8)
+    prep64_kernel<true><<<cb + xb, 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16), src, static_cast<uint4*>(x16), cb);
+  else
+    prep64_kernel<false><<<cb + xb, 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16), src, static_cast<uint4*>(x16), cb);
+  fgq_status st = after_launch();
   const CUtensorMapDataType dt = f8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
   const CUtensorMapSwizzle sw = f8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
   if (st == FGQ_OK && !make_map_2d(&a.a16_map, dt, a16, (uint64_t)g.wrow * 16, (uint64_t)g.M,

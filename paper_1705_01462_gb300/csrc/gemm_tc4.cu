@@ -7,8 +7,9 @@
 // in the 4 columns of group slot j (zeros elsewhere), and D[4 m' + j][p] of one MMA
 // (M = 128, N = 256, K = 16) receives the products of group 4 step + j alone.  A' depends
 // only on the weights, so it is built once per call; the activations are the plain dense
-// operand, expanded to fp16 once per call and loaded by TMA (2D rows or im2col boxes), and
-// no thread builds operands inside the contraction.  Two variants:
+// operand, expanded to fp16 once per call (one launch, prep4_kernel, prepares both) and
+// loaded by TMA (2D rows or im2col boxes), and no thread builds operands inside the
+// contraction.  Two variants:
 //
 //   output (FOLD): the group's scale multiplies inside the MMA (one multiply per group,
 //     Section 4.1): A' carries the fp32 alpha folded into the codes as two fp16 parts,
@@ -49,6 +50,7 @@
 #include <cstdint>
 #include <cstring>
 
+#include "operand_prep.cuh"
 #include "tc_common.cuh"
 
 namespace fgq {
@@ -116,62 +118,64 @@ __device__ __forceinline__ void tile_coords4(const T4Args& a, int tile, int& gi,
   p0 = (int64_t)pt * T4_BN;
 }
 
-// Expands 2-bit codes (00 = 0, 01 = +1, 11 = -1; element k in word k / 16, bits 2 (k % 16))
-// to fp16 {0, +1, -1}: one thread per code word, 16 halves (32 bytes) out.
-__global__ void __launch_bounds__(256) expand_codes_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
-                                                           uint4* __restrict__ a16) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= nwords) return;
-  const uint32_t w = __ldg(codes + i);
-  uint32_t h[8];
-#pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    const uint32_t c0 = (w >> (4 * e)) & 3u, c1 = (w >> (4 * e + 2)) & 3u;
-    const uint32_t lo = (c0 & 1u) ? ((c0 & 2u) ? 0xBC00u : 0x3C00u) : 0u;
-    const uint32_t hi = (c1 & 1u) ? ((c1 & 2u) ? 0xBC00u : 0x3C00u) : 0u;
-    h[e] = lo | (hi << 16);
-  }
-  a16[2 * i] = make_uint4(h[0], h[1], h[2], h[3]);
-  a16[2 * i + 1] = make_uint4(h[4], h[5], h[6], h[7]);
-}
+// One launch prepares both operands of a call.  Blocks [0, fold_blocks) build the
+// block-diagonal ternary operand A' straight from the 2-bit codes, one block per 32-filter
+// tile and slice of the reduction axis: row 4 m' + j of tile (gi, mt) holds, for filter
+// gi Mg + mt 32 + m', the elements of the groups whose index is j modulo 4 (slot j of every
+// K = 16 step) and zeros elsewhere.  FOLD: the elements are alpha(m, g) 2^e_m t split into
+// fp16 hi + lo (hi the fp16 nearest, lo the fp16 nearest the remainder), parts a0 and a1,
+// where e_m puts the row's largest alpha in [2^14, 2^15) (clamped to [-100, 100]; an all-zero
+// row keeps e = 0) so that the low part stays clear of fp16's subnormal range -- each block
+// first finds e_m for its 32 filters (rs[m] = 2^-e_m written by the first slice); otherwise
+// the codes as fp16 {0, +1, -1} in a0.  One thread per 16-byte chunk of A' (8 elements = 2
+// groups, at most one of them in the row's slot).  The other blocks expand the activations
+// to fp16.
+constexpr int PREP4_CHUNKS = 8;  // 16-byte chunks of a row per fold block (64 elements)
 
-// Row scales of the folded operand, one warp per filter row: e_m puts the row's largest
-// alpha in [2^14, 2^15) (clamped to [-100, 100]; an all-zero row keeps e = 0), so that the
-// low fp16 part of every alpha stays clear of fp16's subnormal range; rs[m] = 2^-e_m.
-__global__ void __launch_bounds__(256) row_scale_kernel(const float* __restrict__ alpha, int M, int ng,
-                                                        float* __restrict__ rs) {
-  const int m = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (m >= M) return;
-  float mx = 0.0f;
-  for (int g = lane; g < ng; g += 32) mx = fmaxf(mx, __ldg(alpha + (int64_t)m * ng + g));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  int e = mx > 0.0f ? 14 - ilogbf(mx) : 0;
-  e = e < -100 ? -100 : (e > 100 ? 100 : e);
-  if (lane == 0) rs[m] = ldexpf(1.0f, -e);
-}
-
-// The block-diagonal ternary operand A', straight from the 2-bit codes: row 4 m' + j of tile
-// (gi, mt) holds, for filter gi Mg + mt 32 + m', the elements of the groups whose index is j
-// modulo 4 (slot j of every K = 16 step) and zeros elsewhere.  FOLD: the elements are
-// alpha(m, g) 2^e_m t split into fp16 hi + lo (hi the fp16 nearest, lo the fp16 nearest the
-// remainder), parts a0 and a1; otherwise the codes as fp16 {0, +1, -1} in a0.  One thread
-// per 16-byte chunk (8 elements = 2 groups, at most one of them in the row's slot).
 template <bool FOLD>
-__global__ void __launch_bounds__(256) fold_diag_kernel(const uint32_t* __restrict__ codes, int wrow,
-                                                        const float* __restrict__ alpha, int ng,
-                                                        const float* __restrict__ rs, int Kp, int Mg, int mtiles,
-                                                        int64_t nchunks, uint4* __restrict__ a0,
-                                                        uint4* __restrict__ a1) {
+__global__ void __launch_bounds__(256) prep4_kernel(const uint32_t* __restrict__ codes, int wrow,
+                                                    const float* __restrict__ alpha, int ng, float* __restrict__ rs,
+                                                    int Kp, int Mg, int mtiles, int ksplit, uint4* __restrict__ a0,
+                                                    uint4* __restrict__ a1, int fold_blocks, const prep::ActSrc src,
+                                                    uint4* __restrict__ x16) {
+  if ((int)blockIdx.x >= fold_blocks) {
+    const int64_t nb = (int64_t)gridDim.x - fold_blocks;
+    for (int64_t i = ((int64_t)blockIdx.x - fold_blocks) * blockDim.x + threadIdx.x; i < src.nchunks;
+         i += nb * blockDim.x)
+      prep::act_f16(src, i, x16);
+    return;
+  }
+  const int tile = (int)blockIdx.x / ksplit, ks = (int)blockIdx.x - tile * ksplit;
+  const int gi = tile / mtiles, mt = tile - gi * mtiles;
+  __shared__ float mul[T4_FM];  // 2^e_m of the tile's filters
+  if (FOLD) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+    for (int f = 0; f < T4_FM / 8; ++f) {
+      const int mp = (T4_FM / 8) * warp + f;
+      const int local = mt * T4_FM + mp;
+      float mx = 0.0f;
+      if (local < Mg) {
+        const float* ar = alpha + ((int64_t)gi * Mg + local) * ng;
+        for (int g = lane; g < ng; g += 32) mx = fmaxf(mx, __ldg(ar + g));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      int e = mx > 0.0f ? 14 - ilogbf(mx) : 0;
+      e = e < -100 ? -100 : (e > 100 ? 100 : e);
+      if (lane == 0) {
+        mul[mp] = ldexpf(1.0f, e);
+        if (ks == 0 && local < Mg) rs[(int64_t)gi * Mg + local] = ldexpf(1.0f, -e);
+      }
+    }
+    __syncthreads();
+  }
   const int cpr = Kp / 8;  // chunks per row
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nchunks; i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t r = i / cpr;
-    const int c = (int)(i - r * cpr);
-    const int64_t tile = r / T4_ROWS;
-    const int rr = (int)(r - tile * T4_ROWS);
+  const int c0 = ks * PREP4_CHUNKS;
+  const int nc = (cpr - c0) < PREP4_CHUNKS ? (cpr - c0) : PREP4_CHUNKS;
+  for (int it = threadIdx.x; it < T4_ROWS * nc; it += blockDim.x) {
+    const int rr = it / nc, c = c0 + (it - rr * nc);
     const int mp = rr >> 2, j = rr & 3;
-    const int gi = (int)(tile / mtiles), mt = (int)(tile - (int64_t)gi * mtiles);
     const int local = mt * T4_FM + mp;
     uint32_t h0[4] = {0u, 0u, 0u, 0u}, h1[4] = {0u, 0u, 0u, 0u};
     // group 2c occupies halves 0-3 of the chunk, group 2c + 1 halves 4-7; slot = group % 4
@@ -182,7 +186,7 @@ __global__ void __launch_bounds__(256) fold_diag_kernel(const uint32_t* __restri
       const uint32_t cw = (__ldg(codes + m * wrow + k0 / 16) >> (2 * (k0 % 16))) & 0xffu;
       uint32_t hi = 0x3C00u, lo = 0u;  // fp16 +1 and 0: the codes themselves
       if (FOLD) {
-        const float v = __ldg(alpha + m * ng + grp) / __ldg(rs + m);  // exact: a power-of-two scaling
+        const float v = __ldg(alpha + m * ng + grp) * mul[mp];  // exact: a power-of-two scaling
         const __half hh = __float2half_rn(v);
         hi = __half_as_ushort(hh);
         lo = __half_as_ushort(__float2half_rn(v - __half2float(hh)));  // the remainder, exact in fp32
@@ -209,6 +213,7 @@ __global__ void __launch_bounds__(256) fold_diag_kernel(const uint32_t* __restri
       h1[2] = first ? 0u : q0;
       h1[3] = first ? 0u : q1;
     }
+    const int64_t i = ((int64_t)tile * T4_ROWS + rr) * cpr + c;
     a0[i] = make_uint4(h0[0], h0[1], h0[2], h0[3]);
     if (FOLD) a1[i] = make_uint4(h1[0], h1[1], h1[2], h1[3]);
   }
@@ -812,38 +817,26 @@ fgq_status launch_tc4(const T4Args& args, int grid, cudaStream_t s) {
   return after_launch();
 }
 
-// A' (both parts when folded) and, folded, the row scales rs.
-fgq_status launch_fold_diag(const Geom& g, const uint32_t* codes, const float* alpha, float* rs, int mtiles,
-                            int64_t rows, void* a0, void* a1, cudaStream_t s) {
-  const bool fold = a1 != nullptr;
-  if (fold) {
-    row_scale_kernel<<<(unsigned)((g.M + 7) / 8), 256, 0, s>>>(alpha, g.M, g.ng, rs);
-    const fgq_status st = after_launch();
-    if (st != FGQ_OK) return st;
-  }
-  const int64_t nchunks = rows * (g.Kp / 8);
-  if (nchunks <= 0) return FGQ_OK;
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t want = (nchunks + 255) / 256;
-  const int blocks = (int)(want < 16LL * sms ? want : 16LL * sms);
-  if (fold)
-    fold_diag_kernel<true><<<blocks, 256, 0, s>>>(codes, g.wrow, alpha, g.ng, rs, g.Kp, g.Mg, mtiles, nchunks,
-                                                  static_cast<uint4*>(a0), static_cast<uint4*>(a1));
+// Both operands of a call in one launch: A' (both parts when folded) with the row scales rs,
+// and the activations in fp16.
+fgq_status launch_prep4(const Geom& g, const uint32_t* codes, const float* alpha, float* rs, int mtiles, void* a0,
+                        void* a1, const void* act, void* x16, cudaStream_t s) {
+  const int ksplit = (g.Kp / 8 + PREP4_CHUNKS - 1) / PREP4_CHUNKS;
+  const int fold_blocks = g.groups * mtiles * ksplit;
+  const prep::ActSrc src = prep::act_src(act, g);
+  const int xb = prep::blocks_for(src.nchunks);
+  if (a1)
+    prep4_kernel<true><<<fold_blocks + xb, 256, 0, s>>>(codes, g.wrow, alpha, g.ng, rs, g.Kp, g.Mg, mtiles, ksplit,
+                                                        static_cast<uint4*>(a0), static_cast<uint4*>(a1), fold_blocks,
+                                                        src, static_cast<uint4*>(x16));
   else
-    fold_diag_kernel<false><<<blocks, 256, 0, s>>>(codes, g.wrow, nullptr, g.ng, nullptr, g.Kp, g.Mg, mtiles, nchunks,
-                                                   static_cast<uint4*>(a0), nullptr);
+    prep4_kernel<false><<<fold_blocks + xb, 256, 0, s>>>(codes, g.wrow, nullptr, g.ng, nullptr, g.Kp, g.Mg, mtiles,
+                                                         ksplit, static_cast<uint4*>(a0), nullptr, fold_blocks, src,
+                                                         static_cast<uint4*>(x16));
   return after_launch();
 }
 
 }  // namespace
-
-fgq_status launch_expand_codes(const uint32_t* codes, int64_t nwords, void* a16, cudaStream_t s) {
-  if (nwords <= 0) return FGQ_OK;
-  expand_codes_kernel<<<(unsigned)((nwords + 255) / 256), 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16));
-  return after_launch();
-}
 
 bool tc4_supports(const Geom& g) {
   if (g.G != 4) return false;
@@ -893,8 +886,8 @@ fgq_status launch_tc4_contract(const void* act, const Geom& g, const uint32_t* c
   float* rs = reinterpret_cast<float*>(diag + nparts * diag_bytes);
   uint8_t* x16 = diag + nparts * diag_bytes + rs_bytes;
   if (fold) a.row_scale = rs;
-  fgq_status st = launch_fold_diag(g, codes, alpha, rs, a.mtiles, arows, diag, fold ? diag + diag_bytes : nullptr, s);
-  if (st == FGQ_OK) st = tc::expand_act16(act, g, x16, s);
+  fgq_status st =
+      launch_prep4(g, codes, alpha, rs, a.mtiles, diag, fold ? diag + diag_bytes : nullptr, act, x16, s);
   for (int part = 0; st == FGQ_OK && part < nparts; ++part)
     if (!make_map_2d(&a.a_map[part], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, diag + part * diag_bytes, (uint64_t)g.Kp,
                      (uint64_t)arows, (uint64_t)g.Kp * 2, T4_KT, T4_ROWS, CU_TENSOR_MAP_SWIZZLE_128B))

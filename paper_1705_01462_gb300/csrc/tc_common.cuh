@@ -167,7 +167,6 @@ inline bool make_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base
 // kernel): NHWC, or [P][C] -- only the pixels a strided 1x1 unpadded convolution reads.
 bool act_pointwise(const Geom& g);         // 1x1, unpadded (any stride), or a GEMM: 2D rows
 int64_t act16_elems(const Geom& g);        // elements of the fp16 copy
-fgq_status expand_act16(const void* act, const Geom& g, void* x16, cudaStream_t s);
 // 2D map (pointwise) or im2col map of the fp16 copy: boxes of `pixels` output positions x 64
 // channels, 128-byte swizzle
 bool act16_map(CUtensorMap* m, const void* x16, const Geom& g, uint32_t pixels);
