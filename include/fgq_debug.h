@@ -79,6 +79,19 @@ int fgq_debug_allow_split_fold(int allow);
 int fgq_debug_cta_pairs(int on);
 
 /*
+ * At most k (1 .. 8, clamped) group ranges per output tile in this thread's G >= 64
+ * tensor-core calls; returns the previous limit (default 8).  A layer with fewer output tiles
+ * than SMs splits each tile's groups into ranges and adds the ranges' partial sums into the
+ * output: the same sum in another fp32 rounding order, and with more than two ranges not
+ * bit-reproducible from run to run.  k = 1 keeps whole tiles (one rounding order, the one
+ * the fused requantizing entries use).
+ */
+int fgq_debug_max_ksplit(int k);
+
+/* Group ranges per tile of this thread's last G >= 64 tensor-core call (1: whole tiles). */
+int fgq_debug_last_ksplit(void);
+
+/*
  * The CUDA runtime error (a cudaError_t value) behind the last FGQ_ERR_CUDA that a kernel
  * launch of this thread returned, 0 if none; reading it clears it.  `name` receives the
  * runtime's name of that error (at most `len` bytes including the terminator) when non-null.

@@ -26,6 +26,8 @@ thread_local int64_t t_wait_limit_us = -1;
 thread_local int t_split_fold = 0;
 thread_local int t_last_cuda_error = 0;  // cudaError_t of the last failed launch on this thread
 thread_local int t_cta_pairs = 0;        // G = 4 output kernel on CTA pairs (off: single CTAs)
+thread_local int t_max_ksplit = 8;       // group ranges a G >= 64 tile may be split into
+thread_local int t_last_ksplit = 0;      // ranges of this thread's last G >= 64 tensor-core call
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
@@ -191,6 +193,10 @@ fgq_status after_launch() {
 int64_t debug_wait_limit_us() { return t_wait_limit_us; }
 
 bool debug_cta_pairs() { return t_cta_pairs != 0; }
+
+int debug_max_ksplit() { return t_max_ksplit; }
+
+void note_ksplit(int k) { t_last_ksplit = k; }
 
 namespace {
 
@@ -684,6 +690,14 @@ int fgq_debug_cta_pairs(int on) {
   t_cta_pairs = on ? 1 : 0;
   return prev;
 }
+
+int fgq_debug_max_ksplit(int k) {
+  const int prev = t_max_ksplit;
+  t_max_ksplit = k < 1 ? 1 : (k > 8 ? 8 : k);
+  return prev;
+}
+
+int fgq_debug_last_ksplit(void) { return t_last_ksplit; }
 
 int fgq_debug_last_cuda_error(char* name, size_t len) {
   const int e = t_last_cuda_error;

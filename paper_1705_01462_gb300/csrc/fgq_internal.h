@@ -38,6 +38,8 @@ fgq_status after_launch();
 int64_t debug_wait_limit_us();
 // Whether the G = 4 output kernel runs on CTA pairs (this thread's setting, default off).
 bool debug_cta_pairs();
+int debug_max_ksplit();    // 1 .. 8
+void note_ksplit(int k);   // group ranges of the G >= 64 tensor-core call just launched
 
 // Kernel launchers (each returns FGQ_OK or FGQ_ERR_CUDA / FGQ_ERR_UNSUPPORTED).
 fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* codes, float* alpha,

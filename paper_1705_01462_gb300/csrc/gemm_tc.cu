@@ -110,8 +110,10 @@ struct TcArgs {
   Geom g;
   int mtiles;       // filter tiles per conv group
   int ptiles;       // position tiles
-  int ntiles;       // groups * mtiles * ptiles
-  int ktiles;       // K-tiles per tile (= ng * G / 64)
+  int ntiles;       // work items: groups * mtiles * ptiles tiles, each split into ksplit group ranges
+  int ktiles;       // K-tiles of a whole tile (= ng * G / 64)
+  int ksplit;       // group ranges per tile (1: whole tiles; > 1: partial sums added into the output)
+  int gpk;          // groups per range
   int kt_per_group; // G / 64
   int act_tma;      // 2D activation map (one row per output position); else im2col map
   int out_tma;      // output boxes by TMA store (one conv group, M % 4 == 0, fp32 output)
@@ -119,9 +121,12 @@ struct TcArgs {
   uint32_t wait_sleep_ns;
 };
 
-// Tiles are numbered with the filter tiles of one position tile consecutive, so that
-// CTAs running at the same time share activation boxes in L2.
-__device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, int& m0, int64_t& p0) {
+// Work item w: tile w / ksplit, groups [g0, g1) of range w % ksplit.  Tiles are numbered
+// with the filter tiles of one position tile consecutive, so that CTAs running at the same
+// time share activation boxes in L2.
+__device__ __forceinline__ void item_coords(const TcArgs& a, int w, int& gi, int& m0, int64_t& p0, int& g0, int& g1) {
+  const int tile = w / a.ksplit;
+  const int ks = w - tile * a.ksplit;
   const int per_p = a.g.groups * a.mtiles;
   const int pt = tile / per_p;
   const int r = tile - pt * per_p;
@@ -129,6 +134,8 @@ __device__ __forceinline__ void tile_coords(const TcArgs& a, int tile, int& gi, 
   const int mt = r - gi * a.mtiles;
   m0 = gi * a.g.Mg + mt * TC_BM;
   p0 = (int64_t)pt * TC_BN;
+  g0 = ks * a.gpk;
+  g1 = g0 + a.gpk < a.g.ng ? g0 + a.gpk : a.g.ng;
 }
 
 // One launch prepares both operands of a call: blocks [0, code_blocks) expand the ternary
@@ -208,54 +215,52 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
 
   // ------------------------------------------------------------------ producer
   if (warp == TC_PROD_WARP && lane == 0) {
-    const int total = my_tiles * a.ktiles;
-    // per tile: conv group, first filter and position; the filter tap (tr, ts) and channel
-    // offset tc0 of the next K-tile advance incrementally
-    int gi = 0, m0 = 0, tr = 0, ts = 0, tc0 = 0, kt = 0, tl = 0;
-    int64_t p0 = 0;
-    int n0 = 0, h0 = 0, w0 = 0;  // im2col: the tile's first window origin (input pixel coordinates)
-    int issued = 0;
+    const int kpt = g.Cg / TC_KT;  // K-tiles per filter tap
+    int issued = 0;                // K-tiles issued by this CTA (the ring's sequence number)
     bool ok = true;
-    for (int j = 0; j < total; ++j) {
-      if (kt == 0) {
-        tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
-        tr = ts = tc0 = 0;
-        if (!TMAP) {
-          const int pp = (int)p0;  // < P < 2^31
-          const int wo = pp % g.Wo;
-          const int q = pp / g.Wo;
-          n0 = q / g.Ho;
-          h0 = (q - n0 * g.Ho) * g.stride - g.pad;
-          w0 = wo * g.stride - g.pad;
+    for (int tl = 0; tl < my_tiles && ok; ++tl) {
+      int gi, m0, g0, g1;
+      int64_t p0;
+      item_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0, g0, g1);
+      int n0 = 0, h0 = 0, w0 = 0;  // im2col: the tile's first window origin (input pixel coordinates)
+      if (!TMAP) {
+        const int pp = (int)p0;  // < P < 2^31
+        const int wo = pp % g.Wo;
+        const int q = pp / g.Wo;
+        n0 = q / g.Ho;
+        h0 = (q - n0 * g.Ho) * g.stride - g.pad;
+        w0 = wo * g.stride - g.pad;
+      }
+      // the range's first K-tile and its filter tap (tr, ts) and channel offset tc0, which
+      // then advance incrementally
+      const int kt0 = g0 * a.kt_per_group, kt1 = g1 * a.kt_per_group;
+      int tc0 = (kt0 % kpt) * TC_KT, ts = (kt0 / kpt) % g.S, tr = (kt0 / kpt) / g.S;
+      for (int kt = kt0; kt < kt1; ++kt) {
+        const int j = issued;
+        const int s = j % TC_NST;
+        // the stage's previous contents (K-tile j - TC_NST) have been consumed by the MMAs
+        if (j >= TC_NST &&
+            !mbar_wait_or_abort(&empty[s], ((j / TC_NST) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
+          ok = false;
+          break;
         }
-      }
-      const int s = j % TC_NST;
-      // the stage's previous contents (K-tile j - TC_NST) have been consumed by the MMAs
-      if (j >= TC_NST &&
-          !mbar_wait_or_abort(&empty[s], ((j / TC_NST) & 1) ^ 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
-        ok = false;
-        break;
-      }
-      uint8_t* sa = smem + s * STAGE;
-      const int ch = gi * g.Cg + tc0;  // first channel: a multiple of 64 (128-byte aligned in fp16)
-      mbar_arrive_expect_tx(&full[s], STAGE);
-      tma_load_2d(smem_u32(sa), &a.a16_map, kt * TC_KT, m0, &full[s]);
-      if (TMAP)
-        tma_load_2d(smem_u32(sa + A_TILE), &a.act_map, ch, (int)p0, &full[s]);
-      else
-        tma_load_im2col_4d(smem_u32(sa + A_TILE), &a.act_map, ch, w0, h0, n0, (uint16_t)ts, (uint16_t)tr, &full[s]);
-      issued = j + 1;
-      tc0 += TC_KT;
-      if (tc0 == g.Cg) {
-        tc0 = 0;
-        if (++ts == g.S) {
-          ts = 0;
-          ++tr;
+        uint8_t* sa = smem + s * STAGE;
+        const int ch = gi * g.Cg + tc0;  // first channel: a multiple of 64 (128-byte aligned in fp16)
+        mbar_arrive_expect_tx(&full[s], STAGE);
+        tma_load_2d(smem_u32(sa), &a.a16_map, kt * TC_KT, m0, &full[s]);
+        if (TMAP)
+          tma_load_2d(smem_u32(sa + A_TILE), &a.act_map, ch, (int)p0, &full[s]);
+        else
+          tma_load_im2col_4d(smem_u32(sa + A_TILE), &a.act_map, ch, w0, h0, n0, (uint16_t)ts, (uint16_t)tr, &full[s]);
+        issued = j + 1;
+        tc0 += TC_KT;
+        if (tc0 == g.Cg) {
+          tc0 = 0;
+          if (++ts == g.S) {
+            ts = 0;
+            ++tr;
+          }
         }
-      }
-      if (++kt == a.ktiles) {
-        kt = 0;
-        ++tl;
       }
     }
     if (!ok && !*abort_flag) fail();
@@ -274,7 +279,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     int kt = 0, gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles && ok; ++tl) {
-      for (int grp = 0; grp < g.ng && ok; ++grp, ++gc) {
+      int gi_, m0_, g0, g1;
+      int64_t p0_;
+      item_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi_, m0_, p0_, g0, g1);
+      for (int grp = g0; grp < g1 && ok; ++grp, ++gc) {
         if ((gc & 1) != b) {
           kt += a.kt_per_group;  // the other issuer's group
           continue;
@@ -326,9 +334,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
     int gc = 0;
     bool ok = true;
     for (int tl = 0; tl < my_tiles; ++tl) {
-      int gi, m0;
+      int gi, m0, g0, g1;
       int64_t p0;
-      tile_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0);
+      item_coords(a, (int)blockIdx.x + tl * (int)gridDim.x, gi, m0, p0, g0, g1);
       const int m = m0 + t;
       const bool mok = m < gi * g.Mg + g.Mg && m < g.M;
       const int64_t pbase = p0 + TC_EPI_COLS * half;
@@ -336,12 +344,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
       float acc[TC_EPI_COLS];
 #pragma unroll
       for (int j = 0; j < TC_EPI_COLS; ++j) acc[j] = 0.0f;
-      float al_next = mok ? __ldg(arow) : 0.0f;
-      for (int grp = 0; grp < g.ng; ++grp, ++gc) {
+      float al_next = mok ? __ldg(arow + g0) : 0.0f;
+      for (int grp = g0; grp < g1; ++grp, ++gc) {
         if (!ok) continue;  // after a failed wait: run out the tile, then leave with the others
         const int b = gc & 1;
         const float al = al_next;  // alpha of this group, loaded one group ahead
-        if (mok && grp + 1 < g.ng) al_next = __ldg(arow + grp + 1);
+        if (mok && grp + 1 < g1) al_next = __ldg(arow + grp + 1);
         if (!mbar_wait_or_abort(&acc_full[b], (gc >> 1) & 1, a.wait_limit, abort_flag, a.wait_sleep_ns)) {
           if (!*abort_flag) fail();
           ok = false;
@@ -410,7 +418,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
 #pragma unroll
             for (int hh = 0; hh < 2; ++hh) {
               const int64_t pb = p0 + TC_EPI_COLS * hh + OUT_POS * k;
-              if (pb < g.P) tma_store_2d(&a.out_map, m0, (int)pb, smem_u32(otile + hh * (OUT_POS * TC_BM)));
+              if (pb < g.P) {
+                if (a.ksplit > 1)  // a group range's partial sums: added into the (zeroed) output
+                  tma_reduce_add_2d(&a.out_map, m0, (int)pb, smem_u32(otile + hh * (OUT_POS * TC_BM)));
+                else
+                  tma_store_2d(&a.out_map, m0, (int)pb, smem_u32(otile + hh * (OUT_POS * TC_BM)));
+              }
             }
             bulk_commit();
           }
@@ -430,7 +443,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
 #pragma unroll
         for (int j = 0; j < TC_EPI_COLS; ++j) {
           const int64_t p = pbase + j;
-          if (p < g.P) a.out[p * g.M + m] = sx * acc[j];
+          if (p < g.P) {
+            if (a.ksplit > 1) atomicAdd(a.out + p * g.M + m, sx * acc[j]);
+            else a.out[p * g.M + m] = sx * acc[j];
+          }
         }
       }
     }
@@ -522,9 +538,34 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   a.g = g;
   a.mtiles = (g.Mg + TC_BM - 1) / TC_BM;
   a.ptiles = (int)((g.P + TC_BN - 1) / TC_BN);
-  a.ntiles = g.groups * a.mtiles * a.ptiles;
   a.kt_per_group = g.G / TC_KT;
   a.ktiles = g.ng * a.kt_per_group;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // A layer with fewer tiles than SMs and a long reduction (at least 64 K-tiles: 4096
+  // products per output) splits each tile's groups into ranges of at least two groups whose
+  // partial sums are added into the zeroed output (fp32 adds in L2), taking the count that
+  // fills the device best (each count by more than 5% over the fewer ranges before it).
+  // Shorter reductions lose more to zeroing the output and adding the partial sums than
+  // they gain; outputs that are requantized or group sums keep whole tiles.
+  const int tiles = g.groups * a.mtiles * a.ptiles;
+  int ksplit = 1;
+  if (tiles < sms && a.ktiles >= 64 && !sums && !g.rq_out) {
+    double best = (double)tiles / sms;
+    for (int k = 2; k <= debug_max_ksplit() && k <= g.ng / 2; ++k) {
+      const int64_t items = (int64_t)tiles * k, waves = (items + sms - 1) / sms;
+      const double eff = (double)items / (double)(waves * sms);
+      if (eff > best * 1.05) {
+        best = eff;
+        ksplit = k;
+      }
+    }
+  }
+  a.gpk = (g.ng + ksplit - 1) / ksplit;
+  a.ksplit = (g.ng + a.gpk - 1) / a.gpk;  // every range non-empty
+  a.ntiles = tiles * a.ksplit;
+  note_ksplit(a.ksplit);
   // a test may shorten the waits (debug_wait_limit_us), never the final drains
   const int64_t lim_us = debug_wait_limit_us();
   a.wait_limit = lim_us < 0 ? TC_WAIT_LIMIT : (uint32_t)(lim_us / 20 + 1);
@@ -575,9 +616,8 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
                             (uint64_t)g.M * 4, TC_BM, OUT_POS, CU_TENSOR_MAP_SWIZZLE_NONE)
                     ? 1
                     : 0;
-  int dev = 0, sms = 148;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (st == FGQ_OK && a.ksplit > 1 && cudaMemsetAsync(out, 0, (size_t)g.P * g.M * sizeof(float), s) != cudaSuccess)
+    st = FGQ_ERR_CUDA;
   const int grid = a.ntiles < sms ? a.ntiles : sms;
   if (st == FGQ_OK)
     st = f8 ? launch_tc_variant<true>(a, sums != nullptr, grid, s) : launch_tc_variant<false>(a, sums != nullptr, grid, s);

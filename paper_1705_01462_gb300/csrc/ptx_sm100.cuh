@@ -359,6 +359,14 @@ __device__ __forceinline__ void tma_store_2d(const void* tmap, int c0, int c1, u
                "r"(c0), "r"(c1), "r"(src_smem)
                : "memory");
 }
+// Add a box from shared memory into global memory (fp32 elements of the map), element by
+// element in L2; out-of-range rows/columns of the box are not written.
+__device__ __forceinline__ void tma_reduce_add_2d(const void* tmap, int c0, int c1, uint32_t src_smem) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(c0), "r"(c1), "r"(src_smem)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // All committed bulk stores of this thread have finished reading shared memory.
 __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }

@@ -66,6 +66,8 @@ SIGNATURES = [
     ("fgq_debug_allow_split_fold", _i, [_i]),
     ("fgq_debug_last_cuda_error", _i, [_vp, _sz]),
     ("fgq_debug_cta_pairs", _i, [_i]),
+    ("fgq_debug_max_ksplit", _i, [_i]),
+    ("fgq_debug_last_ksplit", _i, []),
 ]
 
 
@@ -495,6 +497,16 @@ def fgq_debug_allow_split_fold(allow: bool) -> int:
 def fgq_debug_cta_pairs(on: bool) -> int:
     """G = 4 output kernel on CTA pairs or single CTAs (the default) for this thread's calls."""
     return int(lib().fgq_debug_cta_pairs(1 if on else 0))
+
+
+def fgq_debug_max_ksplit(k: int) -> int:
+    """At most k group ranges per G >= 64 tensor-core tile on this thread (1: whole tiles)."""
+    return int(lib().fgq_debug_max_ksplit(int(k)))
+
+
+def fgq_debug_last_ksplit() -> int:
+    """Group ranges per tile of this thread's last G >= 64 tensor-core call."""
+    return int(lib().fgq_debug_last_ksplit())
 
 
 def fgq_debug_last_cuda_error() -> tuple:

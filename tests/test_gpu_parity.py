@@ -329,6 +329,64 @@ def test_tc_gemm_parity(case):
     check_within(gy.cpu().numpy(), y, ym, f"tc gemm {case}")
 
 
+KSPLIT_CASES = [
+    # B, H, W, C, M, R, S, stride, pad, groups, G, act: fewer tiles than SMs, at least 4096
+    # products per output
+    (2, 9, 9, 512, 200, 3, 3, 1, 1, 1, 64, "u8"),     # im2col boxes, ragged P and M tiles
+    (1, 14, 14, 4096, 256, 1, 1, 1, 0, 1, 64, "s8"),  # 1x1: 2D boxes
+    (2, 14, 14, 4096, 128, 1, 1, 2, 0, 1, 64, "u8"),  # strided 1x1: gathered rows
+    (1, 8, 8, 1024, 128, 3, 3, 1, 1, 2, 64, "u8"),    # conv groups = 2: fp32 atomics, no output map
+    (1, 9, 9, 512, 66, 3, 3, 1, 1, 1, 64, "u8"),      # M % 4 != 0: fp32 atomics
+    (2, 7, 7, 512, 128, 3, 3, 1, 1, 1, 128, "u4"),    # e4m3 operands, two K-tiles per group
+    (1, 7, 7, 576, 64, 3, 3, 1, 1, 1, 64, "s4"),      # ng = 81: ranges of unequal length
+]
+
+
+@pytest.mark.parametrize("case", KSPLIT_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_tc_group_range_split(case):
+    """A few-tile layer split into group ranges whose partial sums are added into the output:
+    within the contraction tolerance of the oracle, and of the whole-tile result (the same
+    sum in another fp32 order)."""
+    B, H, W, C, M, R, S, stride, pad, groups, G, act = case
+    rng = np.random.default_rng(zlib.crc32(repr(case).encode()) + 2)
+    Cg = C // groups
+    w = (rng.standard_normal((M, R * S * Cg)) * np.sqrt(2.0 / (R * S * Cg))).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((B, H, W, C), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.conv2d(q, sc, R, S, stride, pad, groups, t, al, G)
+    args = (to_dev(packed), act, to_dev(np.array([sc], np.float32)), B, H, W, C, R, S, stride, pad, groups,
+            to_dev(codes.view(np.int32)), to_dev(al), M, G)
+    fgq.fgq_set_path(fgq.PATH_TC)
+    split = fgq.fgq_conv2d(*args).cpu().numpy()
+    assert fgq.fgq_last_path() == fgq.PATH_TC and fgq.fgq_debug_last_ksplit() > 1
+    prev = fgq.fgq_debug_max_ksplit(1)
+    try:
+        whole = fgq.fgq_conv2d(*args).cpu().numpy()
+        assert fgq.fgq_debug_last_ksplit() == 1
+    finally:
+        fgq.fgq_debug_max_ksplit(prev)
+    check_within(split, y, ym, f"tc conv2d split {case}")
+    check_within(whole, y, ym, f"tc conv2d whole {case}")
+    check_within(split, whole.astype(np.float64), ym, f"split vs whole {case}")
+
+
+def test_tc_gemm_group_range_split():
+    """One-tile GEMM (a fully connected layer at small batch) over 8 group ranges."""
+    P, K, M, G, act = 60, 4096, 128, 64, "u8"
+    rng = np.random.default_rng(4096)
+    w = rng.standard_normal((M, K)).astype(np.float32)
+    t, al, codes = make_codes(w, G)
+    x = random_acts((P, K), act, rng)
+    q, sc, packed = quantize_oracle(x, act)
+    y, ym = O.gemm(q, sc, t, al, G)
+    fgq.fgq_set_path(fgq.PATH_TC)
+    gy = fgq.fgq_gemm(to_dev(packed), act, to_dev(np.array([sc], np.float32)), P, K, to_dev(codes.view(np.int32)),
+                      to_dev(al), M, G)
+    assert fgq.fgq_last_path() == fgq.PATH_TC and fgq.fgq_debug_last_ksplit() == 8
+    check_within(gy.cpu().numpy(), y, ym, "tc gemm split")
+
+
 def test_tc_forced_on_unsupported_shape():
     """A forced tensor-core path on a shape it cannot run returns FGQ_ERR_UNSUPPORTED."""
     fgq.fgq_set_path(fgq.PATH_TC)
