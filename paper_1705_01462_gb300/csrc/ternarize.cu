@@ -89,59 +89,127 @@ __device__ __forceinline__ bool in_window(uint32_t m, int F) {
   return m != 0 && (f ? f : 1) >= F - 8;
 }
 
-// Solve one group held in registers (G <= 16).  Writes alpha and returns the 2G code bits.
-template <int G>
-__device__ __forceinline__ uint32_t solve_group_regs(const float (&v)[G], float& alpha, bool& bad) {
-  uint32_t mag[G];
-  uint32_t s[G];
-  bad = false;
+// Magnitude bits sorted in descending order in registers by Batcher's odd-even merge
+// network (N a power of two; 543 comparators for N = 64).
+template <int N>
+__device__ __forceinline__ void sort_desc(uint32_t (&s)[N]) {
+  // stage (p, k) compares x with x + k where x - k % p lies in the first half of a block of
+  // 2k and both lie in one block of 2p; the loops have constant trip counts so that the
+  // network unrolls into register operations
 #pragma unroll
-  for (int i = 0; i < G; ++i) {
-    mag[i] = __float_as_uint(v[i]) & 0x7fffffffu;
-    bad |= mag[i] >= 0x7f800000u;
-    s[i] = mag[i];
-  }
-  alpha = 0.0f;
-  if (bad) return 0;
-  // bitonic sort, descending
+  for (int p = 1; p < N; p <<= 1) {
 #pragma unroll
-  for (int size = 2; size <= G; size <<= 1) {
+    for (int k = p; k >= 1; k >>= 1) {
 #pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        if ((i & stride) == 0) {
-          const bool desc = (i & size) == 0;
-          const uint32_t a = s[i], b = s[i + stride];
-          const uint32_t mx = a > b ? a : b, mn = a > b ? b : a;
-          s[i] = desc ? mx : mn;
-          s[i + stride] = desc ? mn : mx;
+      for (int x = 0; x < N; ++x) {
+        const int r = k % p;
+        if (x >= r && x + k < N && (x - r) % (2 * k) < k && x / (2 * p) == (x + k) / (2 * p)) {
+          const uint32_t a = s[x], b = s[x + k];
+          s[x] = a > b ? a : b;
+          s[x + k] = a > b ? b : a;
         }
       }
     }
   }
-  if (s[0] == 0) return 0;
-  const int F = max((int)(s[0] >> 23), 1);
-  uint64_t S = 0, bS = 0;
-  uint32_t bk = 0, tau = 0;
-#pragma unroll
-  for (int i = 0; i < G; ++i) {
-    S += fixed_of(s[i], F);
-    const bool run_end = (i == G - 1) || (s[(i + 1) < G ? i + 1 : i] < s[i]);
-    if (run_end && in_window(s[i], F)) {
-      // candidates come in increasing k, so a strict comparison keeps the smaller k on ties
-      if (bk == 0 || j_greater(S, (uint32_t)(i + 1), bS, bk)) {
-        bS = S;
-        bk = (uint32_t)(i + 1);
-        tau = s[i];
-      }
+}
+
+// The search of Eq. 5 over the sorted magnitudes, one element at a time in decreasing
+// order: the best candidate so far (its exact sum bS in units of 2^(F-158), size bk and
+// threshold tau) and fp32 estimates that decide all but near-tie comparisons.
+//
+// Fast form, for a group whose largest exponent F lies in [10, 253]: the window is every
+// magnitude with bits >= wmin = (F - 8) << 23 (all normal), an element's fixed-point value
+// is its significand shifted by its exponent's distance above F - 8, and the estimate fS is
+// the running fp32 sum of the magnitudes scaled by c = 2^(127 - F) (exact scalings; after k
+// adds its relative error is below k 2^-24 <= 2^-17 for k <= 128).  Candidate k's objective
+// fS^2 / k is compared with the best's as fS^2 * bk against bQ * k, bQ = bfS^2 (1 +- 2^-14)
+// kept from the best: each side is within 2^-16.5 of its exact value, so a comparison
+// outside the 2^-14 band is decided correctly by the estimates, and one inside it by the
+// exact 128-bit comparison (strict: a tie keeps the smaller k).  Elements past the window
+// come after every candidate, so what they add to S and fS is never compared.
+struct Eq5Scan {
+  uint64_t S, bS;
+  float fS, bQhi, bQlo, bkf;
+  uint32_t bk, tau;
+};
+
+__device__ __forceinline__ void eq5_init(Eq5Scan& q) {
+  q.S = 0;
+  q.bS = 0;
+  q.fS = 0.0f;
+  q.bQhi = 0.0f;
+  q.bQlo = 0.0f;
+  q.bkf = 0.0f;
+  q.bk = 0;
+  q.tau = 0;
+}
+
+// Element k - 1 (k = 1 .. G) with magnitude bits m; `mn` the next element's bits (0 past
+// the end).  Fast form only.
+__device__ __forceinline__ void eq5_step(Eq5Scan& q, uint32_t m, uint32_t mn, uint32_t k, float kf, int F,
+                                         uint32_t wmin, float c) {
+  const uint32_t sig = (m & 0x7fffffu) | 0x800000u;
+  q.S += (uint64_t)(sig << (((m >> 23) - (uint32_t)(F - 8)) & 31u));
+  q.fS = fmaf(__uint_as_float(m), c, q.fS);
+  if (mn < m && m >= wmin) {  // a threshold between distinct magnitudes, inside the window
+    const float t = q.fS * q.fS;
+    const float lhs = t * q.bkf;
+    bool take;
+    if (q.bk == 0 || lhs > q.bQhi * kf) take = true;
+    else if (lhs < q.bQlo * kf) take = false;
+    else take = j_greater(q.S, k, q.bS, q.bk);
+    if (take) {
+      q.bS = q.S;
+      q.bk = k;
+      q.bkf = kf;
+      q.tau = m;
+      q.bQhi = t * (1.0f + 0x1p-14f);
+      q.bQlo = t * (1.0f - 0x1p-14f);
     }
   }
-  alpha = round_ratio_f32(bS, bk, F - 158);
+}
+
+// General form (any F, subnormal magnitudes included): exact sums and comparisons only.
+__device__ __forceinline__ void eq5_step_exact(Eq5Scan& q, uint32_t m, uint32_t mn, uint32_t k, int F) {
+  q.S += fixed_of(m, F);
+  if (mn < m && in_window(m, F) && (q.bk == 0 || j_greater(q.S, k, q.bS, q.bk))) {
+    q.bS = q.S;
+    q.bk = k;
+    q.tau = m;
+  }
+}
+
+__device__ __forceinline__ bool eq5_fast(int F) { return F >= 10 && F <= 253; }
+
+__device__ __forceinline__ float eq5_scale(int F) { return __uint_as_float((uint32_t)(254 - F) << 23); }
+
+// Solve one group held in registers (G <= 16).  Writes alpha and returns the 2G code bits.
+template <int G>
+__device__ __forceinline__ uint32_t solve_group_regs(const float (&v)[G], float& alpha, bool& bad) {
+  uint32_t s[G];
+#pragma unroll
+  for (int i = 0; i < G; ++i) s[i] = __float_as_uint(v[i]) & 0x7fffffffu;
+  sort_desc<G>(s);
+  bad = s[0] >= 0x7f800000u;  // the largest magnitude: infinite or NaN if any is
+  alpha = 0.0f;
+  if (bad || s[0] == 0) return 0;
+  const int F = max((int)(s[0] >> 23), 1);
+  Eq5Scan q;
+  eq5_init(q);
+  if (eq5_fast(F)) {
+    const uint32_t wmin = (uint32_t)(F - 8) << 23;
+    const float c = eq5_scale(F);
+#pragma unroll
+    for (int i = 0; i < G; ++i) eq5_step(q, s[i], i + 1 < G ? s[i + 1] : 0u, i + 1, (float)(i + 1), F, wmin, c);
+  } else {
+#pragma unroll
+    for (int i = 0; i < G; ++i) eq5_step_exact(q, s[i], i + 1 < G ? s[i + 1] : 0u, i + 1, F);
+  }
+  alpha = round_ratio_f32(q.bS, q.bk, F - 158);
   uint32_t bits = 0;
 #pragma unroll
   for (int i = 0; i < G; ++i) {
-    if (mag[i] >= tau) bits |= ((__float_as_uint(v[i]) >> 31) ? 3u : 1u) << (2 * i);
+    if ((__float_as_uint(v[i]) & 0x7fffffffu) >= q.tau) bits |= ((__float_as_uint(v[i]) >> 31) ? 3u : 1u) << (2 * i);
   }
   return bits;
 }
@@ -214,93 +282,77 @@ __global__ void __launch_bounds__(256) ternarize_small_kernel(const float* __res
 }
 
 // One group of G in {32, 64} weights (group grp = m ng + g of the layer) solved by one
-// thread: the G magnitudes sorted in registers (bitonic network, descending), then the exact
-// scan of solve_group_regs; the signs for the codes are read again (the group's bytes are
-// still in L1), so only the sorted magnitudes occupy registers.
+// thread: the G magnitudes sorted in registers, then written to the thread's column of
+// shared memory (`col`, stride TG_THREADS words: conflict-free) and scanned there by a
+// rolled loop, which keeps the kernel's code small; the signs for the codes are read again
+// (the group's bytes are still in L1).
+constexpr int TG_THREADS = 128;
+
 template <int G>
 __device__ __forceinline__ void thread_group(const float* __restrict__ w, int Kred, int ng, int wrow,
                                              uint32_t* __restrict__ codes, float* __restrict__ alpha,
-                                             unsigned int* err, int vec4, int64_t grp) {
+                                             unsigned int* err, int vec4, int64_t grp, uint32_t* col) {
   const int m = (int)(grp / ng);
   const int g = (int)(grp - (int64_t)m * ng);
   const float* src = w + (int64_t)m * Kred + (int64_t)g * G;
   const int nvalid = Kred - g * G < G ? Kred - g * G : G;
-  uint32_t s[G];
-  bool bad = false;
-  if (vec4 && nvalid == G) {
-#pragma unroll
-    for (int i = 0; i < G; i += 4) {
-      const float4 f = __ldg(reinterpret_cast<const float4*>(src + i));
-      s[i] = __float_as_uint(f.x) & 0x7fffffffu;
-      s[i + 1] = __float_as_uint(f.y) & 0x7fffffffu;
-      s[i + 2] = __float_as_uint(f.z) & 0x7fffffffu;
-      s[i + 3] = __float_as_uint(f.w) & 0x7fffffffu;
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < G; ++i) s[i] = i < nvalid ? __float_as_uint(__ldg(src + i)) & 0x7fffffffu : 0u;
-  }
-#pragma unroll
-  for (int i = 0; i < G; ++i) bad |= s[i] >= 0x7f800000u;
   uint32_t* crow = codes + (int64_t)m * wrow + g * (G / 16);
-  if (bad) {
-    record_error(err, FGQ_ERR_NONFINITE);
-    alpha[grp] = 0.0f;
+  uint32_t tau;
+  {
+    uint32_t s[G];
+    if (vec4 && nvalid == G) {
 #pragma unroll
-    for (int wd = 0; wd < G / 16; ++wd) crow[wd] = 0u;
-    return;
+      for (int i = 0; i < G; i += 4) {
+        const float4 f = __ldg(reinterpret_cast<const float4*>(src + i));
+        s[i] = __float_as_uint(f.x) & 0x7fffffffu;
+        s[i + 1] = __float_as_uint(f.y) & 0x7fffffffu;
+        s[i + 2] = __float_as_uint(f.z) & 0x7fffffffu;
+        s[i + 3] = __float_as_uint(f.w) & 0x7fffffffu;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < G; ++i) s[i] = i < nvalid ? __float_as_uint(__ldg(src + i)) & 0x7fffffffu : 0u;
+    }
+    sort_desc<G>(s);
+    if (s[0] >= 0x7f800000u) {  // the largest magnitude: infinite or NaN if any is
+      record_error(err, FGQ_ERR_NONFINITE);
+      alpha[grp] = 0.0f;
+#pragma unroll
+      for (int wd = 0; wd < G / 16; ++wd) crow[wd] = 0u;
+      return;
+    }
+#pragma unroll
+    for (int i = 0; i < G; ++i) col[i * TG_THREADS] = s[i];
   }
-  // bitonic sort, descending
-#pragma unroll
-  for (int size = 2; size <= G; size <<= 1) {
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-#pragma unroll
+  const uint32_t top = col[0];
+  Eq5Scan q;
+  eq5_init(q);
+  const int F = max((int)(top >> 23), 1);
+  if (top != 0) {
+    if (eq5_fast(F)) {
+      const uint32_t wmin = (uint32_t)(F - 8) << 23;
+      const float c = eq5_scale(F);
+      uint32_t cur = top;
+      float kf = 1.0f;
+#pragma unroll 4
       for (int i = 0; i < G; ++i) {
-        if ((i & stride) == 0) {
-          const bool desc = (i & size) == 0;
-          const uint32_t a = s[i], b = s[i + stride];
-          const uint32_t mx = a > b ? a : b, mn = a > b ? b : a;
-          s[i] = desc ? mx : mn;
-          s[i + stride] = desc ? mn : mx;
-        }
+        const uint32_t nxt = i + 1 < G ? col[(i + 1) * TG_THREADS] : 0u;
+        eq5_step(q, cur, nxt, (uint32_t)(i + 1), kf, F, wmin, c);
+        cur = nxt;
+        kf += 1.0f;
+      }
+    } else {
+      uint32_t cur = top;
+      for (int i = 0; i < G; ++i) {
+        const uint32_t nxt = i + 1 < G ? col[(i + 1) * TG_THREADS] : 0u;
+        eq5_step_exact(q, cur, nxt, (uint32_t)(i + 1), F);
+        cur = nxt;
       }
     }
   }
-  uint32_t bk = 0, tau = 0;
-  uint64_t bS = 0;
-  float bJ = 0.0f;  // fp32 estimate of the best objective, within 2^-21 of bS^2 / bk
-  int F = 1;
-  if (s[0] != 0) {
-    F = max((int)(s[0] >> 23), 1);
-    uint64_t S = 0;
-#pragma unroll
-    for (int i = 0; i < G; ++i) {
-      S += fixed_of(s[i], F);
-      const bool run_end = (i == G - 1) || (s[(i + 1) < G ? i + 1 : i] < s[i]);
-      if (run_end && in_window(s[i], F)) {
-        // candidates come in increasing k, so a strict comparison keeps the smaller k on ties.
-        // An fp32 estimate (relative error below 2^-21) decides every comparison whose two
-        // objectives differ by more than 2^-14; the rest are decided exactly in 128 bits.
-        const float fS = (float)S;
-        const float J = fS * fS * (1.0f / (float)(i + 1));
-        bool take;
-        if (bk == 0 || J > bJ * (1.0f + 0x1p-14f)) take = true;
-        else if (J < bJ * (1.0f - 0x1p-14f)) take = false;
-        else take = j_greater(S, (uint32_t)(i + 1), bS, bk);
-        if (take) {
-          bS = S;
-          bk = (uint32_t)(i + 1);
-          tau = s[i];
-          bJ = J;
-        }
-      }
-    }
-  }
-  alpha[grp] = bk ? round_ratio_f32(bS, bk, F - 158) : 0.0f;
-  // codes: t = sign(w) where |w| >= tau (tau > 0 whenever anything is kept)
-  const uint32_t thr = bk ? tau : 0xffffffffu;
-#pragma unroll
+  alpha[grp] = q.bk ? round_ratio_f32(q.bS, q.bk, F - 158) : 0.0f;
+  tau = q.bk ? q.tau : 0xffffffffu;  // codes: t = sign(w) where |w| >= tau
+#pragma unroll 1
   for (int wd = 0; wd < G / 16; ++wd) {
     uint32_t b[16];
     if (vec4 && nvalid == G) {
@@ -319,21 +371,22 @@ __device__ __forceinline__ void thread_group(const float* __restrict__ w, int Kr
     uint32_t bits = 0;
 #pragma unroll
     for (int e = 0; e < 16; ++e)
-      if ((b[e] & 0x7fffffffu) >= thr) bits |= ((b[e] >> 31) ? 3u : 1u) << (2 * e);
+      if ((b[e] & 0x7fffffffu) >= tau) bits |= ((b[e] >> 31) ? 3u : 1u) << (2 * e);
     crow[wd] = bits;
   }
 }
 
 // One thread per group for G in {32, 64}.
 template <int G>
-__global__ void __launch_bounds__(128) ternarize_thread_kernel(const float* __restrict__ w, int M, int Kred,
-                                                               int ng, int wrow, uint32_t* __restrict__ codes,
-                                                               float* __restrict__ alpha, unsigned int* err,
-                                                               int vec4) {
+__global__ void __launch_bounds__(TG_THREADS) ternarize_thread_kernel(const float* __restrict__ w, int M, int Kred,
+                                                                      int ng, int wrow, uint32_t* __restrict__ codes,
+                                                                      float* __restrict__ alpha, unsigned int* err,
+                                                                      int vec4) {
+  __shared__ uint32_t sorted[G * TG_THREADS];
   const int64_t total = (int64_t)M * ng;
   for (int64_t grp = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; grp < total;
        grp += (int64_t)gridDim.x * blockDim.x)
-    thread_group<G>(w, Kred, ng, wrow, codes, alpha, err, vec4, grp);
+    thread_group<G>(w, Kred, ng, wrow, codes, alpha, err, vec4, grp, sorted + threadIdx.x);
 }
 
 // One group of G in {32, 64, 128} weights (group grp = m ng + g of the layer) solved by one
@@ -498,33 +551,35 @@ struct TernBatch {
 // library is built with is 13.0).
 static_assert(sizeof(TernBatch) <= 32764, "kernel parameter space");
 
-__device__ __forceinline__ int batch_layer(const TernBatch& b, int64_t i) {
-  int lo = 0, hi = b.n - 1;
-  while (lo < hi) {  // largest l with first <= i
-    const int mid = (lo + hi + 1) >> 1;
-    if (b.l[mid].first <= i) lo = mid;
-    else hi = mid - 1;
-  }
-  return lo;
+// The layer of item i (the last layer whose first item is <= i), searched forward from
+// layer l: each thread visits its items in increasing order.
+__device__ __forceinline__ int batch_layer_from(const TernBatch& b, int l, int64_t i) {
+  while (l + 1 < b.n && b.l[l + 1].first <= i) ++l;
+  return l;
 }
 
 template <int G>
 __global__ void __launch_bounds__(256) ternarize_small_batch_kernel(const __grid_constant__ TernBatch b,
                                                                     unsigned int* err) {
+  int l = 0;
   for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < b.total; u += (int64_t)gridDim.x * blockDim.x) {
-    const TernLayer& L = b.l[batch_layer(b, u)];
+    l = batch_layer_from(b, l, u);
+    const TernLayer& L = b.l[l];
     small_unit<G>(L.w, L.Kred, L.ng, L.wrow, reinterpret_cast<uint8_t*>(L.codes), L.alpha, err, L.vec4,
                   L.units_per_row, u - L.first);
   }
 }
 
 template <int G>
-__global__ void __launch_bounds__(128) ternarize_thread_batch_kernel(const __grid_constant__ TernBatch b,
-                                                                     unsigned int* err) {
+__global__ void __launch_bounds__(TG_THREADS) ternarize_thread_batch_kernel(const __grid_constant__ TernBatch b,
+                                                                            unsigned int* err) {
+  __shared__ uint32_t sorted[G * TG_THREADS];
+  int l = 0;
   for (int64_t grp = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; grp < b.total;
        grp += (int64_t)gridDim.x * blockDim.x) {
-    const TernLayer& L = b.l[batch_layer(b, grp)];
-    thread_group<G>(L.w, L.Kred, L.ng, L.wrow, L.codes, L.alpha, err, L.vec4, grp - L.first);
+    l = batch_layer_from(b, l, grp);
+    const TernLayer& L = b.l[l];
+    thread_group<G>(L.w, L.Kred, L.ng, L.wrow, L.codes, L.alpha, err, L.vec4, grp - L.first, sorted + threadIdx.x);
   }
 }
 
@@ -534,8 +589,10 @@ __global__ void __launch_bounds__(256) ternarize_warp_batch_kernel(const __grid_
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  int l = 0;
   for (int64_t grp = warp0; grp < b.total; grp += nwarps) {
-    const TernLayer& L = b.l[batch_layer(b, grp)];
+    l = batch_layer_from(b, l, grp);
+    const TernLayer& L = b.l[l];
     warp_group<G>(L.w, L.Kred, L.ng, L.wrow, L.codes, L.alpha, err, grp - L.first, lane);
   }
 }
@@ -610,8 +667,8 @@ fgq_status launch_ternarize(const float* w, int M, int Kred, int G, uint32_t* co
     case 4: ternarize_small_kernel<4><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
     case 8: ternarize_small_kernel<8><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
     case 16: ternarize_small_kernel<16><<<grid_for(units, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, cb, alpha, err, vec4); break;
-    case 32: ternarize_thread_kernel<32><<<grid_for((int64_t)M * ng, 128), 128, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
-    case 64: ternarize_thread_kernel<64><<<grid_for((int64_t)M * ng, 128), 128, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
+    case 32: ternarize_thread_kernel<32><<<grid_for((int64_t)M * ng, TG_THREADS), TG_THREADS, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
+    case 64: ternarize_thread_kernel<64><<<grid_for((int64_t)M * ng, TG_THREADS), TG_THREADS, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err, vec4); break;
     case 128: ternarize_warp_kernel<128><<<grid_for((int64_t)M * ng * 32, threads), threads, 0, s>>>(w, M, Kred, ng, wrow, codes, alpha, err); break;
     default: return FGQ_ERR_ARG;
   }
@@ -648,8 +705,8 @@ fgq_status launch_ternarize_batch(int n, const float* const* w, const int* M, co
     case 4: ternarize_small_batch_kernel<4><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
     case 8: ternarize_small_batch_kernel<8><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
     case 16: ternarize_small_batch_kernel<16><<<grid_for(total, threads), threads, 0, s>>>(b, err); break;
-    case 32: ternarize_thread_batch_kernel<32><<<grid_for(total, 128), 128, 0, s>>>(b, err); break;
-    case 64: ternarize_thread_batch_kernel<64><<<grid_for(total, 128), 128, 0, s>>>(b, err); break;
+    case 32: ternarize_thread_batch_kernel<32><<<grid_for(total, TG_THREADS), TG_THREADS, 0, s>>>(b, err); break;
+    case 64: ternarize_thread_batch_kernel<64><<<grid_for(total, TG_THREADS), TG_THREADS, 0, s>>>(b, err); break;
     case 128: ternarize_warp_batch_kernel<128><<<grid_for(total * 32, threads), threads, 0, s>>>(b, err); break;
     default: return FGQ_ERR_ARG;
   }
