@@ -190,6 +190,13 @@ fgq_status after_launch() {
   return FGQ_ERR_CUDA;
 }
 
+fgq_status after_launch(cudaError_t launch_result) {
+  const fgq_status st = after_launch();
+  if (launch_result == cudaSuccess) return st;
+  t_last_cuda_error = (int)launch_result;
+  return FGQ_ERR_CUDA;
+}
+
 int64_t debug_wait_limit_us() { return t_wait_limit_us; }
 
 bool debug_cta_pairs() { return t_cta_pairs != 0; }

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <utility>
 
 #include "fgq_internal.h"
 
@@ -98,6 +99,31 @@ __device__ __forceinline__ uint8_t rq_code(float v, const RqMul& r) {
   int x = __float2int_rn(v * r.m1 * r.m2);
   x = max(r.qmin, min(r.qmax, x));
   return (uint8_t)(x & 0xff);
+}
+
+// Programmatic dependent launch: a kernel launched by launch_pdl may be scheduled while the
+// kernel before it on the stream is still running (once every block of that kernel has
+// called pdl_trigger or exited).  It must call pdl_wait -- which returns when the previous
+// kernel has completed and its memory operations are visible -- before it reads or writes
+// any global memory; what comes before (barrier initialisation, tensor-memory allocation,
+// descriptor prefetch) overlaps the previous kernel's tail.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 }  // namespace fgq

@@ -32,6 +32,7 @@ unsigned int* device_error_word();
 
 // Counts one kernel launch (for fgq_launch_count) and converts a launch error.
 fgq_status after_launch();
+fgq_status after_launch(cudaError_t launch_result);  // the result of a cudaLaunchKernelEx
 
 // Wait limit, in microseconds, that a test set on this host thread for the tensor-core
 // kernels' mbarrier waits (fgq_debug_set_wait_limit_us), or -1 for the kernels' own limits.

@@ -145,6 +145,8 @@ template <bool F8>
 __global__ void __launch_bounds__(256) prep64_kernel(const uint32_t* __restrict__ codes, int64_t nwords,
                                                      uint4* __restrict__ a_op, const prep::ActSrc src,
                                                      uint4* __restrict__ x_op, int code_blocks) {
+  pdl_wait();
+  pdl_trigger();
   if ((int)blockIdx.x < code_blocks) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nwords; i += (int64_t)code_blocks * blockDim.x) {
       if (F8) prep::codes_e4m3(codes, i, a_op);
@@ -206,6 +208,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) tc_contract_kernel(const __grid
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the prologue above overlapped the previous kernel; global memory only from here on
+  pdl_wait();
+  pdl_trigger();
   const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
 
   auto fail = [&]() {
@@ -465,8 +470,7 @@ template <bool TMAP, bool SUMS, bool F8>
 fgq_status launch_tc(const TcArgs& args, int grid, cudaStream_t s) {
   constexpr int smem = TcCfg<F8>::SMEM;
   if (!tc::smem_attr_once<tc_contract_kernel<TMAP, SUMS, F8>>(smem)) return FGQ_ERR_CUDA;
-  tc_contract_kernel<TMAP, SUMS, F8><<<grid, TC_THREADS, smem, s>>>(args);
-  return after_launch();
+  return after_launch(launch_pdl(tc_contract_kernel<TMAP, SUMS, F8>, dim3(grid), dim3(TC_THREADS), smem, s, args));
 }
 
 template <bool F8>
@@ -589,11 +593,11 @@ fgq_status launch_tc_contract(const void* act, const Geom& g, const uint32_t* co
   // both operands in one launch, the blocks split by the two jobs' sizes
   const prep::ActSrc src = prep::act_src(act, g);
   const int cb = prep::blocks_for(nwords), xb = prep::blocks_for(src.nchunks);
-  if (f8)
-    prep64_kernel<true><<<cb + xb, 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16), src, static_cast<uint4*>(x16), cb);
-  else
-    prep64_kernel<false><<<cb + xb, 256, 0, s>>>(codes, nwords, static_cast<uint4*>(a16), src, static_cast<uint4*>(x16), cb);
-  fgq_status st = after_launch();
+  fgq_status st = after_launch(
+      f8 ? launch_pdl(prep64_kernel<true>, dim3(cb + xb), dim3(256), 0, s, codes, nwords, static_cast<uint4*>(a16),
+                          src, static_cast<uint4*>(x16), cb)
+         : launch_pdl(prep64_kernel<false>, dim3(cb + xb), dim3(256), 0, s, codes, nwords, static_cast<uint4*>(a16),
+                          src, static_cast<uint4*>(x16), cb));
   const CUtensorMapDataType dt = f8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
   const CUtensorMapSwizzle sw = f8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
   if (st == FGQ_OK && !make_map_2d(&a.a16_map, dt, a16, (uint64_t)g.wrow * 16, (uint64_t)g.M,

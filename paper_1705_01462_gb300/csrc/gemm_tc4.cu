@@ -138,6 +138,8 @@ __global__ void __launch_bounds__(256) prep4_kernel(const uint32_t* __restrict__
                                                     int Kp, int Mg, int mtiles, int ksplit, uint4* __restrict__ a0,
                                                     uint4* __restrict__ a1, int fold_blocks, const prep::ActSrc src,
                                                     uint4* __restrict__ x16) {
+  pdl_wait();
+  pdl_trigger();
   if ((int)blockIdx.x >= fold_blocks) {
     const int64_t nb = (int64_t)gridDim.x - fold_blocks;
     for (int64_t i = ((int64_t)blockIdx.x - fold_blocks) * blockDim.x + threadIdx.x; i < src.nchunks;
@@ -318,6 +320,9 @@ __global__ void __launch_bounds__(T4_THREADS, 1) tc4_contract_kernel(const __gri
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the prologue above overlapped the previous kernel; global memory only from here on
+  pdl_wait();
+  pdl_trigger();
   const int my_tiles = (a.ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
   const int units_per_tile = FOLD ? a.ktiles : 4 * a.ktiles;  // drains per tile
 
@@ -813,8 +818,7 @@ template <bool TMAP, bool FOLD>
 fgq_status launch_tc4(const T4Args& args, int grid, cudaStream_t s) {
   constexpr int smem = T4Cfg<FOLD>::SMEM;
   if (!tc::smem_attr_once<tc4_contract_kernel<TMAP, FOLD>>(smem)) return FGQ_ERR_CUDA;
-  tc4_contract_kernel<TMAP, FOLD><<<grid, T4_THREADS, smem, s>>>(args);
-  return after_launch();
+  return after_launch(launch_pdl(tc4_contract_kernel<TMAP, FOLD>, dim3(grid), dim3(T4_THREADS), smem, s, args));
 }
 
 // Both operands of a call in one launch: A' (both parts when folded) with the row scales rs,
@@ -825,15 +829,15 @@ fgq_status launch_prep4(const Geom& g, const uint32_t* codes, const float* alpha
   const int fold_blocks = g.groups * mtiles * ksplit;
   const prep::ActSrc src = prep::act_src(act, g);
   const int xb = prep::blocks_for(src.nchunks);
+  const dim3 grid(fold_blocks + xb), block(256);
   if (a1)
-    prep4_kernel<true><<<fold_blocks + xb, 256, 0, s>>>(codes, g.wrow, alpha, g.ng, rs, g.Kp, g.Mg, mtiles, ksplit,
-                                                        static_cast<uint4*>(a0), static_cast<uint4*>(a1), fold_blocks,
-                                                        src, static_cast<uint4*>(x16));
-  else
-    prep4_kernel<false><<<fold_blocks + xb, 256, 0, s>>>(codes, g.wrow, nullptr, g.ng, nullptr, g.Kp, g.Mg, mtiles,
-                                                         ksplit, static_cast<uint4*>(a0), nullptr, fold_blocks, src,
-                                                         static_cast<uint4*>(x16));
-  return after_launch();
+    return after_launch(launch_pdl(prep4_kernel<true>, grid, block, 0, s, codes, g.wrow, alpha, g.ng, rs, g.Kp,
+                                       g.Mg, mtiles, ksplit, static_cast<uint4*>(a0), static_cast<uint4*>(a1),
+                                       fold_blocks, src, static_cast<uint4*>(x16)));
+  return after_launch(launch_pdl(prep4_kernel<false>, grid, block, 0, s, codes, g.wrow,
+                                     static_cast<const float*>(nullptr), g.ng, static_cast<float*>(nullptr), g.Kp, g.Mg,
+                                     mtiles, ksplit, static_cast<uint4*>(a0), static_cast<uint4*>(nullptr), fold_blocks,
+                                     src, static_cast<uint4*>(x16)));
 }
 
 }  // namespace

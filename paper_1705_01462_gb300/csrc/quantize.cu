@@ -480,6 +480,8 @@ struct QPair {
 };
 
 __global__ void __launch_bounds__(kBatchThreads) qab_kernel(const __grid_constant__ QPair p, unsigned int* err) {
+  pdl_wait();  // the previous launch's maxima (and the zeroed words) are complete
+  pdl_trigger();
   const int bx = (int)blockIdx.x;
   if (bx < p.q.nblocks) qab_quant_block(p.q, p.q.nblocks - 1 - bx);
   else qab_max_block(p.m, bx - p.q.nblocks, err);
@@ -499,8 +501,7 @@ fgq_status launch_quantize_batch(int n, const float* const* x, const size_t* nel
     const int64_t blocks = (int64_t)p.q.nblocks + p.m.nblocks;
     if (blocks == 0) return FGQ_OK;
     if (blocks > INT32_MAX) return FGQ_ERR_UNSUPPORTED;
-    qab_kernel<<<(unsigned)blocks, kBatchThreads, 0, s>>>(p, err);
-    return after_launch();
+    return after_launch(launch_pdl(qab_kernel, dim3((unsigned)blocks), dim3(kBatchThreads), 0, s, p, err));
   };
   while (i < n) {
     QBatch& b = p.m;
