@@ -663,6 +663,92 @@ __global__ void __launch_bounds__(256) im2col_rows_kernel(const uint8_t* __restr
 
 size_t im2col_rows_smem(const Geom& g, int Kc) { return (size_t)((g.R * g.W * g.C + 15) & ~15) + 3 * (size_t)Kc; }
 
+// The same im2col rows for S C >= 16, where the 16 consecutive k of a 16-byte piece span at
+// most two filter rows r, each a contiguous run of S C bytes of one input row.  One block per
+// output row (b, ho): the R input rows are staged in shared memory (16-byte loads when the
+// rows allow) at byte padB of a row of RS bytes whose margins stay zero (the padding
+// columns), out-of-image rows all zero.  Piece q of col row wo is the 16-byte window of
+// staged row r0 = 16 q / (S C) from its first element, completed from the window of row
+// r0 + 1; each window is five 32-bit shared loads funnel-shifted to its byte offset, and
+// k >= Kred reads zero.  Guards of IM2COL_SEG_GUARD bytes before and after the rows absorb
+// the windows' reach past a row (those bytes are masked out).
+constexpr int IM2COL_SEG_GUARD = 32;
+
+__host__ __device__ inline int im2col_seg_padb(int pad, int C) { return (pad * C + 15) / 16 * 16; }
+__host__ __device__ inline int im2col_seg_rs(int W, int C, int pad) {
+  return (im2col_seg_padb(pad, C) + (W + pad) * C + 20 + 15) / 16 * 16;
+}
+size_t im2col_seg_smem(const Geom& g) { return 2 * (size_t)IM2COL_SEG_GUARD + (size_t)g.R * im2col_seg_rs(g.W, g.C, g.pad); }
+
+__device__ __forceinline__ void window16(const uint8_t* p, uint32_t (&o)[4]) {
+  const uint32_t* a = reinterpret_cast<const uint32_t*>(reinterpret_cast<uintptr_t>(p) & ~uintptr_t(3));
+  const uint32_t sh = 8u * (uint32_t)(reinterpret_cast<uintptr_t>(p) & 3);
+  uint32_t w[5];
+#pragma unroll
+  for (int i = 0; i < 5; ++i) w[i] = a[i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) o[i] = __funnelshift_r(w[i], w[i + 1], sh);
+}
+
+__device__ __forceinline__ uint32_t low_bytes_mask(int t) {  // the low t bytes (t clamped to 0 .. 4)
+  return t >= 4 ? 0xffffffffu : (t <= 0 ? 0u : (1u << (8 * t)) - 1u);
+}
+
+__global__ void __launch_bounds__(256) im2col_seg_kernel(const uint8_t* __restrict__ act, int H, int W, int C, int R,
+                                                        int S, int stride, int pad, int Ho, int Wo, int Kred,
+                                                        int Kc, uint8_t* __restrict__ col) {
+  extern __shared__ __align__(16) uint8_t sm_seg[];
+  const int padB = im2col_seg_padb(pad, C), RS = im2col_seg_rs(W, C, pad);
+  uint8_t* rows = sm_seg + IM2COL_SEG_GUARD;  // [R][RS]
+  const int ho = blockIdx.x % Ho;
+  const int b = blockIdx.x / Ho;
+  const int h0 = ho * stride - pad;
+  const int rowb = W * C;
+  const int nz16 = (2 * IM2COL_SEG_GUARD + R * RS) / 16;
+  for (int i = threadIdx.x; i < nz16; i += blockDim.x) reinterpret_cast<uint4*>(sm_seg)[i] = make_uint4(0u, 0u, 0u, 0u);
+  __syncthreads();
+  if (rowb % 16 == 0 && (reinterpret_cast<uintptr_t>(act) & 15) == 0) {
+    const int n16 = rowb / 16;
+    for (int i = threadIdx.x; i < R * n16; i += blockDim.x) {
+      const int r = i / n16, e = i - r * n16;
+      const int h = h0 + r;
+      if (h >= 0 && h < H)
+        *reinterpret_cast<uint4*>(rows + r * RS + padB + 16 * e) =
+            __ldg(reinterpret_cast<const uint4*>(act + ((int64_t)b * H + h) * rowb) + e);
+    }
+  } else {
+    for (int i = threadIdx.x; i < R * rowb; i += blockDim.x) {
+      const int r = i / rowb, e = i - r * rowb;
+      const int h = h0 + r;
+      if (h >= 0 && h < H) rows[r * RS + padB + e] = __ldg(act + ((int64_t)b * H + h) * rowb + e);
+    }
+  }
+  __syncthreads();
+  const int SC = S * C;
+  const int cpr = Kc / 16;  // 16-byte pieces per col row
+  uint4* dst = reinterpret_cast<uint4*>(col + ((int64_t)b * Ho + ho) * Wo * Kc);
+  for (int i = threadIdx.x; i < Wo * cpr; i += blockDim.x) {
+    const int wo = i / cpr, q = i - wo * cpr;
+    const int k0 = 16 * q;
+    uint32_t o[4] = {0u, 0u, 0u, 0u};
+    if (k0 < Kred) {
+      const int r0 = k0 / SC, j0 = k0 - r0 * SC;
+      const int n0 = SC - j0 < 16 ? SC - j0 : 16;  // bytes of the piece from filter row r0
+      const int base = padB + (wo * stride - pad) * C;  // byte of filter tap s = 0 in a staged row (>= 0)
+      uint32_t A[4], Bw[4] = {0u, 0u, 0u, 0u};
+      window16(rows + r0 * RS + base + j0, A);
+      if (n0 < 16 && r0 + 1 < R) window16(rows + (r0 + 1) * RS + base - n0, Bw);
+      const int nz = Kred - k0;  // bytes of the piece below Kred
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const uint32_t mA = low_bytes_mask(n0 - 4 * w), mZ = low_bytes_mask(nz - 4 * w);
+        o[w] = ((A[w] & mA) | (Bw[w] & ~mA)) & mZ;
+      }
+    }
+    dst[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
 // 8-bit weights wq [M][Kred] as fp16 [M][Kc] (zero-padded), rs = wscale: exact.
 __global__ void __launch_bounds__(256) fold_w8_kernel(const int8_t* __restrict__ wq, const float* __restrict__ wscale,
                                                       int M, int Kred, int Kc, __half* __restrict__ a0,
@@ -777,8 +863,11 @@ fgq_status launch_dense_w8(const void* act, const Geom& g, const int8_t* wq, con
   uint8_t* col = static_cast<uint8_t*>(tmp);
   __half* a0 = reinterpret_cast<__half*>(col + col_bytes);
   float* rs = reinterpret_cast<float*>(col + col_bytes + a_bytes);
-  const size_t rows_smem = im2col_rows_smem(g, Kc);
-  if (rows_smem <= (size_t)IM2COL_ROWS_SMEM && g.S <= 254 && g.R * g.W * g.C < 65536 &&
+  const size_t rows_smem = im2col_rows_smem(g, Kc), seg_smem = im2col_seg_smem(g);
+  if (g.S * g.C >= 16 && seg_smem <= (size_t)IM2COL_ROWS_SMEM && (int64_t)g.B * g.Ho < INT32_MAX)
+    im2col_seg_kernel<<<(unsigned)((int64_t)g.B * g.Ho), 256, seg_smem, s>>>(
+        static_cast<const uint8_t*>(act), g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
+  else if (rows_smem <= (size_t)IM2COL_ROWS_SMEM && g.S <= 254 && g.R * g.W * g.C < 65536 &&
       (int64_t)g.B * g.Ho < INT32_MAX)
     im2col_rows_kernel<<<(unsigned)((int64_t)g.B * g.Ho), 256, rows_smem, s>>>(
         static_cast<const uint8_t*>(act), g.H, g.W, g.C, g.R, g.S, g.stride, g.pad, g.Ho, g.Wo, g.Kred, Kc, col);
