@@ -154,11 +154,7 @@ __global__ void __launch_bounds__(256) prep64_kernel(const uint32_t* __restrict_
     }
   } else {
     const int64_t nb = (int64_t)gridDim.x - code_blocks;
-    for (int64_t i = ((int64_t)blockIdx.x - code_blocks) * blockDim.x + threadIdx.x; i < src.nchunks;
-         i += nb * blockDim.x) {
-      if (F8) prep::act_e4m3(src, i, x_op);
-      else prep::act_f16(src, i, x_op);
-    }
+    prep::act_expand<F8>(src, ((int64_t)blockIdx.x - code_blocks) * blockDim.x + threadIdx.x, nb * blockDim.x, x_op);
   }
 }
 

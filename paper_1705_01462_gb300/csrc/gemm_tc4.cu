@@ -142,9 +142,7 @@ __global__ void __launch_bounds__(256) prep4_kernel(const uint32_t* __restrict__
   pdl_trigger();
   if ((int)blockIdx.x >= fold_blocks) {
     const int64_t nb = (int64_t)gridDim.x - fold_blocks;
-    for (int64_t i = ((int64_t)blockIdx.x - fold_blocks) * blockDim.x + threadIdx.x; i < src.nchunks;
-         i += nb * blockDim.x)
-      prep::act_f16(src, i, x16);
+    prep::act_expand<false>(src, ((int64_t)blockIdx.x - fold_blocks) * blockDim.x + threadIdx.x, nb * blockDim.x, x16);
     return;
   }
   const int tile = (int)blockIdx.x / ksplit, ks = (int)blockIdx.x - tile * ksplit;

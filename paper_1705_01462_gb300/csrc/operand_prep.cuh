@@ -141,6 +141,52 @@ __device__ __forceinline__ void act_e4m3(const ActSrc& s, int64_t i, uint4* out)
   out[i] = s.sgn ? e4m3x16<true>(v.x, v.y) : e4m3x16<false>(v.x, v.y);
 }
 
+// Expanded chunks first, first + step, ... of the activations (fp16, or e4m3 when F8):
+// four chunks' source loads are issued before any is converted, so that each thread keeps
+// four independent loads in flight (a single load per thread and iteration left these
+// streaming loops bound by the load latency).
+template <bool F8>
+__device__ __forceinline__ void act_expand(const ActSrc& s, int64_t first, int64_t step, uint4* out) {
+  constexpr int U = 4;
+  int64_t i = first;
+  for (; i + (U - 1) * step < s.nchunks; i += U * step) {
+    uint4 v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t src = src_chunk(s, i + u * step);
+      if (s.abits == 8) {
+        v[u] = __ldg(reinterpret_cast<const uint4*>(s.act) + src);
+      } else {
+        const uint2 h = __ldg(reinterpret_cast<const uint2*>(s.act) + src);
+        v[u] = make_uint4(h.x, h.y, 0u, 0u);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t c = i + u * step;
+      if (F8) {
+        out[c] = s.sgn ? e4m3x16<true>(v[u].x, v[u].y) : e4m3x16<false>(v[u].x, v[u].y);
+      } else {
+        uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+        uint4 o0, o1;
+        if (s.abits == 8) {
+          if (s.sgn) f16x16<8, true>(w, o0, o1);
+          else f16x16<8, false>(w, o0, o1);
+        } else {
+          if (s.sgn) f16x16<4, true>(w, o0, o1);
+          else f16x16<4, false>(w, o0, o1);
+        }
+        out[2 * c] = o0;
+        out[2 * c + 1] = o1;
+      }
+    }
+  }
+  for (; i < s.nchunks; i += step) {
+    if (F8) act_e4m3(s, i, out);
+    else act_f16(s, i, out);
+  }
+}
+
 // One code word (16 two-bit codes: 00 = 0, 01 = +1, 11 = -1) as 16 fp16 (32 bytes at
 // out + 2 i) or 16 e4m3 (16 bytes at out + i: 0x00, 0x38, 0xB8).
 __device__ __forceinline__ void codes_f16(const uint32_t* codes, int64_t i, uint4* out) {
@@ -173,13 +219,14 @@ __device__ __forceinline__ void codes_e4m3(const uint32_t* codes, int64_t i, uin
   out[i] = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-// Blocks of 256 threads for n work items: enough to fill the device, each thread looping.
+// Blocks of 256 threads for n work items: up to a full device (8 blocks of 256 threads per
+// SM), each thread looping.
 inline int blocks_for(int64_t n) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t want = (n + 255) / 256;
-  return (int)(want < 4LL * sms ? (want > 0 ? want : 1) : 4LL * sms);
+  return (int)(want < 8LL * sms ? (want > 0 ? want : 1) : 8LL * sms);
 }
 
 }  // namespace prep
