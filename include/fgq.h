@@ -154,9 +154,10 @@ size_t fgq_quantize_act_batch_workspace_bytes(int n);
  * fp32 [1]), with the results (bit for bit), layouts and non-finite handling of
  * fgq_quantize_act.  x, nelem, type, q, scale_out are HOST arrays of n entries holding device
  * pointers, sizes and types (read during the call, not kept); tensors with nelem[i] == 0 are
- * skipped.  The tensors are processed in order in chunks of up to 64 MB of input (a larger
- * tensor forms its own chunk), two kernel launches per chunk (the maxima, then the codes),
- * so the second pass reads what the first left in the L2.  workspace: device scratch of
+ * skipped.  The tensors are processed in order in chunks of up to 48 MB of input (a larger
+ * tensor forms its own chunk); launch k reduces chunk k to its maxima and quantizes chunk
+ * k - 1 (one launch more than there are chunks), so the second pass over a chunk follows the
+ * first closely enough to find much of it in the L2.  workspace: device scratch of
  * fgq_quantize_act_batch_workspace_bytes(n) bytes, 4-byte aligned (its contents on entry
  * do not matter).  The outputs must not overlap the inputs or one another.
  * Errors: FGQ_ERR_ARG (n < 0 or n > FGQ_QUANTIZE_BATCH_MAX, a null array or pointer, a bad
