@@ -694,16 +694,38 @@ __device__ __forceinline__ uint32_t low_bytes_mask(int t) {  // the low t bytes 
   return t >= 4 ? 0xffffffffu : (t <= 0 ? 0u : (1u << (8 * t)) - 1u);
 }
 
+// __byte_perm selector taking bytes [0, t) of a and the rest of b (t clamped to 0 .. 4).
+__device__ __forceinline__ uint32_t merge_sel(int t) {
+  t = t < 0 ? 0 : (t > 4 ? 4 : t);
+  return 0x7654u - (0x4444u & ((1u << (4 * t)) - 1u));
+}
+
+constexpr int IM2COL_SEG_MAX_CPR = IM2COL_MAX_KC / 16;
+
 __global__ void __launch_bounds__(256) im2col_seg_kernel(const uint8_t* __restrict__ act, int H, int W, int C, int R,
                                                         int S, int stride, int pad, int Ho, int Wo, int Kred,
                                                         int Kc, uint8_t* __restrict__ col) {
   extern __shared__ __align__(16) uint8_t sm_seg[];
+  // per piece q of a col row (the same for every row): the offsets of its two windows from the
+  // row's tap-0 byte, and n0 | nz << 8 (bytes from filter row r0; bytes below Kred)
+  __shared__ int tab_a[IM2COL_SEG_MAX_CPR], tab_b[IM2COL_SEG_MAX_CPR], tab_n[IM2COL_SEG_MAX_CPR];
   const int padB = im2col_seg_padb(pad, C), RS = im2col_seg_rs(W, C, pad);
   uint8_t* rows = sm_seg + IM2COL_SEG_GUARD;  // [R][RS]
   const int ho = blockIdx.x % Ho;
   const int b = blockIdx.x / Ho;
   const int h0 = ho * stride - pad;
   const int rowb = W * C;
+  const int SC = S * C;
+  const int cpr = Kc / 16;  // 16-byte pieces per col row
+  for (int q = threadIdx.x; q < cpr; q += blockDim.x) {
+    const int k0 = 16 * q;
+    const int r0 = k0 / SC, j0 = k0 - r0 * SC;
+    const int n0 = SC - j0 < 16 ? SC - j0 : 16;
+    const int nz = k0 >= Kred ? 0 : (Kred - k0 < 16 ? Kred - k0 : 16);
+    tab_a[q] = r0 * RS + j0;
+    tab_b[q] = (n0 < 16 && r0 + 1 < R) ? (r0 + 1) * RS - n0 : -1;
+    tab_n[q] = n0 | (nz << 8);
+  }
   const int nz16 = (2 * IM2COL_SEG_GUARD + R * RS) / 16;
   for (int i = threadIdx.x; i < nz16; i += blockDim.x) reinterpret_cast<uint4*>(sm_seg)[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncthreads();
@@ -724,28 +746,34 @@ __global__ void __launch_bounds__(256) im2col_seg_kernel(const uint8_t* __restri
     }
   }
   __syncthreads();
-  const int SC = S * C;
-  const int cpr = Kc / 16;  // 16-byte pieces per col row
   uint4* dst = reinterpret_cast<uint4*>(col + ((int64_t)b * Ho + ho) * Wo * Kc);
+  // piece i = wo cpr + q, advanced by blockDim pieces without a division per piece
+  const int dwo = (int)blockDim.x / cpr, dq = (int)blockDim.x - dwo * cpr;
+  int wo = (int)threadIdx.x / cpr, q = (int)threadIdx.x - wo * cpr;
   for (int i = threadIdx.x; i < Wo * cpr; i += blockDim.x) {
-    const int wo = i / cpr, q = i - wo * cpr;
-    const int k0 = 16 * q;
+    const int tn = tab_n[q];
+    const int n0 = tn & 0xff, nz = tn >> 8;
     uint32_t o[4] = {0u, 0u, 0u, 0u};
-    if (k0 < Kred) {
-      const int r0 = k0 / SC, j0 = k0 - r0 * SC;
-      const int n0 = SC - j0 < 16 ? SC - j0 : 16;  // bytes of the piece from filter row r0
-      const int base = padB + (wo * stride - pad) * C;  // byte of filter tap s = 0 in a staged row (>= 0)
+    if (nz > 0) {
+      const uint8_t* tap0 = rows + padB + (wo * stride - pad) * C;  // byte of filter tap s = 0 in staged row 0
       uint32_t A[4], Bw[4] = {0u, 0u, 0u, 0u};
-      window16(rows + r0 * RS + base + j0, A);
-      if (n0 < 16 && r0 + 1 < R) window16(rows + (r0 + 1) * RS + base - n0, Bw);
-      const int nz = Kred - k0;  // bytes of the piece below Kred
+      window16(tap0 + tab_a[q], A);
+      const int ob = tab_b[q];
+      if (ob >= 0) window16(tap0 + ob, Bw);
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const uint32_t mA = low_bytes_mask(n0 - 4 * w), mZ = low_bytes_mask(nz - 4 * w);
-        o[w] = ((A[w] & mA) | (Bw[w] & ~mA)) & mZ;
+      for (int w = 0; w < 4; ++w) o[w] = __byte_perm(A[w], Bw[w], merge_sel(n0 - 4 * w));
+      if (nz < 16) {  // the row's last piece below Kred: zero its bytes from nz on
+#pragma unroll
+        for (int w = 0; w < 4; ++w) o[w] &= low_bytes_mask(nz - 4 * w);
       }
     }
     dst[i] = make_uint4(o[0], o[1], o[2], o[3]);
+    wo += dwo;
+    q += dq;
+    if (q >= cpr) {
+      q -= cpr;
+      ++wo;
+    }
   }
 }
 
